@@ -1,0 +1,223 @@
+/*
+ * chimera.h — C ABI of one Chimera draft-and-verify step on one GB300 (sm_103a).
+ *
+ * Chimera (arXiv 2402.15758) speeds up greedy decoding of a Llama-style LLM without
+ * changing its output.  Each step:
+ *   1. drafts K tokens with the lightweight draft model: a trigram encoder
+ *      (eq. "trigram_calculations"), a full-context Transformer block over the base
+ *      model's last hidden states and the trigram states (eq.
+ *      "fullcontext_calculations"), and K residual decoding heads (eq. "residual
+ *      decoding head"), head k predicting word n+2+k from [h_LLM_n ; h_full_{n+1+k}];
+ *   2. expands the per-head top-k tokens into a static candidate tree (Section
+ *      "Inference");
+ *   3. verifies every tree node in one tree-masked forward of the base model
+ *      (Section "Verification");
+ *   4. greedily accepts the longest path whose tokens equal the base model's argmax,
+ *      and compacts the accepted nodes' KV entries into the cache.
+ * The emitted stream equals plain greedy autoregressive decoding (eq. 1, argmax).
+ *
+ * Conventions
+ *   - Every call returns a chimera_status; the message of the last failure is in
+ *     chimera_last_error().  Calls on one context are not thread-safe.
+ *   - Weights are caller-owned DEVICE memory that must outlive the context.
+ *     Matrices are row-major [out][in] (one output feature per row, y = W x).
+ *     dtype 0 = fp32 everywhere; dtype 1 = bf16 weights/activations with fp32
+ *     accumulation and an fp32 residual stream.
+ *   - The context owns the paged KV caches (blocks of 16 positions), the draft KV
+ *     cache, all scratch and the captured CUDA graph of the step.
+ *   - Host buffers are caller-owned host memory.  chimera_step / chimera_generate /
+ *     chimera_prefill return after their work on the context's stream is done.
+ *   - Positions are 0-based.  After prefill of a prompt x[0..n-1] the state is
+ *     (x[0..n], n) where x[n] — the "root" — is the base model's own next token.
+ *     A step emits the root plus the L accepted drafted tokens (1..depth+1 tokens);
+ *     the bonus token (base argmax after the accepted path) becomes the next root.
+ */
+#ifndef CHIMERA_H
+#define CHIMERA_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct chimera_ctx chimera_ctx;
+
+typedef enum {
+  CHIMERA_OK = 0,
+  CHIMERA_EINVAL = -1,     /* bad argument (shape, pointer, token id, batch) */
+  CHIMERA_ENOMEM = -2,     /* device allocation failed */
+  CHIMERA_ECAPACITY = -3,  /* a sequence would exceed max_seq_len KV slots */
+  CHIMERA_ECUDA = -4,      /* a CUDA call or kernel failed */
+  CHIMERA_ETIMEDOUT = -5,  /* a bounded device-side wait gave up */
+  CHIMERA_ESTATE = -6      /* call out of order (e.g. step before prefill) */
+} chimera_status;
+
+/* Model and decoding shapes.  Table 1 of the paper gives layers / hidden size /
+ * heads of the backbones; the draft has one full-context block of the same shape
+ * and n_draft_heads residual heads of shape [vocab][2*d_model]. */
+typedef struct {
+  int n_layers, d_model, n_heads, head_dim, ffn_dim, vocab;
+  int dtype;            /* 0 = fp32, 1 = bf16 */
+  float rms_eps;        /* RMSNorm epsilon (1e-6) */
+  float rope_theta;     /* RoPE base (10000) */
+  int n_draft_heads;    /* K, 1..8 */
+  int tree_nodes;       /* N including the root, 2..64 */
+  int topk[8];          /* rank limit per head (1..8); the tree draws ranks < topk[k] */
+  int max_batch;        /* sequences per context, 1..64 */
+  int max_seq_len;      /* KV slots per sequence (prompt + generated + N tree slots) */
+  int kv_block;         /* must be 16 */
+} chimera_config;
+
+/* One Llama block: RMSNorm gains [d]; wqkv [3d][d] (rows q, then k, then v; head h
+ * at rows h*hd..h*hd+hd-1 of each part); wo [d][d]; w_gate, w_up [F][d]; w_down [d][F]. */
+typedef struct {
+  const void* attn_norm;
+  const void* wqkv;
+  const void* wo;
+  const void* ffn_norm;
+  const void* w_gate;
+  const void* w_up;
+  const void* w_down;
+} chimera_block_weights;
+
+typedef struct {
+  const void* embed;                   /* [V][d] */
+  const chimera_block_weights* layers; /* host array [n_layers] of device pointers */
+  const void* final_norm;              /* [d] */
+  const void* lm_head;                 /* [V][d] */
+  const void* tri_w1;                  /* [d][3d]: W1 of the trigram encoder, input
+                                          [x_{i-2}; x_{i-1}; x_i] */
+  const void* tri_w2;                  /* [d][d]: W2 */
+  chimera_block_weights draft;         /* full-context encoder block */
+  const void* const* heads;            /* host array [K] of [V][2d]: Theta_k, input
+                                          [h_LLM_n ; h_full_{n+1+k}] */
+} chimera_weights;
+
+/* Create a context.  `cuda_stream` is a cudaStream_t (NULL: the context creates its
+ * own non-blocking stream).  Validates shapes, records the weight pointers and
+ * allocates the KV pools (max_batch * max_seq_len slots), scratch and the tree.
+ * EINVAL on bad shapes or a NULL weight, ENOMEM on allocation failure. */
+chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
+                            void* cuda_stream, chimera_ctx** out);
+
+/* Prefill `batch` prompts (host int32, concatenated; lens[b] >= 1 tokens each, ids in
+ * [0, vocab)) with the causal base forward, fill the base and draft KV caches and
+ * set each root to the base model's greedy next token (eq. 1).  Resets any previous
+ * state of the context.  EINVAL / ECAPACITY on bad input. */
+chimera_status chimera_prefill(chimera_ctx* ctx, int batch, const int32_t* tokens,
+                               const int32_t* lens);
+
+/* One draft-and-verify step for every sequence.  out_tokens: host int32
+ * [batch][depth+1] (depth = number of draft heads) receives the emitted tokens of
+ * each sequence (root first); out_count: host int32 [batch] their number (1..depth+1).
+ * ESTATE before prefill, ECAPACITY when n + N + depth + 1 > max_seq_len. */
+chimera_status chimera_step(chimera_ctx* ctx, int32_t* out_tokens, int32_t* out_count);
+
+/* n_steps steps back to back on the device (one synchronisation at the end).
+ * out_tokens: host int32 [batch][n_steps * (depth+1)], each sequence's emitted
+ * tokens packed in order; out_count: host int32 [batch] total emitted per sequence.
+ * Capacity is checked up front for the worst case (every step accepts depth tokens). */
+chimera_status chimera_generate(chimera_ctx* ctx, int n_steps, int32_t* out_tokens,
+                                int32_t* out_count);
+
+/* Enqueue n_steps steps on the context stream and return without synchronising
+ * (no host output; capacity checked for the worst case).  For timing. */
+chimera_status chimera_step_async(chimera_ctx* ctx, int n_steps);
+
+/* Block until the context stream is idle and report device-side errors. */
+chimera_status chimera_sync(chimera_ctx* ctx);
+
+void chimera_free(chimera_ctx* ctx);
+const char* chimera_last_error(const chimera_ctx* ctx);
+
+/* Static tree descriptor (reading of Section "Inference" with Table 4 marginals):
+ * depth[N], parent[N] (-1 for the root), rank[N] (rank drawn from head depth-1),
+ * anc[N] (bit j set iff node j is an ancestor-or-self).  Host outputs of size N. */
+chimera_status chimera_tree(const chimera_ctx* ctx, int32_t* depth, int32_t* parent,
+                            int32_t* rank, uint64_t* anc);
+
+/* Per-kernel timing of one step, launched eagerly with CUDA events around every
+ * launch (test and benchmark hook).  kinds: host int32 [max] kernel class (see
+ * CHIMERA_KIND_*), ms: host float [max], bytes: host double [max] algorithmic HBM
+ * bytes of the launch.  *count receives the number of launches. */
+enum {
+  CHIMERA_KIND_LINEAR = 1,
+  CHIMERA_KIND_ATTENTION = 2,
+  CHIMERA_KIND_NORM = 3,
+  CHIMERA_KIND_ROPE_KV = 4,
+  CHIMERA_KIND_SWIGLU = 5,
+  CHIMERA_KIND_EMBED = 6,
+  CHIMERA_KIND_TOPK = 7,
+  CHIMERA_KIND_ARGMAX = 8,
+  CHIMERA_KIND_TREE = 9,
+  CHIMERA_KIND_ACCEPT = 10,
+  CHIMERA_KIND_COMPACT = 11,
+  CHIMERA_KIND_OTHER = 12
+};
+enum { CHIMERA_PHASE_DRAFT = 0, CHIMERA_PHASE_VERIFY = 1, CHIMERA_PHASE_COMMIT = 2 };
+chimera_status chimera_profile_step(chimera_ctx* ctx, int max, int32_t* kinds, int32_t* phases,
+                                    float* ms, double* bytes, int32_t* count);
+
+/* ---- test hooks (part of the library; used by the parity tests) ---- */
+
+/* Replace the drafted tokens of tree nodes 1..N-1 for the NEXT step only
+ * (node_tokens: host int32 [batch][N], entry 0 ignored; ids in [0, vocab)). */
+chimera_status chimera_debug_override_tree(chimera_ctx* ctx, const int32_t* node_tokens);
+
+/* Replace the root token x[n] of every sequence (host int32 [batch]). */
+chimera_status chimera_debug_set_root(chimera_ctx* ctx, const int32_t* roots);
+
+enum {
+  CHIMERA_DBG_NODE_TOKENS = 1,    /* int32 [batch][N] tree tokens of the last step */
+  CHIMERA_DBG_VERIFY_LOGITS = 2,  /* f32 [batch][N][V] */
+  CHIMERA_DBG_VERIFY_HIDDEN = 3,  /* dtype [batch][N][d] post final norm */
+  CHIMERA_DBG_ARGMAX = 4,         /* int32 [batch][N] */
+  CHIMERA_DBG_PATH = 5,           /* int32 [batch][depth+1] accepted node indices */
+  CHIMERA_DBG_ACCEPT_LEN = 6,     /* int32 [batch] L (drafted tokens accepted) */
+  CHIMERA_DBG_DRAFT_LOGITS = 7,   /* f32 [K][batch][V] residual-head scores */
+  CHIMERA_DBG_TOPK = 8,           /* int32 [batch][K][kmax] */
+  CHIMERA_DBG_HFULL = 9,          /* dtype [K][batch][d] full-context outputs */
+  CHIMERA_DBG_N = 10,             /* int32 [batch] committed length n */
+  CHIMERA_DBG_TOKENS = 11,        /* int32 [batch][max_seq_len + 1] token history */
+  CHIMERA_DBG_PREFILL_LOGITS = 12 /* f32 [batch][V] LM-head scores of the last prompt row
+                                     (valid until the first step) */
+};
+/* Copy a device buffer of the context to host memory; `bytes` must equal its size. */
+chimera_status chimera_debug_read(chimera_ctx* ctx, int what, void* host_dst, size_t bytes);
+
+/* Gather KV rows [pos0, pos0+count) of sequence `seq` from the paged cache of base
+ * layer `layer` (layer = -1: the draft block's cache) into host buffers
+ * k_dst / v_dst of shape [count][H][hd] (dtype of the model). */
+chimera_status chimera_debug_read_kv(chimera_ctx* ctx, int layer, int seq, int pos0, int count,
+                                     void* k_dst, void* v_dst);
+
+/* ---- kernel-level entry points (stateless; for per-kernel parity tests) ---- */
+
+/* Y[M][N] (epilogue)= X[M][K] . W[N][K]^T on the given stream (NULL: default).
+ * dtype 1: X, W bf16 (K, ldx multiples of 8; X, W 16-byte aligned), tcgen05 kernel;
+ * dtype 0: everything fp32.  epi 0: Y = acc, 1: Y = SiLU(acc), 2: Y(fp32) += acc.
+ * out_f32 selects an fp32 Y for epi 0/1 with dtype 1.  Device pointers.  Uses a
+ * per-process workspace allocated on first use. */
+chimera_status chimera_op_linear(int dtype, int epi, int out_f32, int M, int N, int K,
+                                 const void* X, int ldx, const void* W, void* Y, int ldy,
+                                 void* cuda_stream);
+
+/* Tree-masked attention over a paged KV pool [blocks][H][2][16][hd] (device):
+ * q [batch*q_rows][ldq] rotated queries, query i of sequence b at row b*q_rows+i;
+ * n_ctx (device int32 [batch]) committed rows visible to all; n_local rows follow at
+ * slots n_ctx..; query i sees local row j iff bit j of anc[q_local0+i] (device
+ * uint64); page_table device int32 [batch][max_pages]; out [batch*q_rows][ldo].
+ * nq <= 64, n_local <= 64, hd in {64, 128}. */
+chimera_status chimera_op_attention(int dtype, int batch, int n_heads, int head_dim, int nq,
+                                    int q_local0, int n_local, const void* q, int ldq, int q_rows,
+                                    const void* pool, const int32_t* page_table, int max_pages,
+                                    const int32_t* n_ctx, const uint64_t* anc, void* out, int ldo,
+                                    int splits, void* cuda_stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CHIMERA_H */

@@ -1,0 +1,131 @@
+// Host-side launchers of the sm_103a kernels (internal to the library).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace chimera {
+
+// ----------------------------------------------------------------------------
+// bf16 linear on tcgen05: Y[M][N] (epilogue) = X[M][K] . W[N][K]^T
+// ----------------------------------------------------------------------------
+struct TcLinearParams {
+  CUtensorMap tmA;   // W: [N][K] bf16, box 128 x 64, 128-byte swizzle
+  CUtensorMap tmB;   // X: [M][K] bf16 (row pitch ldx), box BN x 64, 128-byte swizzle
+  int M, N, K;
+  int BN;            // token tile = UMMA N (multiple of 16, <= 256)
+  int tok_tiles, feat_tiles, kblocks;
+  long long units;   // feat_tiles * tok_tiles * kblocks
+  int stages;        // smem pipeline depth
+  int epi;           // EPI_*
+  int out_f32;       // Y is fp32 (else bf16) for EPI_STORE / EPI_SILU
+  void* Y;
+  int ldy;
+  float* ws;         // split partials: [grid][2][128 * BN] fp32
+  int* counters;     // [feat_tiles * tok_tiles], all zero between launches
+  int* err;          // device error word
+  uint32_t tmem_cols;
+  uint32_t acc_stride;  // TMEM column distance between the two accumulators
+};
+
+struct TcLinearPlan {
+  TcLinearParams p;
+  int grid = 0;
+  size_t smem = 0;
+  double weight_bytes = 0;  // algorithmic bytes streamed per launch (W once)
+};
+
+// Largest grid of the linear kernel (one CTA per SM) and the workspace it needs.
+int tc_num_sms();
+size_t tc_ws_floats(int max_bn);
+int tc_max_tiles();
+
+// Encode the plan for one call site.  X/W/Y are device pointers; ws/counters are
+// scratch owned by the caller (sizes from tc_ws_floats / tc_max_tiles).
+// Returns 0 on success, otherwise a negative code and a message in `msg`.
+int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, int ldx, const void* W,
+                   void* Y, int ldy, int epi, int out_f32, float* ws, int* counters, int* err,
+                   char* msg, size_t msg_len);
+cudaError_t tc_linear_launch(const TcLinearPlan& plan, cudaStream_t s);
+
+// ----------------------------------------------------------------------------
+// fp32 linear (SIMT, exact fp32 FMA order per output)
+// ----------------------------------------------------------------------------
+cudaError_t f32_linear(int M, int N, int K, const float* X, int ldx, const float* W, float* Y,
+                       int ldy, int epi, cudaStream_t s);
+
+// ----------------------------------------------------------------------------
+// attention over the paged KV cache with a per-query ancestor bitmask
+// ----------------------------------------------------------------------------
+struct AttnParams {
+  const void* q;          // rotated queries, row (b * q_rows + i), head h at col h*hd
+  int ldq, q_rows;
+  int nq;                 // queries per sequence
+  const int* nq_dev;      // optional per-sequence query count (overrides nq when set)
+  int q_local0;           // local row index of query 0 (mask lookup: anc[q_local0 + i])
+  int n_local;            // local rows at slots n..n+n_local-1
+  const int* n_local_dev; // optional per-sequence local count
+  const unsigned long long* anc;  // [q_local0 + nq] ancestor-or-self masks over local rows
+  const void* pool;       // [blocks][H][2][16][hd]
+  long long pool_layer_stride;  // elements between layers (0 for the draft pool)
+  int layer;
+  const int* page_table;  // [B][max_pages]
+  int max_pages;
+  const int* n_ctx;       // [B] committed rows (all visible)
+  void* out;              // [b * q_rows + i][H * hd]
+  int ldo;
+  int B, H, hd;
+  float scale;
+  int splits;             // KV splits per (b, h)
+  float* ws;              // [B][H][splits][nq_max][hd + 2]
+  int* counters;          // [B][H], zero between launches
+  int nq_max;
+};
+cudaError_t attention(const AttnParams& p, int dtype, cudaStream_t s);
+size_t attn_ws_floats(int B, int H, int splits, int nq_max, int hd);
+
+// ----------------------------------------------------------------------------
+// row-wise / small kernels
+// ----------------------------------------------------------------------------
+cudaError_t rmsnorm(int dtype, int in_f32, const void* X, int ldx, const void* g, void* Y, int ldy,
+                    int rows, int d, float eps, cudaStream_t s);
+
+struct RopeKvParams {
+  const void* qkv;   // [rows][ldqkv]
+  int ldqkv;
+  int q_col, k_col, v_col;  // column offsets (q_col < 0: no query output)
+  void* q_out;       // [rows][H*hd]
+  int ldq;
+  void* pool;
+  long long pool_layer_stride;
+  int layer;
+  const int* page_table;
+  int max_pages;
+  const int* n;        // [B]
+  int rows_per_seq;
+  const int* valid;    // optional [B] rows written to the cache
+  int valid_plus;      // valid[b] + valid_plus rows are written (accept length -> path length)
+  int pos_base, slot_base;
+  const int* pos_off;  // optional [rows_per_seq]
+  const float2* rope;  // [max_pos][hd/2] (cos, sin)
+  int max_pos;
+  int B, H, hd;
+  int* err;
+};
+cudaError_t rope_kv(const RopeKvParams& p, int dtype, cudaStream_t s);
+
+cudaError_t swiglu(int dtype, const void* gu, int ldgu, int F, void* h, int ldh, int rows,
+                   cudaStream_t s);
+
+// x[r][:] = E[tok(r)] with tok(r) = tokens[r] (mode 0) or tok_hist[b][n[b]+i] for
+// i < valid[b] and 0 otherwise (mode 1, prefill chunks).
+cudaError_t embed(int dtype, const void* E, int d, int V, float* x, int rows, int rows_per_seq,
+                  const int* tokens, const int* tok_hist, int hist_stride, const int* n,
+                  const int* valid, int* err, cudaStream_t s);
+
+cudaError_t argmax_rows(const float* logits, int V, int rows, int* out, cudaStream_t s);
+cudaError_t topk_rows(const float* logits, int V, int rows, int k, int* idx, float* val,
+                      int out_stride, cudaStream_t s);
+
+}  // namespace chimera

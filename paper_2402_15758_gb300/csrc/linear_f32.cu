@@ -1,0 +1,59 @@
+// fp32 linear for the fp32 model configuration: Y[M][N] (epilogue)= X[M][K] . W[N][K]^T.
+// One warp per output feature streams that weight row once (coalesced) against up to
+// MT token rows; fp32 FMA in a fixed order, then a butterfly sum over the warp.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace chimera {
+namespace {
+
+constexpr int MT = 16;
+constexpr int WARPS = 8;
+
+__global__ void __launch_bounds__(WARPS * 32) f32_linear_kernel(const float* __restrict__ X, int ldx,
+                                                             const float* __restrict__ W,
+                                                             float* __restrict__ Y, int ldy, int M,
+                                                             int N, int K, int epi) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int f = blockIdx.x * WARPS + warp;
+  const int m0 = blockIdx.y * MT;
+  if (f >= N) return;
+  float acc[MT];
+#pragma unroll
+  for (int i = 0; i < MT; ++i) acc[i] = 0.f;
+  const float* w = W + static_cast<size_t>(f) * K;
+  for (int k = lane; k < K; k += 32) {
+    const float wv = w[k];
+#pragma unroll
+    for (int i = 0; i < MT; ++i)
+      if (m0 + i < M) acc[i] = fmaf(wv, X[static_cast<size_t>(m0 + i) * ldx + k], acc[i]);
+  }
+#pragma unroll
+  for (int i = 0; i < MT; ++i) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) acc[i] += __shfl_xor_sync(0xffffffffu, acc[i], o);
+  }
+  if (lane == 0) {
+#pragma unroll
+    for (int i = 0; i < MT; ++i) {
+      const int m = m0 + i;
+      if (m >= M) break;
+      float* y = Y + static_cast<size_t>(m) * ldy + f;
+      if (epi == EPI_RESID)
+        *y += acc[i];
+      else
+        *y = (epi == EPI_SILU) ? silu_f(acc[i]) : acc[i];
+    }
+  }
+}
+
+}  // namespace
+
+cudaError_t f32_linear(int M, int N, int K, const float* X, int ldx, const float* W, float* Y,
+                       int ldy, int epi, cudaStream_t s) {
+  dim3 grid((N + WARPS - 1) / WARPS, (M + MT - 1) / MT);
+  f32_linear_kernel<<<grid, WARPS * 32, 0, s>>>(X, ldx, W, Y, ldy, M, N, K, epi);
+  return cudaGetLastError();
+}
+
+}  // namespace chimera

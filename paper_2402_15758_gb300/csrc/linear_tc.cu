@@ -1,0 +1,400 @@
+// Weight-streaming bf16 linear on the 5th-generation tensor cores (sm_103a).
+//
+//   Y[M][N] (epilogue)= X[M][K] . W[N][K]^T,  fp32 accumulation in tensor memory.
+//
+// Swap-AB: the weight tile (128 output features x 64 K) is the MMA's A operand
+// (UMMA M = 128) and the token tile (BN rows x 64 K, BN = 16..256) is its B operand,
+// so the skinny token dimension of the draft (1..8 rows) and of the tree verify
+// (16..256 rows) becomes the MMA N.  At these sizes the kernel is bound by streaming
+// W from HBM once.
+//
+// Work split: stream-K.  The (feature tile, token tile, K block) units are cut into
+// gridDim.x equal contiguous ranges (one persistent CTA per SM), so every SM streams
+// the same number of weight bytes whatever the matrix shape.  A tile whose K range
+// spans several CTAs is finished by the last CTA to arrive (an atomic counter per
+// tile): every contributor writes its fp32 partial to a workspace slot, and the last
+// one sums the partials in contributor order (deterministic) and runs the epilogue.
+// No CTA ever waits on another.
+//
+// Roles (192 threads): warp 0 issues TMA loads into an n-stage shared-memory ring,
+// warp 1 issues tcgen05.mma into one of two TMEM accumulators, warps 2..5 drain the
+// other accumulator (tcgen05.ld) and run the epilogue, so the loads of the next
+// segment overlap the epilogue of the previous one.
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace chimera {
+namespace {
+
+constexpr int BM = 128;   // weight rows per tile (UMMA M)
+constexpr int BK = 64;    // K per stage: one 128-byte swizzle atom of bf16
+constexpr int UK = 16;    // UMMA K for 16-bit inputs
+constexpr int MAX_STAGES = 12;
+constexpr int THREADS = 192;
+constexpr int PIPE_SMEM = 200 * 1024;
+constexpr int MAX_BN = 256;
+constexpr int MAX_TILES = 8192;
+
+__device__ __forceinline__ int cta_of_unit(long long u, long long U, int G) {
+  return static_cast<int>(((u + 1) * G - 1) / U);
+}
+__device__ __forceinline__ long long unit_begin(int c, long long U, int G) {
+  return static_cast<long long>(c) * U / G;
+}
+
+__device__ __forceinline__ void epi_apply(const TcLinearParams& p, int m, int f, float v) {
+  if (m >= p.M || f >= p.N) return;
+  const size_t idx = static_cast<size_t>(m) * p.ldy + f;
+  if (p.epi == EPI_RESID) {
+    float* y = static_cast<float*>(p.Y);
+    y[idx] += v;
+    return;
+  }
+  if (p.epi == EPI_SILU) v = silu_f(v);
+  if (p.out_f32)
+    static_cast<float*>(p.Y)[idx] = v;
+  else
+    static_cast<bf16*>(p.Y)[idx] = __float2bfloat16_rn(v);
+}
+
+__device__ __forceinline__ bool bar_any(int id, int nthreads, bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred pi, po;\n\t"
+      "setp.ne.u32 pi, %1, 0;\n\t"
+      "bar.red.or.pred po, %2, %3, pi;\n\t"
+      "selp.u32 %0, 1, 0, po;\n\t}"
+      : "=r"(r)
+      : "r"(static_cast<uint32_t>(pred)), "r"(id), "r"(nthreads)
+      : "memory");
+  return r != 0;
+}
+
+__device__ __forceinline__ bool mbar_wait_plain(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
+  const uint64_t t0 = global_timer_ns();
+  while (!mbar_try_wait(bar, parity)) {
+    if (global_timer_ns() - t0 > limit_ns) return false;
+  }
+  return true;
+}
+
+__global__ void __launch_bounds__(THREADS, 1) tc_linear_kernel(const __grid_constant__ TcLinearParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  const int stage_bytes = BM * BK * 2 + p.BN * BK * 2;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + p.stages * stage_bytes);
+  uint64_t* empty = full + MAX_STAGES;
+  uint64_t* tfull = empty + MAX_STAGES;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* drain = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  int* s_abort = reinterpret_cast<int*>(tmem_slot + 1);
+  int* s_last = s_abort + 1;
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < p.stages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&tfull[b], 1);
+      mbar_init(&tempty[b], 128);
+    }
+    mbar_init(drain, 1);
+    *s_abort = 0;
+    *s_last = 0;
+    mbar_fence_init();
+  }
+  if (warp == 0 && lane == 0) {
+    prefetch_tensormap(&p.tmA);
+    prefetch_tensormap(&p.tmB);
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, p.tmem_cols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const long long U = p.units;
+  const int G = gridDim.x;
+  const int cta = blockIdx.x;
+  const long long u_begin = unit_begin(cta, U, G);
+  const long long u_end = unit_begin(cta + 1, U, G);
+  const int KB = p.kblocks;
+  volatile int* abort = s_abort;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer ----------------
+      const uint64_t pol_w = policy_evict_first();
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t issued_mask = 0, issued_par = 0;
+      for (long long u = u_begin; u < u_end && !*abort;) {
+        const int t = static_cast<int>(u / KB);
+        int kb = static_cast<int>(u % KB);
+        const long long seg_end = min(u_end, static_cast<long long>(t + 1) * KB);
+        const int ft = t / p.tok_tiles, tt = t % p.tok_tiles;
+        for (; u < seg_end; ++u, ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1u, abort)) break;
+          uint8_t* sa = smem + stage * stage_bytes;
+          uint8_t* sb = sa + BM * BK * 2;
+          mbar_arrive_expect_tx(&full[stage], static_cast<uint32_t>(stage_bytes));
+          tma_load_2d_hint(sa, &p.tmA, kb * BK, ft * BM, &full[stage], pol_w);
+          tma_load_2d(sb, &p.tmB, kb * BK, tt * p.BN, &full[stage]);
+          issued_mask |= 1u << stage;
+          issued_par = (issued_par & ~(1u << stage)) | (phase << stage);
+          if (++stage == p.stages) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      if (*abort) {
+        // let copies that are still in flight land before the CTA exits
+        for (int s = 0; s < p.stages; ++s)
+          if (issued_mask >> s & 1u) mbar_wait_plain(&full[s], issued_par >> s & 1u, 200000000ull);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------- MMA issuer ----------------
+      const uint32_t idesc = idesc_bf16_m128(p.BN);
+      int stage = 0;
+      uint32_t phase = 0;
+      int buf = 0;
+      uint32_t aphase = 0;
+      for (long long u = u_begin; u < u_end && !*abort;) {
+        const int t = static_cast<int>(u / KB);
+        const long long seg_end = min(u_end, static_cast<long long>(t + 1) * KB);
+        if (!mbar_wait(&tempty[buf], aphase ^ 1u, abort)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + buf * p.acc_stride;
+        bool first = true;
+        for (; u < seg_end; ++u) {
+          if (!mbar_wait(&full[stage], phase, abort)) break;
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + stage * stage_bytes);
+          const uint32_t sb = sa + BM * BK * 2;
+#pragma unroll
+          for (int k = 0; k < BK / UK; ++k) {
+            tc_mma_bf16(d_tmem, sw128_desc(sa + k * 32), sw128_desc(sb + k * 32), idesc,
+                        (first && k == 0) ? 0u : 1u);
+          }
+          first = false;
+          tc_commit(&empty[stage]);
+          if (++stage == p.stages) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        tc_commit(&tfull[buf]);
+        buf ^= 1;
+        if (buf == 0) aphase ^= 1u;
+      }
+      if (*abort) {
+        // every MMA issued so far must complete before TMEM is released
+        tc_commit(drain);
+        mbar_wait_plain(drain, 0, 200000000ull);
+      }
+    }
+  } else {
+    // ---------------- epilogue (warps 2..5, TMEM lanes 32*(warp%4) ..) ----------------
+    const int q = warp & 3;
+    const int row = q * 32 + lane;
+    int buf = 0;
+    uint32_t aphase = 0;
+    for (long long u = u_begin; u < u_end;) {
+      const int t = static_cast<int>(u / KB);
+      const long long seg_end = min(u_end, static_cast<long long>(t + 1) * KB);
+      u = seg_end;
+      const bool ok = mbar_wait(&tfull[buf], aphase, abort);
+      if (bar_any(1, 128, !ok)) break;
+      tc_fence_after();
+      const int ft = t / p.tok_tiles, tt = t % p.tok_tiles;
+      const long long tu0 = static_cast<long long>(t) * KB;
+      const int c_first = cta_of_unit(tu0, U, G);
+      const int c_last = cta_of_unit(tu0 + KB - 1, U, G);
+      const int nparts = c_last - c_first + 1;
+      const int f = ft * BM + row;
+      const int m0 = tt * p.BN;
+      const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + buf * p.acc_stride;
+      if (nparts == 1) {
+        for (int c0 = 0; c0 < p.BN; c0 += 16) {
+          float v[16];
+          tmem_ld_16(tbase + c0, v);
+#pragma unroll
+          for (int j = 0; j < 16; ++j) epi_apply(p, m0 + c0 + j, f, v[j]);
+        }
+        tc_fence_before();
+        mbar_arrive(&tempty[buf]);
+      } else {
+        const int my_slot = 2 * cta + ((u_begin / KB == t) ? 0 : 1);
+        float* wsp = p.ws + static_cast<size_t>(my_slot) * BM * p.BN;
+        for (int c0 = 0; c0 < p.BN; c0 += 16) {
+          float v[16];
+          tmem_ld_16(tbase + c0, v);
+#pragma unroll
+          for (int j = 0; j < 16; ++j) __stcg(&wsp[(c0 + j) * BM + row], v[j]);
+        }
+        tc_fence_before();
+        mbar_arrive(&tempty[buf]);
+        __threadfence();
+        named_bar(1, 128);
+        if (threadIdx.x == 64) {
+          const int old = atomicAdd(&p.counters[t], 1);
+          *s_last = (old == nparts - 1) ? 1 : 0;
+        }
+        named_bar(1, 128);
+        if (*s_last) {
+          __threadfence();
+          for (int col = 0; col < p.BN; ++col) {
+            if (m0 + col >= p.M) break;
+            float acc = 0.f;
+            for (int cc = c_first; cc <= c_last; ++cc) {
+              const int sl = 2 * cc + ((unit_begin(cc, U, G) / KB == t) ? 0 : 1);
+              acc += __ldcg(&p.ws[static_cast<size_t>(sl) * BM * p.BN + col * BM + row]);
+            }
+            epi_apply(p, m0 + col, f, acc);
+          }
+          if (threadIdx.x == 64) p.counters[t] = 0;
+        }
+        named_bar(1, 128);
+      }
+      buf ^= 1;
+      if (buf == 0) aphase ^= 1u;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, p.tmem_cols);
+  }
+  if (threadIdx.x == 0 && *abort) atomicOr(p.err, ERR_TIMEOUT);
+}
+
+// ----------------------------------------------------------------------------
+// host side
+// ----------------------------------------------------------------------------
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(ptr);
+  });
+  return fn;
+}
+
+int encode_2d_bf16(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
+                   uint64_t pitch_elems, uint32_t box_inner, uint32_t box_outer) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return -1;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {pitch_elems * 2};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? 0 : -2;
+}
+
+uint32_t pow2ceil(uint32_t v) {
+  uint32_t r = 1;
+  while (r < v) r <<= 1;
+  return r;
+}
+
+}  // namespace
+
+int tc_num_sms() {
+  int dev = 0, n = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+  return n > 0 ? n : 1;
+}
+
+size_t tc_ws_floats(int max_bn) {
+  return static_cast<size_t>(tc_num_sms()) * 2 * BM * static_cast<size_t>(max_bn);
+}
+
+int tc_max_tiles() { return MAX_TILES; }
+
+int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, int ldx, const void* W,
+                   void* Y, int ldy, int epi, int out_f32, float* ws, int* counters, int* err,
+                   char* msg, size_t msg_len) {
+  auto fail = [&](const char* m) {
+    if (msg && msg_len) snprintf(msg, msg_len, "linear(M=%d,N=%d,K=%d): %s", M, N, K, m);
+    return -1;
+  };
+  if (M < 1 || N < 1 || K < 8) return fail("empty or too-small shape");
+  if (K % 8 != 0 || ldx % 8 != 0) return fail("K and the row pitch of X must be multiples of 8");
+  if (ldx < K || ldy < N) return fail("row pitch smaller than the row");
+  if ((reinterpret_cast<uintptr_t>(X) & 15) || (reinterpret_cast<uintptr_t>(W) & 15))
+    return fail("X and W must be 16-byte aligned");
+  if (epi == EPI_RESID && !out_f32) return fail("residual epilogue needs an fp32 output");
+  TcLinearParams& p = plan->p;
+  memset(&p, 0, sizeof(p));
+  p.M = M;
+  p.N = N;
+  p.K = K;
+  p.BN = M <= MAX_BN ? ((M + 15) / 16) * 16 : MAX_BN;
+  p.tok_tiles = (M + p.BN - 1) / p.BN;
+  p.feat_tiles = (N + BM - 1) / BM;
+  p.kblocks = (K + BK - 1) / BK;
+  if (static_cast<long long>(p.feat_tiles) * p.tok_tiles > MAX_TILES) return fail("too many tiles");
+  p.units = static_cast<long long>(p.feat_tiles) * p.tok_tiles * p.kblocks;
+  const int stage_bytes = BM * BK * 2 + p.BN * BK * 2;
+  p.stages = PIPE_SMEM / stage_bytes;
+  if (p.stages > MAX_STAGES) p.stages = MAX_STAGES;
+  if (p.stages < 2) return fail("token tile too large");
+  p.epi = epi;
+  p.out_f32 = out_f32;
+  p.Y = Y;
+  p.ldy = ldy;
+  p.ws = ws;
+  p.counters = counters;
+  p.err = err;
+  p.acc_stride = pow2ceil(static_cast<uint32_t>(p.BN));
+  p.tmem_cols = pow2ceil(2 * p.acc_stride);
+  if (p.tmem_cols < 32) p.tmem_cols = 32;
+  if (p.tmem_cols > 512) return fail("accumulators exceed tensor memory");
+  if (encode_2d_bf16(&p.tmA, W, K, N, K, BK, BM) != 0) return fail("tensor map of W");
+  if (encode_2d_bf16(&p.tmB, X, K, M, ldx, BK, p.BN) != 0) return fail("tensor map of X");
+  const int sms = tc_num_sms();
+  plan->grid = static_cast<int>(p.units < sms ? p.units : sms);
+  plan->smem = 1024 + static_cast<size_t>(p.stages) * stage_bytes + 2 * MAX_STAGES * 8 + 5 * 8 + 64;
+  plan->weight_bytes = 2.0 * N * K;
+  return 0;
+}
+
+cudaError_t tc_linear_launch(const TcLinearPlan& plan, cudaStream_t s) {
+  static std::once_flag once;
+  std::call_once(once, [] {
+    cudaFuncSetAttribute(tc_linear_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
+  });
+  tc_linear_kernel<<<plan.grid, THREADS, plan.smem, s>>>(plan.p);
+  return cudaGetLastError();
+}
+
+}  // namespace chimera

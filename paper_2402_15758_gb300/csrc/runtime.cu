@@ -1,0 +1,1203 @@
+// Host runtime of the C ABI: context, paged KV allocator, static tree, the launch plan
+// of one step (captured once into a CUDA graph and replayed), prefill, debug hooks and
+// the stateless kernel-level entry points.
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <functional>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "../../include/chimera.h"
+#include "common.cuh"
+#include "kernels.h"
+#include "step_kernels.h"
+
+using namespace chimera;
+
+namespace {
+
+constexpr int CHUNK = 64;        // prefill rows per sequence per pass (one 64-bit mask)
+constexpr int LOG_CAP = 4096;    // per-step accepted-count log
+constexpr int MAX_KMAX = 8;
+
+struct Lin {
+  bool tc = false;
+  TcLinearPlan tp;
+  int M = 0, N = 0, K = 0, ldx = 0, ldy = 0, epi = 0, out_f32 = 0;
+  const void* X = nullptr;
+  const void* W = nullptr;
+  void* Y = nullptr;
+  double bytes = 0;
+};
+
+struct ProfEvent {
+  int kind, phase;
+  double bytes;
+  cudaEvent_t a, b;
+};
+
+// Static tree (reading of Section "Inference"): the N-1 rank tuples with the largest
+// product of per-head marginal top-k accuracies of Table 4 (Chimera rows).
+struct Tree {
+  int n = 0, depth_max = 0;
+  std::vector<int> depth, parent, rank, child_start, child;
+  std::vector<uint64_t> anc;
+};
+
+bool build_tree(const int* topk, int K, int N, Tree* t, std::string* err) {
+  static const int acc[4][5] = {{66, 78, 83, 87, 90}, {49, 55, 60, 68, 75}, {38, 44, 49, 55, 62},
+                                {33, 38, 43, 46, 54}};
+  int marg[4][5];
+  for (int h = 0; h < 4; ++h)
+    for (int r = 0; r < 5; ++r) marg[h][r] = r == 0 ? acc[h][0] : acc[h][r] - acc[h][r - 1];
+  if (K > 4) {
+    *err = "the static tree covers at most 4 draft heads (Table 4)";
+    return false;
+  }
+  struct Cand {
+    long long score;
+    std::vector<int> r;
+  };
+  std::vector<Cand> cands;
+  std::vector<int> cur;
+  // enumerate every rank tuple of depth 1..K with r_i < min(topk[i], 5)
+  std::function<void(int, long long)> rec = [&](int d, long long s) {
+    if (d > 0) {
+      long long sc = s;
+      for (int i = d; i < 4; ++i) sc *= 100;
+      cands.push_back({sc, cur});
+    }
+    if (d == K) return;
+    const int lim = std::min(topk[d], 5);
+    for (int r = 0; r < lim; ++r) {
+      cur.push_back(r);
+      rec(d + 1, s * marg[d][r]);
+      cur.pop_back();
+    }
+  };
+  rec(0, 1);
+  if (static_cast<int>(cands.size()) < N - 1) {
+    *err = "tree_nodes exceeds the number of rank tuples allowed by topk";
+    return false;
+  }
+  std::sort(cands.begin(), cands.end(), [](const Cand& a, const Cand& b) {
+    if (a.score != b.score) return a.score > b.score;
+    if (a.r.size() != b.r.size()) return a.r.size() < b.r.size();
+    return a.r < b.r;
+  });
+  std::vector<std::vector<int>> nodes(1);
+  for (int i = 0; i < N - 1; ++i) nodes.push_back(cands[i].r);
+  std::sort(nodes.begin() + 1, nodes.end(), [](const std::vector<int>& a, const std::vector<int>& b) {
+    if (a.size() != b.size()) return a.size() < b.size();
+    return a < b;
+  });
+  t->n = N;
+  t->depth.assign(N, 0);
+  t->parent.assign(N, -1);
+  t->rank.assign(N, 0);
+  t->anc.assign(N, 0);
+  t->depth_max = 0;
+  for (int i = 1; i < N; ++i) {
+    t->depth[i] = static_cast<int>(nodes[i].size());
+    t->rank[i] = nodes[i].back();
+    std::vector<int> pre(nodes[i].begin(), nodes[i].end() - 1);
+    for (int j = 0; j < i; ++j)
+      if (nodes[j] == pre) t->parent[i] = j;
+    if (t->parent[i] < 0) {
+      *err = "static tree is not prefix-closed";
+      return false;
+    }
+    t->depth_max = std::max(t->depth_max, t->depth[i]);
+  }
+  for (int i = 0; i < N; ++i) {
+    uint64_t m = 0;
+    for (int j = i; j >= 0; j = t->parent[j]) m |= 1ull << j;
+    t->anc[i] = m;
+  }
+  t->child_start.assign(N + 1, 0);
+  t->child.clear();
+  for (int i = 0; i < N; ++i) {
+    t->child_start[i] = static_cast<int>(t->child.size());
+    for (int c = i + 1; c < N; ++c)
+      if (t->parent[c] == i) t->child.push_back(c);
+  }
+  t->child_start[N] = static_cast<int>(t->child.size());
+  if (t->child.empty()) t->child.push_back(0);
+  return true;
+}
+
+}  // namespace
+
+struct chimera_ctx {
+  chimera_config cfg;
+  int L = 0, d = 0, H = 0, hd = 0, F = 0, V = 0, K = 0, N = 0, KMAX = 0, D1 = 0, Bmax = 0, cap = 0;
+  int dtype = 0;
+  size_t esz = 4;
+  cudaStream_t stream = nullptr;
+  bool own_stream = false;
+  int num_sms = 1;
+
+  // weights (device pointers, caller-owned)
+  const void* embed = nullptr;
+  std::vector<chimera_block_weights> layers;
+  chimera_block_weights draft{};
+  const void* final_norm = nullptr;
+  const void* lm_head = nullptr;
+  const void* tri_w1 = nullptr;
+  const void* tri_w2 = nullptr;
+  std::vector<const void*> heads;
+
+  Tree tree;
+  std::vector<uint64_t> chain;
+  int *d_depth = nullptr, *d_rank = nullptr, *d_child_start = nullptr, *d_child = nullptr;
+  unsigned long long *d_anc = nullptr, *d_chain = nullptr;
+
+  // device state
+  int *d_n = nullptr, *d_tok = nullptr, *d_node_tok = nullptr, *d_topk = nullptr, *d_amax = nullptr;
+  int *d_path = nullptr, *d_L = nullptr, *d_bonus = nullptr, *d_ovr = nullptr, *d_ovr_flag = nullptr;
+  int *d_valid = nullptr, *d_last = nullptr, *d_count_log = nullptr, *d_step = nullptr, *d_err = nullptr;
+  float* d_topk_val = nullptr;
+  int tok_stride = 0;
+
+  // KV
+  void* kv = nullptr;
+  void* dkv = nullptr;
+  long long kv_layer_stride = 0;  // elements
+  int NB = 0, max_pages = 0;
+  int* d_pt = nullptr;
+  std::vector<int> h_pt;
+  std::vector<std::vector<int>> seq_blocks;
+  std::vector<int> free_blocks;
+  bool pt_dirty = false;
+  float2* d_rope = nullptr;
+  int max_pos = 0;
+
+  // activations
+  int R = 0;
+  float* x = nullptr;
+  void *xn = nullptr, *qkv = nullptr, *qr = nullptr, *ao = nullptr, *gu = nullptr, *hf = nullptr, *hfin = nullptr;
+  float* logits = nullptr;
+  void *tbuf = nullptr, *ubuf = nullptr, *headin = nullptr, *hfull_log = nullptr, *hsel = nullptr, *kvtmp = nullptr;
+  float *dres = nullptr, *hlog = nullptr;
+
+  // scratch of the split kernels
+  float* lin_ws = nullptr;
+  int* lin_cnt = nullptr;
+  float* att_ws = nullptr;
+  size_t att_ws_floats = 0;
+  int* att_cnt = nullptr;
+
+  // plan of the current batch
+  int batch = 0;
+  std::vector<int> host_n;
+  std::vector<Lin> ver, pre;  // 5 per layer: qkv, wo, gate, up, down
+  Lin ver_lm, pre_lm, pre_dkv, tri1, tri2, dqkv, dwo, dgate, dup, ddown, commit_kv;
+  std::vector<Lin> dhead;
+  int att_splits_ver = 1, att_splits_pre = 1, att_splits_draft = 1;
+  cudaGraphExec_t graph = nullptr;
+  bool prefilled = false;
+  bool ovr_pending = false;
+
+  int* h_stage = nullptr;  // pinned staging
+  size_t h_stage_ints = 0;
+
+  // profiling
+  bool prof = false;
+  std::vector<ProfEvent> prof_ev;
+  size_t prof_used = 0;
+  int cur_phase = 0;
+
+  std::string err;
+  std::vector<void*> allocs;
+};
+
+namespace {
+
+chimera_status fail(chimera_ctx* c, chimera_status st, const std::string& msg) {
+  if (c) c->err = msg;
+  return st;
+}
+
+#define CK(call)                                                                     \
+  do {                                                                               \
+    cudaError_t e_ = (call);                                                         \
+    if (e_ != cudaSuccess)                                                           \
+      return fail(ctx, CHIMERA_ECUDA, std::string(#call) + ": " + cudaGetErrorString(e_)); \
+  } while (0)
+
+template <typename T>
+bool dalloc(chimera_ctx* ctx, T** p, size_t count) {
+  void* q = nullptr;
+  if (count == 0) count = 1;
+  if (cudaMalloc(&q, count * sizeof(T)) != cudaSuccess) return false;
+  ctx->allocs.push_back(q);
+  *p = static_cast<T*>(q);
+  return true;
+}
+bool dalloc_bytes(chimera_ctx* ctx, void** p, size_t bytes) {
+  if (bytes == 0) bytes = 16;
+  if (cudaMalloc(p, bytes) != cudaSuccess) return false;
+  ctx->allocs.push_back(*p);
+  return true;
+}
+
+// ---------------------------------------------------------------------------
+// launch helpers (events around every launch when profiling)
+// ---------------------------------------------------------------------------
+struct Scope {
+  chimera_ctx* c;
+  ProfEvent* ev = nullptr;
+  Scope(chimera_ctx* ctx, int kind, double bytes) : c(ctx) {
+    if (!c->prof) return;
+    if (c->prof_used == c->prof_ev.size()) {
+      ProfEvent e{};
+      cudaEventCreate(&e.a);
+      cudaEventCreate(&e.b);
+      c->prof_ev.push_back(e);
+    }
+    ev = &c->prof_ev[c->prof_used++];
+    ev->kind = kind;
+    ev->phase = c->cur_phase;
+    ev->bytes = bytes;
+    cudaEventRecord(ev->a, c->stream);
+  }
+  ~Scope() {
+    if (ev) cudaEventRecord(ev->b, c->stream);
+  }
+};
+
+cudaError_t run_lin(chimera_ctx* ctx, const Lin& l) {
+  Scope sc(ctx, CHIMERA_KIND_LINEAR, l.bytes);
+  if (l.tc) return tc_linear_launch(l.tp, ctx->stream);
+  return f32_linear(l.M, l.N, l.K, static_cast<const float*>(l.X), l.ldx, static_cast<const float*>(l.W),
+                    static_cast<float*>(l.Y), l.ldy, l.epi, ctx->stream);
+}
+
+bool make_lin(chimera_ctx* ctx, Lin* l, int M, int N, int K, const void* X, int ldx, const void* W, void* Y,
+              int ldy, int epi, int out_f32) {
+  l->M = M;
+  l->N = N;
+  l->K = K;
+  l->X = X;
+  l->ldx = ldx;
+  l->W = W;
+  l->Y = Y;
+  l->ldy = ldy;
+  l->epi = epi;
+  l->out_f32 = out_f32;
+  l->bytes = static_cast<double>(N) * K * ctx->esz;
+  l->tc = ctx->dtype == 1;
+  if (!l->tc) return true;
+  char msg[256];
+  if (tc_linear_plan(&l->tp, M, N, K, X, ldx, W, Y, ldy, epi, out_f32, ctx->lin_ws, ctx->lin_cnt, ctx->d_err, msg,
+                     sizeof(msg)) != 0) {
+    ctx->err = msg;
+    return false;
+  }
+  return true;
+}
+
+int att_splits(const chimera_ctx* ctx, int B) {
+  const int target = 2 * ctx->num_sms;
+  int s = (target + B * ctx->H - 1) / (B * ctx->H);
+  return std::max(1, std::min(16, s));
+}
+
+cudaError_t run_attention(chimera_ctx* ctx, bool draft_pool, int layer, int nq, const int* nq_dev, int q_local0,
+                          int n_local, const int* n_local_dev, const unsigned long long* anc, int q_rows, int splits,
+                          int nq_max, double bytes) {
+  Scope sc(ctx, CHIMERA_KIND_ATTENTION, bytes);
+  AttnParams p{};
+  p.q = ctx->qr;
+  p.ldq = ctx->d;
+  p.q_rows = q_rows;
+  p.nq = nq;
+  p.nq_dev = nq_dev;
+  p.q_local0 = q_local0;
+  p.n_local = n_local;
+  p.n_local_dev = n_local_dev;
+  p.anc = anc;
+  p.pool = draft_pool ? ctx->dkv : ctx->kv;
+  p.pool_layer_stride = draft_pool ? 0 : ctx->kv_layer_stride;
+  p.layer = draft_pool ? 0 : layer;
+  p.page_table = ctx->d_pt;
+  p.max_pages = ctx->max_pages;
+  p.n_ctx = ctx->d_n;
+  p.out = ctx->ao;
+  p.ldo = ctx->d;
+  p.B = ctx->batch;
+  p.H = ctx->H;
+  p.hd = ctx->hd;
+  p.scale = 1.0f / std::sqrt(static_cast<float>(ctx->hd));
+  p.splits = splits;
+  p.ws = ctx->att_ws;
+  p.counters = ctx->att_cnt;
+  p.nq_max = nq_max;
+  if (attn_ws_floats(p.B, p.H, splits, nq_max, p.hd) > ctx->att_ws_floats) return cudaErrorInvalidValue;
+  return attention(p, ctx->dtype, ctx->stream);
+}
+
+cudaError_t run_rope(chimera_ctx* ctx, bool draft_pool, int layer, const void* src, int ldsrc, int q_col, int k_col,
+                     int v_col, int rows_per_seq, const int* valid, int valid_plus, int pos_base, int slot_base,
+                     const int* pos_off) {
+  Scope sc(ctx, CHIMERA_KIND_ROPE_KV, 0);
+  RopeKvParams p{};
+  p.qkv = src;
+  p.ldqkv = ldsrc;
+  p.q_col = q_col;
+  p.k_col = k_col;
+  p.v_col = v_col;
+  p.q_out = ctx->qr;
+  p.ldq = ctx->d;
+  p.pool = draft_pool ? ctx->dkv : ctx->kv;
+  p.pool_layer_stride = draft_pool ? 0 : ctx->kv_layer_stride;
+  p.layer = draft_pool ? 0 : layer;
+  p.page_table = ctx->d_pt;
+  p.max_pages = ctx->max_pages;
+  p.n = ctx->d_n;
+  p.rows_per_seq = rows_per_seq;
+  p.valid = valid;
+  p.valid_plus = valid_plus;
+  p.pos_base = pos_base;
+  p.slot_base = slot_base;
+  p.pos_off = pos_off;
+  p.rope = ctx->d_rope;
+  p.max_pos = ctx->max_pos;
+  p.B = ctx->batch;
+  p.H = ctx->H;
+  p.hd = ctx->hd;
+  p.err = ctx->d_err;
+  return rope_kv(p, ctx->dtype, ctx->stream);
+}
+
+cudaError_t run_norm(chimera_ctx* ctx, int in_f32, const void* X, int ldx, const void* g, void* Y, int ldy,
+                     int rows) {
+  Scope sc(ctx, CHIMERA_KIND_NORM, 0);
+  return rmsnorm(ctx->dtype, in_f32, X, ldx, g, Y, ldy, rows, ctx->d, ctx->cfg.rms_eps, ctx->stream);
+}
+
+#define RUN(call)                                            \
+  do {                                                       \
+    cudaError_t e_ = (call);                                 \
+    if (e_ != cudaSuccess) return e_;                        \
+  } while (0)
+
+char* eoff(const chimera_ctx* ctx, void* base, size_t elems) {
+  return static_cast<char*>(base) + elems * ctx->esz;
+}
+
+// One Llama layer over the rows of `plan` (5 linears), shared by verify and prefill.
+cudaError_t enqueue_layer(chimera_ctx* ctx, int l, const Lin* lin, int rows, int rows_per_seq, const int* valid,
+                          const int* pos_off, const unsigned long long* anc, int splits, double kv_bytes) {
+  const chimera_block_weights& w = ctx->layers[l];
+  const int d = ctx->d;
+  RUN(run_norm(ctx, 1, ctx->x, d, w.attn_norm, ctx->xn, d, rows));
+  RUN(run_lin(ctx, lin[0]));
+  RUN(run_rope(ctx, false, l, ctx->qkv, 3 * d, 0, d, 2 * d, rows_per_seq, valid, 0, 0, 0, pos_off));
+  RUN(run_attention(ctx, false, l, rows_per_seq, valid, 0, rows_per_seq, valid, anc, rows_per_seq, splits,
+                    rows_per_seq, kv_bytes));
+  RUN(run_lin(ctx, lin[1]));
+  RUN(run_norm(ctx, 1, ctx->x, d, w.ffn_norm, ctx->xn, d, rows));
+  RUN(run_lin(ctx, lin[2]));
+  RUN(run_lin(ctx, lin[3]));
+  {
+    Scope sc(ctx, CHIMERA_KIND_SWIGLU, 0);
+    RUN(swiglu(ctx->dtype, ctx->gu, 2 * ctx->F, ctx->F, ctx->hf, ctx->F, rows, ctx->stream));
+  }
+  RUN(run_lin(ctx, lin[4]));
+  return cudaSuccess;
+}
+
+double kv_read_bytes(const chimera_ctx* ctx, int extra_rows, bool draft) {
+  double rows = 0;
+  for (int b = 0; b < ctx->batch; ++b) rows += ctx->host_n[b] + extra_rows;
+  return rows * 2.0 * ctx->d * ctx->esz * (draft ? 1 : 1);
+}
+
+// The whole step on the context stream (graph-capturable: every dynamic value is read
+// from device memory).
+cudaError_t enqueue_step(chimera_ctx* ctx) {
+  const int B = ctx->batch, d = ctx->d, K = ctx->K, N = ctx->N, V = ctx->V, F = ctx->F;
+  cudaStream_t s = ctx->stream;
+  (void)F;
+  // ---- draft: K sequential sub-steps ----
+  ctx->cur_phase = CHIMERA_PHASE_DRAFT;
+  for (int k = 0; k < K; ++k) {
+    {
+      Scope sc(ctx, CHIMERA_KIND_EMBED, 0);
+      RUN(launch_trigram_gather(ctx->dtype, ctx->embed, d, V, ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_topk, K,
+                                ctx->KMAX, k, ctx->tbuf, B, ctx->d_err, s));
+    }
+    RUN(run_lin(ctx, ctx->tri1));
+    RUN(run_lin(ctx, ctx->tri2));
+    RUN(run_norm(ctx, 1, ctx->dres, d, ctx->draft.attn_norm, ctx->xn, d, B));
+    RUN(run_lin(ctx, ctx->dqkv));
+    RUN(run_rope(ctx, true, 0, ctx->qkv, 3 * d, 0, d, 2 * d, 1, nullptr, 0, k, k, nullptr));
+    RUN(run_attention(ctx, true, 0, 1, nullptr, k, k + 1, nullptr, ctx->d_chain, 1, ctx->att_splits_draft, 1,
+                      kv_read_bytes(ctx, k + 1, true)));
+    RUN(run_lin(ctx, ctx->dwo));
+    RUN(run_norm(ctx, 1, ctx->dres, d, ctx->draft.ffn_norm, ctx->xn, d, B));
+    RUN(run_lin(ctx, ctx->dgate));
+    RUN(run_lin(ctx, ctx->dup));
+    {
+      Scope sc(ctx, CHIMERA_KIND_SWIGLU, 0);
+      RUN(swiglu(ctx->dtype, ctx->gu, 2 * ctx->F, ctx->F, ctx->hf, ctx->F, B, s));
+    }
+    RUN(run_lin(ctx, ctx->ddown));
+    {
+      Scope sc(ctx, CHIMERA_KIND_OTHER, 0);
+      RUN(launch_hfull_store(ctx->dtype, ctx->dres, d, ctx->headin, eoff(ctx, ctx->hfull_log, static_cast<size_t>(k) * B * d),
+                             B, s));
+    }
+    RUN(run_lin(ctx, ctx->dhead[k]));
+    {
+      Scope sc(ctx, CHIMERA_KIND_TOPK, 0);
+      RUN(topk_rows(ctx->hlog + static_cast<size_t>(k) * B * V, V, B, ctx->KMAX, ctx->d_topk + k * ctx->KMAX,
+                    ctx->d_topk_val + k * ctx->KMAX, K * ctx->KMAX, s));
+    }
+  }
+  // ---- tree ----
+  ctx->cur_phase = CHIMERA_PHASE_VERIFY;
+  {
+    Scope sc(ctx, CHIMERA_KIND_TREE, 0);
+    RUN(launch_tree_expand(ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_topk, K, ctx->KMAX, ctx->d_depth, ctx->d_rank,
+                           N, ctx->d_ovr_flag, ctx->d_ovr, ctx->d_node_tok, B, s));
+  }
+  // ---- verify: one base forward over every tree node ----
+  {
+    Scope sc(ctx, CHIMERA_KIND_EMBED, 0);
+    RUN(embed(ctx->dtype, ctx->embed, d, V, ctx->x, B * N, N, ctx->d_node_tok, nullptr, 0, nullptr, nullptr,
+              ctx->d_err, s));
+  }
+  const double kvb = kv_read_bytes(ctx, N, false);
+  for (int l = 0; l < ctx->L; ++l)
+    RUN(enqueue_layer(ctx, l, &ctx->ver[5 * l], B * N, N, nullptr, ctx->d_depth, ctx->d_anc, ctx->att_splits_ver, kvb));
+  RUN(run_norm(ctx, 1, ctx->x, d, ctx->final_norm, ctx->hfin, d, B * N));
+  RUN(run_lin(ctx, ctx->ver_lm));
+  {
+    Scope sc(ctx, CHIMERA_KIND_ARGMAX, 0);
+    RUN(argmax_rows(ctx->logits, V, B * N, ctx->d_amax, s));
+  }
+  // ---- accept and commit ----
+  ctx->cur_phase = CHIMERA_PHASE_COMMIT;
+  {
+    Scope sc(ctx, CHIMERA_KIND_ACCEPT, 0);
+    RUN(launch_accept(ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_node_tok, ctx->d_amax, ctx->d_child_start,
+                      ctx->d_child, N, ctx->D1, ctx->d_path, ctx->d_L, ctx->d_bonus, B, s));
+  }
+  {
+    Scope sc(ctx, CHIMERA_KIND_COMPACT, 0);
+    RUN(launch_compact(ctx->kv, ctx->kv_layer_stride * static_cast<long long>(ctx->esz), ctx->L, ctx->H,
+                       static_cast<int>(ctx->hd * ctx->esz), ctx->d_n, ctx->d_path, ctx->d_L, ctx->D1, ctx->d_pt,
+                       ctx->max_pages, B, s));
+  }
+  {
+    Scope sc(ctx, CHIMERA_KIND_OTHER, 0);
+    RUN(launch_gather_hidden(ctx->dtype, ctx->hfin, d, N, ctx->d_path, ctx->d_L, ctx->D1, ctx->hsel, ctx->headin, B, s));
+  }
+  RUN(run_norm(ctx, ctx->dtype == 0 ? 1 : 0, ctx->hsel, d, ctx->draft.attn_norm, ctx->xn, d, B * ctx->D1));
+  RUN(run_lin(ctx, ctx->commit_kv));
+  RUN(run_rope(ctx, true, 0, ctx->kvtmp, 2 * d, -1, 0, d, ctx->D1, ctx->d_L, 1, 0, 0, nullptr));
+  {
+    Scope sc(ctx, CHIMERA_KIND_OTHER, 0);
+    RUN(launch_finalize(ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_L, ctx->d_bonus, ctx->d_count_log, LOG_CAP,
+                        ctx->d_step, B, s));
+  }
+  return cudaSuccess;
+}
+
+// (Re)build every linear call site for `batch` sequences.
+bool build_plans(chimera_ctx* ctx, int B) {
+  const int d = ctx->d, F = ctx->F, V = ctx->V, N = ctx->N;
+  const int f32 = 1, tb = ctx->dtype == 0 ? 1 : 0;  // bf16 storage -> out_f32 = 0
+  ctx->ver.assign(5 * ctx->L, Lin());
+  ctx->pre.assign(5 * ctx->L, Lin());
+  auto layer_plans = [&](std::vector<Lin>& v, int M) {
+    for (int l = 0; l < ctx->L; ++l) {
+      const chimera_block_weights& w = ctx->layers[l];
+      Lin* p = &v[5 * l];
+      if (!make_lin(ctx, &p[0], M, 3 * d, d, ctx->xn, d, w.wqkv, ctx->qkv, 3 * d, EPI_STORE, tb)) return false;
+      if (!make_lin(ctx, &p[1], M, d, d, ctx->ao, d, w.wo, ctx->x, d, EPI_RESID, f32)) return false;
+      if (!make_lin(ctx, &p[2], M, F, d, ctx->xn, d, w.w_gate, ctx->gu, 2 * F, EPI_STORE, tb)) return false;
+      if (!make_lin(ctx, &p[3], M, F, d, ctx->xn, d, w.w_up, eoff(ctx, ctx->gu, F), 2 * F, EPI_STORE, tb)) return false;
+      if (!make_lin(ctx, &p[4], M, d, F, ctx->hf, F, w.w_down, ctx->x, d, EPI_RESID, f32)) return false;
+    }
+    return true;
+  };
+  if (!layer_plans(ctx->ver, B * N)) return false;
+  if (!layer_plans(ctx->pre, B * CHUNK)) return false;
+  if (!make_lin(ctx, &ctx->ver_lm, B * N, V, d, ctx->hfin, d, ctx->lm_head, ctx->logits, V, EPI_STORE, f32)) return false;
+  if (!make_lin(ctx, &ctx->pre_lm, B, V, d, ctx->headin, 2 * d, ctx->lm_head, ctx->logits, V, EPI_STORE, f32)) return false;
+  const void* dl_kv = eoff(ctx, const_cast<void*>(ctx->draft.wqkv), static_cast<size_t>(d) * d);
+  if (!make_lin(ctx, &ctx->pre_dkv, B * CHUNK, 2 * d, d, ctx->xn, d, dl_kv, ctx->kvtmp, 2 * d, EPI_STORE, tb)) return false;
+  if (!make_lin(ctx, &ctx->commit_kv, B * ctx->D1, 2 * d, d, ctx->xn, d, dl_kv, ctx->kvtmp, 2 * d, EPI_STORE, tb))
+    return false;
+  // draft (M = B rows)
+  if (!make_lin(ctx, &ctx->tri1, B, d, 3 * d, ctx->tbuf, 3 * d, ctx->tri_w1, ctx->ubuf, d, EPI_SILU, tb)) return false;
+  if (!make_lin(ctx, &ctx->tri2, B, d, d, ctx->ubuf, d, ctx->tri_w2, ctx->dres, d, EPI_STORE, f32)) return false;
+  const chimera_block_weights& w = ctx->draft;
+  if (!make_lin(ctx, &ctx->dqkv, B, 3 * d, d, ctx->xn, d, w.wqkv, ctx->qkv, 3 * d, EPI_STORE, tb)) return false;
+  if (!make_lin(ctx, &ctx->dwo, B, d, d, ctx->ao, d, w.wo, ctx->dres, d, EPI_RESID, f32)) return false;
+  if (!make_lin(ctx, &ctx->dgate, B, F, d, ctx->xn, d, w.w_gate, ctx->gu, 2 * F, EPI_STORE, tb)) return false;
+  if (!make_lin(ctx, &ctx->dup, B, F, d, ctx->xn, d, w.w_up, eoff(ctx, ctx->gu, F), 2 * F, EPI_STORE, tb)) return false;
+  if (!make_lin(ctx, &ctx->ddown, B, d, F, ctx->hf, F, w.w_down, ctx->dres, d, EPI_RESID, f32)) return false;
+  ctx->dhead.assign(ctx->K, Lin());
+  for (int k = 0; k < ctx->K; ++k)
+    if (!make_lin(ctx, &ctx->dhead[k], B, V, 2 * d, ctx->headin, 2 * d, ctx->heads[k],
+                  ctx->hlog + static_cast<size_t>(k) * B * V, V, EPI_STORE, f32))
+      return false;
+  ctx->att_splits_ver = att_splits(ctx, B);
+  ctx->att_splits_pre = att_splits(ctx, B);
+  ctx->att_splits_draft = att_splits(ctx, B);
+  return true;
+}
+
+chimera_status ensure_blocks(chimera_ctx* ctx, int b, int slots) {
+  if (slots > ctx->cap)
+    return fail(ctx, CHIMERA_ECAPACITY, "sequence " + std::to_string(b) + " needs " + std::to_string(slots) +
+                                            " KV slots > max_seq_len " + std::to_string(ctx->cap));
+  auto& blocks = ctx->seq_blocks[b];
+  while (static_cast<int>(blocks.size()) * 16 < slots) {
+    if (ctx->free_blocks.empty()) return fail(ctx, CHIMERA_ECAPACITY, "KV block pool exhausted");
+    const int blk = ctx->free_blocks.back();
+    ctx->free_blocks.pop_back();
+    ctx->h_pt[b * ctx->max_pages + blocks.size()] = blk;
+    blocks.push_back(blk);
+    ctx->pt_dirty = true;
+  }
+  return CHIMERA_OK;
+}
+
+chimera_status flush_page_table(chimera_ctx* ctx) {
+  if (!ctx->pt_dirty) return CHIMERA_OK;
+  CK(cudaMemcpyAsync(ctx->d_pt, ctx->h_pt.data(), ctx->h_pt.size() * sizeof(int), cudaMemcpyHostToDevice, ctx->stream));
+  CK(cudaStreamSynchronize(ctx->stream));
+  ctx->pt_dirty = false;
+  return CHIMERA_OK;
+}
+
+chimera_status check_err(chimera_ctx* ctx) {
+  int e = 0;
+  CK(cudaMemcpyAsync(&ctx->h_stage[0], ctx->d_err, sizeof(int), cudaMemcpyDeviceToHost, ctx->stream));
+  CK(cudaStreamSynchronize(ctx->stream));
+  e = ctx->h_stage[0];
+  if (e == 0) return CHIMERA_OK;
+  CK(cudaMemsetAsync(ctx->d_err, 0, sizeof(int), ctx->stream));
+  if (e & ERR_TIMEOUT) return fail(ctx, CHIMERA_ETIMEDOUT, "a bounded device wait timed out");
+  if (e & ERR_CAPACITY) return fail(ctx, CHIMERA_ECAPACITY, "a kernel hit the KV capacity bound");
+  return fail(ctx, CHIMERA_EINVAL, "a kernel saw an out-of-range token id or index");
+}
+
+chimera_status steps_prepare(chimera_ctx* ctx, int n_steps) {
+  if (!ctx->prefilled) return fail(ctx, CHIMERA_ESTATE, "step before prefill");
+  const int need = std::max(ctx->N, ctx->K) + 1;
+  for (int b = 0; b < ctx->batch; ++b) {
+    const long long slots = static_cast<long long>(ctx->host_n[b]) + static_cast<long long>(n_steps - 1) * ctx->D1 + need +
+                            ctx->D1;
+    if (slots > ctx->cap)
+      return fail(ctx, CHIMERA_ECAPACITY, "sequence " + std::to_string(b) + " would exceed max_seq_len");
+    chimera_status st = ensure_blocks(ctx, b, static_cast<int>(slots));
+    if (st != CHIMERA_OK) return st;
+  }
+  return flush_page_table(ctx);
+}
+
+chimera_status launch_steps(chimera_ctx* ctx, int n_steps) {
+  if (!ctx->graph) {
+    cudaGraph_t g = nullptr;
+    CK(cudaStreamBeginCapture(ctx->stream, cudaStreamCaptureModeThreadLocal));
+    cudaError_t e = enqueue_step(ctx);
+    cudaError_t e2 = cudaStreamEndCapture(ctx->stream, &g);
+    if (e != cudaSuccess || e2 != cudaSuccess) {
+      if (g) cudaGraphDestroy(g);
+      return fail(ctx, CHIMERA_ECUDA, std::string("capturing the step: ") + cudaGetErrorString(e != cudaSuccess ? e : e2));
+    }
+    e = cudaGraphInstantiate(&ctx->graph, g, 0);
+    cudaGraphDestroy(g);
+    if (e != cudaSuccess) return fail(ctx, CHIMERA_ECUDA, std::string("instantiating the step graph: ") + cudaGetErrorString(e));
+  }
+  if (ctx->ovr_pending) {
+    const int one = 1;
+    CK(cudaMemcpyAsync(ctx->d_ovr_flag, &one, sizeof(int), cudaMemcpyHostToDevice, ctx->stream));
+  }
+  for (int i = 0; i < n_steps; ++i) {
+    CK(cudaGraphLaunch(ctx->graph, ctx->stream));
+    if (i == 0 && ctx->ovr_pending) {
+      CK(cudaMemsetAsync(ctx->d_ovr_flag, 0, sizeof(int), ctx->stream));
+      ctx->ovr_pending = false;
+    }
+  }
+  return CHIMERA_OK;
+}
+
+chimera_status read_new_tokens(chimera_ctx* ctx, int32_t* out_tokens, int per_seq, int32_t* out_count) {
+  const int B = ctx->batch;
+  std::vector<int> n_new(B);
+  CK(cudaMemcpyAsync(n_new.data(), ctx->d_n, B * sizeof(int), cudaMemcpyDeviceToHost, ctx->stream));
+  CK(cudaStreamSynchronize(ctx->stream));
+  chimera_status st = check_err(ctx);
+  if (st != CHIMERA_OK) return st;
+  for (int b = 0; b < B; ++b) {
+    const int cnt = n_new[b] - ctx->host_n[b];
+    if (cnt < 1 || cnt > per_seq) return fail(ctx, CHIMERA_ECUDA, "inconsistent committed length after a step");
+    CK(cudaMemcpyAsync(out_tokens + static_cast<size_t>(b) * per_seq,
+                       ctx->d_tok + static_cast<size_t>(b) * ctx->tok_stride + ctx->host_n[b], cnt * sizeof(int),
+                       cudaMemcpyDeviceToHost, ctx->stream));
+    out_count[b] = cnt;
+  }
+  CK(cudaStreamSynchronize(ctx->stream));
+  for (int b = 0; b < B; ++b) ctx->host_n[b] = n_new[b];
+  return CHIMERA_OK;
+}
+
+void free_ctx(chimera_ctx* ctx) {
+  if (!ctx) return;
+  if (ctx->graph) cudaGraphExecDestroy(ctx->graph);
+  for (auto& e : ctx->prof_ev) {
+    cudaEventDestroy(e.a);
+    cudaEventDestroy(e.b);
+  }
+  for (void* p : ctx->allocs) cudaFree(p);
+  if (ctx->h_stage) cudaFreeHost(ctx->h_stage);
+  if (ctx->own_stream && ctx->stream) cudaStreamDestroy(ctx->stream);
+  delete ctx;
+}
+
+bool valid_block(const chimera_block_weights& b) {
+  return b.attn_norm && b.wqkv && b.wo && b.ffn_norm && b.w_gate && b.w_up && b.w_down;
+}
+
+}  // namespace
+
+// ===========================================================================
+// C ABI
+// ===========================================================================
+extern "C" {
+
+chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w, void* cuda_stream,
+                            chimera_ctx** out) {
+  if (!out) return CHIMERA_EINVAL;
+  *out = nullptr;
+  if (!cfg || !w) return CHIMERA_EINVAL;
+  const chimera_config& c = *cfg;
+  if (c.n_layers < 1 || c.d_model < 32 || c.n_heads < 1 || c.head_dim * c.n_heads != c.d_model ||
+      (c.head_dim != 64 && c.head_dim != 128) || c.ffn_dim < 8 || c.vocab < 8 || (c.dtype != 0 && c.dtype != 1) ||
+      c.n_draft_heads < 1 || c.n_draft_heads > 4 || c.tree_nodes < 2 || c.tree_nodes > 64 || c.max_batch < 1 ||
+      c.max_batch > 64 || c.kv_block != 16 || c.max_seq_len < 32 || !(c.rms_eps > 0) || !(c.rope_theta > 0))
+    return CHIMERA_EINVAL;
+  if (c.dtype == 1 && (c.d_model % 64 != 0 || c.ffn_dim % 8 != 0)) return CHIMERA_EINVAL;
+  for (int k = 0; k < c.n_draft_heads; ++k)
+    if (c.topk[k] < 1 || c.topk[k] > MAX_KMAX) return CHIMERA_EINVAL;
+  if (!w->embed || !w->layers || !w->final_norm || !w->lm_head || !w->tri_w1 || !w->tri_w2 || !w->heads ||
+      !valid_block(w->draft))
+    return CHIMERA_EINVAL;
+  for (int l = 0; l < c.n_layers; ++l)
+    if (!valid_block(w->layers[l])) return CHIMERA_EINVAL;
+  for (int k = 0; k < c.n_draft_heads; ++k)
+    if (!w->heads[k]) return CHIMERA_EINVAL;
+
+  chimera_ctx* ctx = new chimera_ctx();
+  ctx->cfg = c;
+  ctx->L = c.n_layers;
+  ctx->d = c.d_model;
+  ctx->H = c.n_heads;
+  ctx->hd = c.head_dim;
+  ctx->F = c.ffn_dim;
+  ctx->V = c.vocab;
+  ctx->K = c.n_draft_heads;
+  ctx->N = c.tree_nodes;
+  ctx->dtype = c.dtype;
+  ctx->esz = c.dtype == 0 ? 4 : 2;
+  ctx->Bmax = c.max_batch;
+  ctx->cap = c.max_seq_len;
+  ctx->KMAX = 1;
+  for (int k = 0; k < ctx->K; ++k) ctx->KMAX = std::max(ctx->KMAX, c.topk[k]);
+  std::string terr;
+  if (!build_tree(c.topk, ctx->K, ctx->N, &ctx->tree, &terr)) {
+    ctx->err = terr;
+    free_ctx(ctx);
+    return CHIMERA_EINVAL;
+  }
+  ctx->D1 = ctx->tree.depth_max + 1;
+  ctx->embed = w->embed;
+  ctx->layers.assign(w->layers, w->layers + c.n_layers);
+  ctx->draft = w->draft;
+  ctx->final_norm = w->final_norm;
+  ctx->lm_head = w->lm_head;
+  ctx->tri_w1 = w->tri_w1;
+  ctx->tri_w2 = w->tri_w2;
+  ctx->heads.assign(w->heads, w->heads + c.n_draft_heads);
+  ctx->num_sms = tc_num_sms();
+
+  if (cuda_stream) {
+    ctx->stream = static_cast<cudaStream_t>(cuda_stream);
+  } else {
+    if (cudaStreamCreateWithFlags(&ctx->stream, cudaStreamNonBlocking) != cudaSuccess) {
+      free_ctx(ctx);
+      return CHIMERA_ECUDA;
+    }
+    ctx->own_stream = true;
+  }
+
+  const int B = ctx->Bmax, d = ctx->d, F = ctx->F, V = ctx->V, N = ctx->N, K = ctx->K;
+  ctx->tok_stride = ctx->cap + 1;
+  ctx->max_pages = (ctx->cap + 15) / 16;
+  ctx->NB = B * ctx->max_pages;
+  ctx->kv_layer_stride = static_cast<long long>(ctx->NB) * ctx->H * 2 * 16 * ctx->hd;
+  ctx->max_pos = ctx->cap + 64;
+  ctx->R = B * std::max(N, CHUNK);
+  const int Rc = B * std::max(CHUNK, ctx->D1);
+  bool ok = true;
+  ok = ok && dalloc_bytes(ctx, &ctx->kv, static_cast<size_t>(ctx->kv_layer_stride) * ctx->L * ctx->esz);
+  ok = ok && dalloc_bytes(ctx, &ctx->dkv, static_cast<size_t>(ctx->kv_layer_stride) * ctx->esz);
+  ok = ok && dalloc(ctx, &ctx->d_pt, static_cast<size_t>(B) * ctx->max_pages);
+  ok = ok && dalloc(ctx, &ctx->d_rope, static_cast<size_t>(ctx->max_pos) * (ctx->hd / 2));
+  ok = ok && dalloc(ctx, &ctx->x, static_cast<size_t>(ctx->R) * d);
+  ok = ok && dalloc_bytes(ctx, &ctx->xn, static_cast<size_t>(std::max(ctx->R, Rc)) * d * ctx->esz);
+  ok = ok && dalloc_bytes(ctx, &ctx->qkv, static_cast<size_t>(ctx->R) * 3 * d * ctx->esz);
+  ok = ok && dalloc_bytes(ctx, &ctx->qr, static_cast<size_t>(ctx->R) * d * ctx->esz);
+  ok = ok && dalloc_bytes(ctx, &ctx->ao, static_cast<size_t>(ctx->R) * d * ctx->esz);
+  ok = ok && dalloc_bytes(ctx, &ctx->gu, static_cast<size_t>(ctx->R) * 2 * F * ctx->esz);
+  ok = ok && dalloc_bytes(ctx, &ctx->hf, static_cast<size_t>(ctx->R) * F * ctx->esz);
+  ok = ok && dalloc_bytes(ctx, &ctx->hfin, static_cast<size_t>(ctx->R) * d * ctx->esz);
+  ok = ok && dalloc(ctx, &ctx->logits, static_cast<size_t>(B) * N * V);
+  ok = ok && dalloc_bytes(ctx, &ctx->tbuf, static_cast<size_t>(B) * 3 * d * ctx->esz);
+  ok = ok && dalloc_bytes(ctx, &ctx->ubuf, static_cast<size_t>(B) * d * ctx->esz);
+  ok = ok && dalloc(ctx, &ctx->dres, static_cast<size_t>(B) * d);
+  ok = ok && dalloc_bytes(ctx, &ctx->headin, static_cast<size_t>(B) * 2 * d * ctx->esz);
+  ok = ok && dalloc_bytes(ctx, &ctx->hfull_log, static_cast<size_t>(K) * B * d * ctx->esz);
+  ok = ok && dalloc(ctx, &ctx->hlog, static_cast<size_t>(K) * B * V);
+  ok = ok && dalloc_bytes(ctx, &ctx->hsel, static_cast<size_t>(B) * ctx->D1 * d * ctx->esz);
+  ok = ok && dalloc_bytes(ctx, &ctx->kvtmp, static_cast<size_t>(Rc) * 2 * d * ctx->esz);
+  ok = ok && dalloc(ctx, &ctx->d_n, B);
+  ok = ok && dalloc(ctx, &ctx->d_tok, static_cast<size_t>(B) * ctx->tok_stride);
+  ok = ok && dalloc(ctx, &ctx->d_node_tok, static_cast<size_t>(B) * N);
+  ok = ok && dalloc(ctx, &ctx->d_topk, static_cast<size_t>(B) * K * ctx->KMAX);
+  ok = ok && dalloc(ctx, &ctx->d_topk_val, static_cast<size_t>(B) * K * ctx->KMAX);
+  ok = ok && dalloc(ctx, &ctx->d_amax, static_cast<size_t>(std::max(B * N, B)));
+  ok = ok && dalloc(ctx, &ctx->d_path, static_cast<size_t>(B) * ctx->D1);
+  ok = ok && dalloc(ctx, &ctx->d_L, B);
+  ok = ok && dalloc(ctx, &ctx->d_bonus, B);
+  ok = ok && dalloc(ctx, &ctx->d_ovr, static_cast<size_t>(B) * N);
+  ok = ok && dalloc(ctx, &ctx->d_ovr_flag, 1);
+  ok = ok && dalloc(ctx, &ctx->d_valid, B);
+  ok = ok && dalloc(ctx, &ctx->d_last, B);
+  ok = ok && dalloc(ctx, &ctx->d_count_log, static_cast<size_t>(B) * LOG_CAP);
+  ok = ok && dalloc(ctx, &ctx->d_step, 1);
+  ok = ok && dalloc(ctx, &ctx->d_err, 1);
+  ok = ok && dalloc(ctx, &ctx->d_depth, N);
+  ok = ok && dalloc(ctx, &ctx->d_rank, N);
+  ok = ok && dalloc(ctx, &ctx->d_anc, N);
+  ok = ok && dalloc(ctx, &ctx->d_chain, 64);
+  ok = ok && dalloc(ctx, &ctx->d_child_start, N + 1);
+  ok = ok && dalloc(ctx, &ctx->d_child, ctx->tree.child.size());
+  if (ctx->dtype == 1) {
+    ok = ok && dalloc(ctx, &ctx->lin_ws, tc_ws_floats(256));
+    ok = ok && dalloc(ctx, &ctx->lin_cnt, static_cast<size_t>(tc_max_tiles()));
+  }
+  ctx->att_ws_floats = attn_ws_floats(B, ctx->H, 16, std::max(N, CHUNK), ctx->hd);
+  ok = ok && dalloc(ctx, &ctx->att_ws, ctx->att_ws_floats);
+  ok = ok && dalloc(ctx, &ctx->att_cnt, static_cast<size_t>(B) * ctx->H);
+  if (ok && cudaMallocHost(reinterpret_cast<void**>(&ctx->h_stage), 4096 * sizeof(int)) != cudaSuccess) ok = false;
+  if (!ok) {
+    free_ctx(ctx);
+    return CHIMERA_ENOMEM;
+  }
+  ctx->h_stage_ints = 4096;
+
+  // zero-initialised state and scratch
+  cudaStream_t s = ctx->stream;
+  bool zok = true;
+  zok = zok && cudaMemsetAsync(ctx->kv, 0, static_cast<size_t>(ctx->kv_layer_stride) * ctx->L * ctx->esz, s) == cudaSuccess;
+  zok = zok && cudaMemsetAsync(ctx->dkv, 0, static_cast<size_t>(ctx->kv_layer_stride) * ctx->esz, s) == cudaSuccess;
+  zok = zok && cudaMemsetAsync(ctx->att_cnt, 0, static_cast<size_t>(B) * ctx->H * sizeof(int), s) == cudaSuccess;
+  if (ctx->lin_cnt)
+    zok = zok && cudaMemsetAsync(ctx->lin_cnt, 0, static_cast<size_t>(tc_max_tiles()) * sizeof(int), s) == cudaSuccess;
+  zok = zok && cudaMemsetAsync(ctx->d_err, 0, sizeof(int), s) == cudaSuccess;
+  zok = zok && cudaMemsetAsync(ctx->d_ovr_flag, 0, sizeof(int), s) == cudaSuccess;
+  zok = zok && cudaMemsetAsync(ctx->d_step, 0, sizeof(int), s) == cudaSuccess;
+  zok = zok && cudaMemsetAsync(ctx->d_topk, 0, static_cast<size_t>(B) * K * ctx->KMAX * sizeof(int), s) == cudaSuccess;
+  zok = zok && cudaMemsetAsync(ctx->headin, 0, static_cast<size_t>(B) * 2 * d * ctx->esz, s) == cudaSuccess;
+  zok = zok && cudaMemsetAsync(ctx->x, 0, static_cast<size_t>(ctx->R) * d * sizeof(float), s) == cudaSuccess;
+
+  // tree, chain masks and the RoPE table (fp64 on the host, rounded to fp32)
+  std::vector<unsigned long long> chain(64);
+  for (int i = 0; i < 64; ++i) chain[i] = i == 63 ? ~0ull : ((1ull << (i + 1)) - 1);
+  const int half = ctx->hd / 2;
+  std::vector<float2> rope(static_cast<size_t>(ctx->max_pos) * half);
+  for (int p = 0; p < ctx->max_pos; ++p)
+    for (int j = 0; j < half; ++j) {
+      const double inv = std::pow(static_cast<double>(c.rope_theta), -2.0 * j / ctx->hd);
+      const double a = static_cast<double>(p) * inv;
+      rope[static_cast<size_t>(p) * half + j] = make_float2(static_cast<float>(std::cos(a)), static_cast<float>(std::sin(a)));
+    }
+  const Tree& t = ctx->tree;
+  std::vector<unsigned long long> anc(t.anc.begin(), t.anc.end());
+  zok = zok && cudaMemcpyAsync(ctx->d_depth, t.depth.data(), N * sizeof(int), cudaMemcpyHostToDevice, s) == cudaSuccess;
+  zok = zok && cudaMemcpyAsync(ctx->d_rank, t.rank.data(), N * sizeof(int), cudaMemcpyHostToDevice, s) == cudaSuccess;
+  zok = zok && cudaMemcpyAsync(ctx->d_anc, anc.data(), N * sizeof(unsigned long long), cudaMemcpyHostToDevice, s) == cudaSuccess;
+  zok = zok && cudaMemcpyAsync(ctx->d_chain, chain.data(), 64 * sizeof(unsigned long long), cudaMemcpyHostToDevice, s) == cudaSuccess;
+  zok = zok && cudaMemcpyAsync(ctx->d_child_start, t.child_start.data(), (N + 1) * sizeof(int), cudaMemcpyHostToDevice, s) == cudaSuccess;
+  zok = zok && cudaMemcpyAsync(ctx->d_child, t.child.data(), t.child.size() * sizeof(int), cudaMemcpyHostToDevice, s) == cudaSuccess;
+  zok = zok && cudaMemcpyAsync(ctx->d_rope, rope.data(), rope.size() * sizeof(float2), cudaMemcpyHostToDevice, s) == cudaSuccess;
+  zok = zok && cudaStreamSynchronize(s) == cudaSuccess;
+  if (!zok) {
+    free_ctx(ctx);
+    return CHIMERA_ECUDA;
+  }
+  ctx->h_pt.assign(static_cast<size_t>(B) * ctx->max_pages, 0);
+  ctx->seq_blocks.assign(B, {});
+  ctx->free_blocks.clear();
+  for (int i = ctx->NB - 1; i >= 0; --i) ctx->free_blocks.push_back(i);
+  *out = ctx;
+  return CHIMERA_OK;
+}
+
+chimera_status chimera_prefill(chimera_ctx* ctx, int batch, const int32_t* tokens, const int32_t* lens) {
+  if (!ctx) return CHIMERA_EINVAL;
+  if (batch < 1 || batch > ctx->Bmax || !tokens || !lens) return fail(ctx, CHIMERA_EINVAL, "bad batch or NULL input");
+  long long total = 0;
+  int max_len = 0;
+  for (int b = 0; b < batch; ++b) {
+    if (lens[b] < 1) return fail(ctx, CHIMERA_EINVAL, "empty prompt");
+    total += lens[b];
+    max_len = std::max(max_len, static_cast<int>(lens[b]));
+  }
+  for (long long i = 0; i < total; ++i)
+    if (tokens[i] < 0 || tokens[i] >= ctx->V) return fail(ctx, CHIMERA_EINVAL, "token id out of range");
+  const int need = std::max(ctx->N, ctx->K) + 1 + ctx->D1;
+  for (int b = 0; b < batch; ++b)
+    if (lens[b] + need > ctx->cap) return fail(ctx, CHIMERA_ECAPACITY, "prompt too long for max_seq_len");
+
+  // reset: free every block, rebuild plans for this batch, drop the step graph
+  ctx->prefilled = false;
+  for (auto& blocks : ctx->seq_blocks) {
+    for (int blk : blocks) ctx->free_blocks.push_back(blk);
+    blocks.clear();
+  }
+  std::fill(ctx->h_pt.begin(), ctx->h_pt.end(), 0);
+  ctx->pt_dirty = true;
+  if (ctx->graph) {
+    cudaGraphExecDestroy(ctx->graph);
+    ctx->graph = nullptr;
+  }
+  ctx->batch = batch;
+  if (!build_plans(ctx, batch)) return CHIMERA_EINVAL;
+  for (int b = 0; b < batch; ++b) {
+    chimera_status st = ensure_blocks(ctx, b, lens[b] + need);
+    if (st != CHIMERA_OK) return st;
+  }
+  chimera_status st = flush_page_table(ctx);
+  if (st != CHIMERA_OK) return st;
+
+  cudaStream_t s = ctx->stream;
+  CK(cudaMemsetAsync(ctx->d_n, 0, ctx->Bmax * sizeof(int), s));
+  CK(cudaMemsetAsync(ctx->d_tok, 0, static_cast<size_t>(ctx->Bmax) * ctx->tok_stride * sizeof(int), s));
+  CK(cudaMemsetAsync(ctx->d_step, 0, sizeof(int), s));
+  CK(cudaMemsetAsync(ctx->d_ovr_flag, 0, sizeof(int), s));
+  ctx->ovr_pending = false;
+  {
+    long long off = 0;
+    for (int b = 0; b < batch; ++b) {
+      CK(cudaMemcpyAsync(ctx->d_tok + static_cast<size_t>(b) * ctx->tok_stride, tokens + off, lens[b] * sizeof(int),
+                         cudaMemcpyHostToDevice, s));
+      off += lens[b];
+    }
+    CK(cudaStreamSynchronize(s));
+  }
+  ctx->host_n.assign(batch, 0);
+  const int d = ctx->d, B = batch;
+  const int chunks = (max_len + CHUNK - 1) / CHUNK;
+  const void* dl_norm = ctx->draft.attn_norm;
+  for (int cidx = 0; cidx < chunks; ++cidx) {
+    int* hv = ctx->h_stage;
+    for (int b = 0; b < B; ++b) {
+      const int v = std::max(0, std::min(CHUNK, lens[b] - cidx * CHUNK));
+      hv[b] = v;
+      const int li = lens[b] - 1 - cidx * CHUNK;
+      hv[64 + b] = (li >= 0 && li < CHUNK) ? li : -1;
+    }
+    CK(cudaMemcpyAsync(ctx->d_valid, hv, B * sizeof(int), cudaMemcpyHostToDevice, s));
+    CK(cudaMemcpyAsync(ctx->d_last, hv + 64, B * sizeof(int), cudaMemcpyHostToDevice, s));
+    CK(embed(ctx->dtype, ctx->embed, d, ctx->V, ctx->x, B * CHUNK, CHUNK, nullptr, ctx->d_tok, ctx->tok_stride, ctx->d_n,
+             ctx->d_valid, ctx->d_err, s));
+    for (int l = 0; l < ctx->L; ++l)
+      CK(enqueue_layer(ctx, l, &ctx->pre[5 * l], B * CHUNK, CHUNK, ctx->d_valid, nullptr, ctx->d_chain,
+                       ctx->att_splits_pre, 0));
+    CK(rmsnorm(ctx->dtype, 1, ctx->x, d, ctx->final_norm, ctx->hfin, d, B * CHUNK, d, ctx->cfg.rms_eps, s));
+    // draft-layer K/V of the chunk's H_LLM rows
+    CK(rmsnorm(ctx->dtype, ctx->dtype == 0 ? 1 : 0, ctx->hfin, d, dl_norm, ctx->xn, d, B * CHUNK, d, ctx->cfg.rms_eps, s));
+    CK(run_lin(ctx, ctx->pre_dkv));
+    CK(run_rope(ctx, true, 0, ctx->kvtmp, 2 * d, -1, 0, d, CHUNK, ctx->d_valid, 0, 0, 0, nullptr));
+    CK(launch_prefill_advance(ctx->dtype, ctx->hfin, d, CHUNK, ctx->d_valid, ctx->d_last, ctx->d_n, ctx->headin, B, s));
+    CK(cudaStreamSynchronize(s));  // the staging buffer is reused by the next chunk
+  }
+  // root = greedy next token of each prompt (eq. 1)
+  CK(run_lin(ctx, ctx->pre_lm));
+  CK(argmax_rows(ctx->logits, ctx->V, B, ctx->d_amax, s));
+  CK(launch_set_root(ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_amax, B, s));
+  CK(cudaStreamSynchronize(s));
+  st = check_err(ctx);
+  if (st != CHIMERA_OK) return st;
+  for (int b = 0; b < B; ++b) ctx->host_n[b] = lens[b];
+  ctx->prefilled = true;
+  return CHIMERA_OK;
+}
+
+chimera_status chimera_step(chimera_ctx* ctx, int32_t* out_tokens, int32_t* out_count) {
+  if (!ctx) return CHIMERA_EINVAL;
+  if (!out_tokens || !out_count) return fail(ctx, CHIMERA_EINVAL, "NULL output");
+  chimera_status st = steps_prepare(ctx, 1);
+  if (st != CHIMERA_OK) return st;
+  st = launch_steps(ctx, 1);
+  if (st != CHIMERA_OK) return st;
+  return read_new_tokens(ctx, out_tokens, ctx->D1, out_count);
+}
+
+chimera_status chimera_generate(chimera_ctx* ctx, int n_steps, int32_t* out_tokens, int32_t* out_count) {
+  if (!ctx) return CHIMERA_EINVAL;
+  if (n_steps < 1 || !out_tokens || !out_count) return fail(ctx, CHIMERA_EINVAL, "bad arguments");
+  chimera_status st = steps_prepare(ctx, n_steps);
+  if (st != CHIMERA_OK) return st;
+  st = launch_steps(ctx, n_steps);
+  if (st != CHIMERA_OK) return st;
+  return read_new_tokens(ctx, out_tokens, n_steps * ctx->D1, out_count);
+}
+
+chimera_status chimera_step_async(chimera_ctx* ctx, int n_steps) {
+  if (!ctx) return CHIMERA_EINVAL;
+  if (n_steps < 1) return fail(ctx, CHIMERA_EINVAL, "n_steps < 1");
+  chimera_status st = steps_prepare(ctx, n_steps);
+  if (st != CHIMERA_OK) return st;
+  st = launch_steps(ctx, n_steps);
+  if (st != CHIMERA_OK) return st;
+  // host_n is refreshed by chimera_sync
+  return CHIMERA_OK;
+}
+
+chimera_status chimera_sync(chimera_ctx* ctx) {
+  if (!ctx) return CHIMERA_EINVAL;
+  CK(cudaStreamSynchronize(ctx->stream));
+  if (ctx->batch > 0) {
+    CK(cudaMemcpy(ctx->host_n.data(), ctx->d_n, ctx->batch * sizeof(int), cudaMemcpyDeviceToHost));
+  }
+  return check_err(ctx);
+}
+
+void chimera_free(chimera_ctx* ctx) {
+  if (ctx && ctx->stream) cudaStreamSynchronize(ctx->stream);
+  free_ctx(ctx);
+}
+
+const char* chimera_last_error(const chimera_ctx* ctx) { return ctx ? ctx->err.c_str() : "NULL context"; }
+
+chimera_status chimera_tree(const chimera_ctx* ctx, int32_t* depth, int32_t* parent, int32_t* rank, uint64_t* anc) {
+  if (!ctx) return CHIMERA_EINVAL;
+  for (int i = 0; i < ctx->N; ++i) {
+    if (depth) depth[i] = ctx->tree.depth[i];
+    if (parent) parent[i] = ctx->tree.parent[i];
+    if (rank) rank[i] = ctx->tree.rank[i];
+    if (anc) anc[i] = ctx->tree.anc[i];
+  }
+  return CHIMERA_OK;
+}
+
+chimera_status chimera_profile_step(chimera_ctx* ctx, int max, int32_t* kinds, int32_t* phases, float* ms,
+                                    double* bytes, int32_t* count) {
+  if (!ctx) return CHIMERA_EINVAL;
+  if (!count) return fail(ctx, CHIMERA_EINVAL, "NULL count");
+  chimera_status st = steps_prepare(ctx, 1);
+  if (st != CHIMERA_OK) return st;
+  ctx->prof = true;
+  ctx->prof_used = 0;
+  cudaError_t e = enqueue_step(ctx);
+  ctx->prof = false;
+  if (e != cudaSuccess) return fail(ctx, CHIMERA_ECUDA, std::string("profiled step: ") + cudaGetErrorString(e));
+  CK(cudaStreamSynchronize(ctx->stream));
+  const int n = static_cast<int>(ctx->prof_used);
+  for (int i = 0; i < n && i < max; ++i) {
+    float t = 0;
+    cudaEventElapsedTime(&t, ctx->prof_ev[i].a, ctx->prof_ev[i].b);
+    if (kinds) kinds[i] = ctx->prof_ev[i].kind;
+    if (phases) phases[i] = ctx->prof_ev[i].phase;
+    if (ms) ms[i] = t;
+    if (bytes) bytes[i] = ctx->prof_ev[i].bytes;
+  }
+  *count = n;
+  CK(cudaMemcpy(ctx->host_n.data(), ctx->d_n, ctx->batch * sizeof(int), cudaMemcpyDeviceToHost));
+  return check_err(ctx);
+}
+
+chimera_status chimera_debug_override_tree(chimera_ctx* ctx, const int32_t* node_tokens) {
+  if (!ctx) return CHIMERA_EINVAL;
+  if (!ctx->prefilled) return fail(ctx, CHIMERA_ESTATE, "override before prefill");
+  if (!node_tokens) return fail(ctx, CHIMERA_EINVAL, "NULL tokens");
+  const size_t n = static_cast<size_t>(ctx->batch) * ctx->N;
+  for (size_t i = 0; i < n; ++i)
+    if (i % ctx->N != 0 && (node_tokens[i] < 0 || node_tokens[i] >= ctx->V))
+      return fail(ctx, CHIMERA_EINVAL, "override token out of range");
+  CK(cudaMemcpy(ctx->d_ovr, node_tokens, n * sizeof(int), cudaMemcpyHostToDevice));
+  ctx->ovr_pending = true;
+  return CHIMERA_OK;
+}
+
+chimera_status chimera_debug_set_root(chimera_ctx* ctx, const int32_t* roots) {
+  if (!ctx) return CHIMERA_EINVAL;
+  if (!ctx->prefilled) return fail(ctx, CHIMERA_ESTATE, "set_root before prefill");
+  for (int b = 0; b < ctx->batch; ++b) {
+    if (roots[b] < 0 || roots[b] >= ctx->V) return fail(ctx, CHIMERA_EINVAL, "root out of range");
+    CK(cudaMemcpy(ctx->d_tok + static_cast<size_t>(b) * ctx->tok_stride + ctx->host_n[b], &roots[b], sizeof(int),
+                  cudaMemcpyHostToDevice));
+  }
+  return CHIMERA_OK;
+}
+
+chimera_status chimera_debug_read(chimera_ctx* ctx, int what, void* dst, size_t bytes) {
+  if (!ctx) return CHIMERA_EINVAL;
+  if (!dst) return fail(ctx, CHIMERA_EINVAL, "NULL destination");
+  const size_t B = ctx->batch ? ctx->batch : 1, N = ctx->N, V = ctx->V, d = ctx->d, K = ctx->K;
+  const void* src = nullptr;
+  size_t need = 0;
+  switch (what) {
+    case CHIMERA_DBG_NODE_TOKENS: src = ctx->d_node_tok; need = B * N * 4; break;
+    case CHIMERA_DBG_VERIFY_LOGITS: src = ctx->logits; need = B * N * V * 4; break;
+    case CHIMERA_DBG_VERIFY_HIDDEN: src = ctx->hfin; need = B * N * d * ctx->esz; break;
+    case CHIMERA_DBG_ARGMAX: src = ctx->d_amax; need = B * N * 4; break;
+    case CHIMERA_DBG_PATH: src = ctx->d_path; need = B * ctx->D1 * 4; break;
+    case CHIMERA_DBG_ACCEPT_LEN: src = ctx->d_L; need = B * 4; break;
+    case CHIMERA_DBG_DRAFT_LOGITS: src = ctx->hlog; need = K * B * V * 4; break;
+    case CHIMERA_DBG_TOPK: src = ctx->d_topk; need = B * K * ctx->KMAX * 4; break;
+    case CHIMERA_DBG_HFULL: src = ctx->hfull_log; need = K * B * d * ctx->esz; break;
+    case CHIMERA_DBG_N: src = ctx->d_n; need = B * 4; break;
+    case CHIMERA_DBG_TOKENS: src = ctx->d_tok; need = B * ctx->tok_stride * 4; break;
+    case CHIMERA_DBG_PREFILL_LOGITS: src = ctx->logits; need = B * V * 4; break;
+    default: return fail(ctx, CHIMERA_EINVAL, "unknown debug buffer");
+  }
+  if (bytes != need)
+    return fail(ctx, CHIMERA_EINVAL, "debug read: expected " + std::to_string(need) + " bytes, got " + std::to_string(bytes));
+  CK(cudaStreamSynchronize(ctx->stream));
+  CK(cudaMemcpy(dst, src, need, cudaMemcpyDeviceToHost));
+  return CHIMERA_OK;
+}
+
+chimera_status chimera_debug_read_kv(chimera_ctx* ctx, int layer, int seq, int pos0, int count, void* k_dst,
+                                     void* v_dst) {
+  if (!ctx) return CHIMERA_EINVAL;
+  if (layer < -1 || layer >= ctx->L || seq < 0 || seq >= ctx->batch || pos0 < 0 || count < 0 ||
+      pos0 + count > static_cast<int>(ctx->seq_blocks[seq].size()) * 16 || !k_dst || !v_dst)
+    return fail(ctx, CHIMERA_EINVAL, "bad KV read");
+  CK(cudaStreamSynchronize(ctx->stream));
+  const size_t row = static_cast<size_t>(ctx->hd) * ctx->esz;
+  const char* pool = static_cast<const char*>(layer < 0 ? ctx->dkv : ctx->kv) +
+                     (layer < 0 ? 0 : static_cast<size_t>(layer) * ctx->kv_layer_stride * ctx->esz);
+  for (int i = 0; i < count; ++i) {
+    const int slot = pos0 + i;
+    const int page = ctx->h_pt[seq * ctx->max_pages + slot / 16];
+    for (int h = 0; h < ctx->H; ++h) {
+      const char* base = pool + ((static_cast<size_t>(page) * ctx->H + h) * 2) * 16 * row + (slot % 16) * row;
+      CK(cudaMemcpy(static_cast<char*>(k_dst) + (static_cast<size_t>(i) * ctx->H + h) * row, base, row,
+                    cudaMemcpyDeviceToHost));
+      CK(cudaMemcpy(static_cast<char*>(v_dst) + (static_cast<size_t>(i) * ctx->H + h) * row, base + 16 * row, row,
+                    cudaMemcpyDeviceToHost));
+    }
+  }
+  return CHIMERA_OK;
+}
+
+// ---------------------------------------------------------------------------
+// stateless kernel-level entry points
+// ---------------------------------------------------------------------------
+namespace {
+struct OpScratch {
+  int device = -1;
+  float* lin_ws = nullptr;
+  int* lin_cnt = nullptr;
+  int* err = nullptr;
+  float* att_ws = nullptr;
+  size_t att_floats = 0;
+  int* att_cnt = nullptr;
+};
+std::mutex g_op_mu;
+OpScratch g_op;
+
+bool op_scratch() {
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (g_op.device == dev) return true;
+  OpScratch s;
+  s.device = dev;
+  s.att_floats = static_cast<size_t>(16) << 20;
+  if (cudaMalloc(&s.lin_ws, tc_ws_floats(256) * sizeof(float)) != cudaSuccess) return false;
+  if (cudaMalloc(&s.lin_cnt, tc_max_tiles() * sizeof(int)) != cudaSuccess) return false;
+  if (cudaMalloc(&s.err, sizeof(int)) != cudaSuccess) return false;
+  if (cudaMalloc(&s.att_ws, s.att_floats * sizeof(float)) != cudaSuccess) return false;
+  if (cudaMalloc(&s.att_cnt, 64 * 256 * sizeof(int)) != cudaSuccess) return false;
+  cudaMemset(s.lin_cnt, 0, tc_max_tiles() * sizeof(int));
+  cudaMemset(s.err, 0, sizeof(int));
+  cudaMemset(s.att_cnt, 0, 64 * 256 * sizeof(int));
+  if (cudaDeviceSynchronize() != cudaSuccess) return false;
+  g_op = s;
+  return true;
+}
+}  // namespace
+
+chimera_status chimera_op_linear(int dtype, int epi, int out_f32, int M, int N, int K, const void* X, int ldx,
+                                 const void* W, void* Y, int ldy, void* cuda_stream) {
+  if ((dtype != 0 && dtype != 1) || epi < 0 || epi > 2 || M < 1 || N < 1 || K < 1 || !X || !W || !Y || ldx < K ||
+      ldy < N)
+    return CHIMERA_EINVAL;
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  if (dtype == 0) return f32_linear(M, N, K, static_cast<const float*>(X), ldx, static_cast<const float*>(W),
+                                    static_cast<float*>(Y), ldy, epi, s) == cudaSuccess
+                             ? CHIMERA_OK
+                             : CHIMERA_ECUDA;
+  std::lock_guard<std::mutex> lk(g_op_mu);
+  if (!op_scratch()) return CHIMERA_ENOMEM;
+  TcLinearPlan plan;
+  char msg[256];
+  if (tc_linear_plan(&plan, M, N, K, X, ldx, W, Y, ldy, epi, epi == EPI_RESID ? 1 : out_f32, g_op.lin_ws, g_op.lin_cnt,
+                     g_op.err, msg, sizeof(msg)) != 0)
+    return CHIMERA_EINVAL;
+  return tc_linear_launch(plan, s) == cudaSuccess ? CHIMERA_OK : CHIMERA_ECUDA;
+}
+
+chimera_status chimera_op_attention(int dtype, int batch, int n_heads, int head_dim, int nq, int q_local0, int n_local,
+                                    const void* q, int ldq, int q_rows, const void* pool, const int32_t* page_table,
+                                    int max_pages, const int32_t* n_ctx, const uint64_t* anc, void* out, int ldo,
+                                    int splits, void* cuda_stream) {
+  if ((dtype != 0 && dtype != 1) || batch < 1 || n_heads < 1 || (head_dim != 64 && head_dim != 128) || nq < 1 ||
+      nq > 64 || n_local < 0 || n_local > 64 || q_local0 < 0 || !q || !pool || !page_table || !n_ctx || !anc || !out ||
+      splits < 1 || splits > 64 || batch * n_heads > 64 * 256)
+    return CHIMERA_EINVAL;
+  std::lock_guard<std::mutex> lk(g_op_mu);
+  if (!op_scratch()) return CHIMERA_ENOMEM;
+  AttnParams p{};
+  p.q = q;
+  p.ldq = ldq;
+  p.q_rows = q_rows;
+  p.nq = nq;
+  p.q_local0 = q_local0;
+  p.n_local = n_local;
+  p.anc = reinterpret_cast<const unsigned long long*>(anc);
+  p.pool = pool;
+  p.page_table = page_table;
+  p.max_pages = max_pages;
+  p.n_ctx = n_ctx;
+  p.out = out;
+  p.ldo = ldo;
+  p.B = batch;
+  p.H = n_heads;
+  p.hd = head_dim;
+  p.scale = 1.0f / std::sqrt(static_cast<float>(head_dim));
+  p.splits = splits;
+  p.ws = g_op.att_ws;
+  p.counters = g_op.att_cnt;
+  p.nq_max = nq;
+  if (attn_ws_floats(batch, n_heads, splits, nq, head_dim) > g_op.att_floats) return CHIMERA_EINVAL;
+  return attention(p, dtype, static_cast<cudaStream_t>(cuda_stream)) == cudaSuccess ? CHIMERA_OK : CHIMERA_ECUDA;
+}
+
+}  // extern "C"

@@ -1,0 +1,259 @@
+// Small kernels that stitch the step together: trigram gather, tree expansion,
+// greedy acceptance, KV compaction, hidden-state gathers and state update.
+#include "common.cuh"
+#include "step_kernels.h"
+
+namespace chimera {
+namespace {
+
+// Trigram input of draft sub-step k (eq. trigram_calculations): the embeddings of
+// x[n-2+k], x[n-1+k], x[n+k], where x[n] is the root and x[n+1+j] is head j's top-1.
+// A position before the start of the sequence contributes a zero block.
+template <typename T>
+__global__ void trigram_gather_kernel(const T* __restrict__ E, int d, int V, const int* n_arr,
+                                      const int* tok, int tok_stride, const int* topk, int K,
+                                      int KMAX, int k, T* __restrict__ out, int* err) {
+  const int b = blockIdx.x;
+  const int n = n_arr[b];
+  for (int t = 0; t < 3; ++t) {
+    const int i = n - 2 + k + t;
+    int id = -1;
+    if (i >= 0) id = i <= n ? tok[static_cast<size_t>(b) * tok_stride + i]
+                            : topk[(b * K + (i - n - 1)) * KMAX];
+    if (id >= V) {
+      if (threadIdx.x == 0) atomicOr(err, ERR_BAD_INDEX);
+      id = 0;
+    }
+    T* o = out + static_cast<size_t>(b) * 3 * d + t * d;
+    const T* e = E + static_cast<size_t>(id < 0 ? 0 : id) * d;
+    for (int c = threadIdx.x; c < d; c += blockDim.x) o[c] = id < 0 ? from_f<T>(0.f) : e[c];
+  }
+}
+
+// headin[b][d..2d) = h_full (the draft block output), kept per head for debugging.
+template <typename T>
+__global__ void hfull_store_kernel(const float* __restrict__ dres, int d, T* __restrict__ headin,
+                                   T* __restrict__ hlog) {
+  const int b = blockIdx.x;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) {
+    const T v = from_f<T>(dres[static_cast<size_t>(b) * d + c]);
+    headin[static_cast<size_t>(b) * 2 * d + d + c] = v;
+    hlog[static_cast<size_t>(b) * d + c] = v;
+  }
+}
+
+// Node tokens of the static tree: the root is x[n]; node i at depth >= 1 takes the
+// rank_i-th token of head depth_i - 1 (Section "Inference").
+__global__ void tree_expand_kernel(const int* n_arr, const int* tok, int tok_stride, const int* topk,
+                                   int K, int KMAX, const int* depth, const int* rank, int N,
+                                   const int* ovr_flag, const int* ovr, int* node_tok) {
+  const int b = blockIdx.x, i = threadIdx.x;
+  if (i >= N) return;
+  int t;
+  if (i == 0)
+    t = tok[static_cast<size_t>(b) * tok_stride + n_arr[b]];
+  else if (*ovr_flag)
+    t = ovr[b * N + i];
+  else
+    t = topk[(b * K + depth[i] - 1) * KMAX + rank[i]];
+  node_tok[b * N + i] = t;
+}
+
+// Greedy acceptance (Section "Verification"): from the root, move to the child whose
+// token equals the base argmax of the current node; the argmax after the last
+// accepted node is the bonus token.  Writes the path and the accepted tokens into
+// the token history at x[n..n+L].
+__global__ void accept_kernel(const int* n_arr, int* tok, int tok_stride, const int* node_tok,
+                              const int* amax, const int* child_start, const int* child, int N,
+                              int D1, int* path, int* Lacc, int* bonus) {
+  const int b = blockIdx.x;
+  if (threadIdx.x != 0) return;
+  const int n = n_arr[b];
+  int cur = 0, L = 0;
+  path[b * D1] = 0;
+  while (true) {
+    const int p = amax[b * N + cur];
+    int nxt = -1;
+    for (int c = child_start[cur]; c < child_start[cur + 1]; ++c)
+      if (node_tok[b * N + child[c]] == p) {
+        nxt = child[c];
+        break;
+      }
+    if (nxt < 0 || L + 1 >= D1) break;
+    cur = nxt;
+    ++L;
+    path[b * D1 + L] = cur;
+    tok[static_cast<size_t>(b) * tok_stride + n + L] = node_tok[b * N + cur];
+  }
+  for (int j = L + 1; j < D1; ++j) path[b * D1 + j] = path[b * D1 + L];
+  Lacc[b] = L;
+  bonus[b] = amax[b * N + cur];
+}
+
+// Move the accepted nodes' K/V rows from tree slot n+path[j] to slot n+j (j = 1..L)
+// in every layer.  All source rows are loaded before any store: a destination slot
+// can be the source of another path entry.
+__global__ void compact_kernel(char* pool, long long layer_stride_bytes, int H, int row_bytes,
+                               const int* n_arr, const int* path, const int* Lacc, int D1,
+                               const int* page_table, int max_pages) {
+  const int b = blockIdx.y;
+  const int L = Lacc[b];
+  if (L == 0) return;
+  const int layer = blockIdx.x / (2 * H);
+  const int kv = (blockIdx.x / H) & 1;
+  const int h = blockIdx.x % H;
+  const int n = n_arr[b];
+  const int chunks = row_bytes / 16;
+  const int j = 1 + threadIdx.x / chunks;
+  const int c = threadIdx.x % chunks;
+  char* base = pool + layer * layer_stride_bytes;
+  auto row_ptr = [&](int slot) {
+    const int page = page_table[b * max_pages + (slot >> 4)];
+    return reinterpret_cast<uint4*>(base + ((static_cast<size_t>(page) * H + h) * 2 + kv) * 16 * row_bytes +
+                                    static_cast<size_t>(slot & 15) * row_bytes) + c;
+  };
+  uint4 v = make_uint4(0, 0, 0, 0);
+  const bool active = j <= L && j < D1;
+  if (active) v = *row_ptr(n + path[b * D1 + j]);
+  __syncthreads();
+  if (active) *row_ptr(n + j) = v;
+}
+
+// hsel[b][j] = verify hidden of path node j (j <= L; later rows repeat the last);
+// headin[b][0..d) = hidden of the last accepted node (h_LLM of the new prefix end).
+template <typename T>
+__global__ void gather_hidden_kernel(const T* __restrict__ hfin, int d, int N, const int* path,
+                                     const int* Lacc, int D1, T* __restrict__ hsel,
+                                     T* __restrict__ headin) {
+  const int b = blockIdx.x, j = blockIdx.y;
+  const int L = Lacc[b];
+  const int node = path[b * D1 + (j <= L ? j : L)];
+  const T* src = hfin + static_cast<size_t>(b * N + node) * d;
+  T* dst = hsel + static_cast<size_t>(b * D1 + j) * d;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) {
+    const T v = src[c];
+    dst[c] = v;
+    if (j == L) headin[static_cast<size_t>(b) * 2 * d + c] = v;
+  }
+}
+
+// Commit: x[n+L+1] = bonus (the next root), n += L + 1, per-step count log.
+__global__ void finalize_kernel(int* n_arr, int* tok, int tok_stride, const int* Lacc,
+                                const int* bonus, int* count_log, int log_cap, int* step, int B) {
+  const int b = threadIdx.x;
+  const int s = *step;
+  __syncthreads();
+  if (b < B) {
+    const int L = Lacc[b];
+    const int n = n_arr[b];
+    tok[static_cast<size_t>(b) * tok_stride + n + L + 1] = bonus[b];
+    n_arr[b] = n + L + 1;
+    count_log[b * log_cap + (s % log_cap)] = L + 1;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) *step = s + 1;
+}
+
+// Prefill chunk bookkeeping: keep h_LLM of the last prompt row, advance n.
+template <typename T>
+__global__ void prefill_advance_kernel(const T* __restrict__ hfin, int d, int rows_per_seq,
+                                       const int* valid, const int* last, int* n_arr,
+                                       T* __restrict__ headin) {
+  const int b = blockIdx.x;
+  const int li = last[b];
+  if (li >= 0) {
+    const T* src = hfin + static_cast<size_t>(b * rows_per_seq + li) * d;
+    for (int c = threadIdx.x; c < d; c += blockDim.x) headin[static_cast<size_t>(b) * 2 * d + c] = src[c];
+  }
+  if (threadIdx.x == 0) n_arr[b] += valid[b];
+}
+
+__global__ void set_root_kernel(const int* n_arr, int* tok, int tok_stride, const int* amax, int B) {
+  const int b = threadIdx.x;
+  if (b < B) tok[static_cast<size_t>(b) * tok_stride + n_arr[b]] = amax[b];
+}
+
+}  // namespace
+
+cudaError_t launch_trigram_gather(int dtype, const void* E, int d, int V, const int* n, const int* tok,
+                                  int tok_stride, const int* topk, int K, int KMAX, int k, void* out,
+                                  int B, int* err, cudaStream_t s) {
+  if (dtype == 0)
+    trigram_gather_kernel<float><<<B, 256, 0, s>>>(static_cast<const float*>(E), d, V, n, tok, tok_stride,
+                                                   topk, K, KMAX, k, static_cast<float*>(out), err);
+  else
+    trigram_gather_kernel<bf16><<<B, 256, 0, s>>>(static_cast<const bf16*>(E), d, V, n, tok, tok_stride,
+                                                  topk, K, KMAX, k, static_cast<bf16*>(out), err);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_hfull_store(int dtype, const float* dres, int d, void* headin, void* hlog, int B,
+                               cudaStream_t s) {
+  if (dtype == 0)
+    hfull_store_kernel<float><<<B, 256, 0, s>>>(dres, d, static_cast<float*>(headin), static_cast<float*>(hlog));
+  else
+    hfull_store_kernel<bf16><<<B, 256, 0, s>>>(dres, d, static_cast<bf16*>(headin), static_cast<bf16*>(hlog));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_tree_expand(const int* n, const int* tok, int tok_stride, const int* topk, int K, int KMAX,
+                               const int* depth, const int* rank, int N, const int* ovr_flag, const int* ovr,
+                               int* node_tok, int B, cudaStream_t s) {
+  tree_expand_kernel<<<B, 64, 0, s>>>(n, tok, tok_stride, topk, K, KMAX, depth, rank, N, ovr_flag, ovr, node_tok);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_accept(const int* n, int* tok, int tok_stride, const int* node_tok, const int* amax,
+                          const int* child_start, const int* child, int N, int D1, int* path, int* Lacc,
+                          int* bonus, int B, cudaStream_t s) {
+  accept_kernel<<<B, 32, 0, s>>>(n, tok, tok_stride, node_tok, amax, child_start, child, N, D1, path, Lacc,
+                                 bonus);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_compact(void* pool, long long layer_stride_bytes, int n_layers, int H, int row_bytes,
+                           const int* n, const int* path, const int* Lacc, int D1, const int* page_table,
+                           int max_pages, int B, cudaStream_t s) {
+  const int threads = (row_bytes / 16) * (D1 - 1);
+  if (threads <= 0) return cudaSuccess;
+  dim3 grid(n_layers * 2 * H, B);
+  compact_kernel<<<grid, threads, 0, s>>>(static_cast<char*>(pool), layer_stride_bytes, H, row_bytes, n, path,
+                                          Lacc, D1, page_table, max_pages);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather_hidden(int dtype, const void* hfin, int d, int N, const int* path, const int* Lacc,
+                                 int D1, void* hsel, void* headin, int B, cudaStream_t s) {
+  dim3 grid(B, D1);
+  if (dtype == 0)
+    gather_hidden_kernel<float><<<grid, 256, 0, s>>>(static_cast<const float*>(hfin), d, N, path, Lacc, D1,
+                                                     static_cast<float*>(hsel), static_cast<float*>(headin));
+  else
+    gather_hidden_kernel<bf16><<<grid, 256, 0, s>>>(static_cast<const bf16*>(hfin), d, N, path, Lacc, D1,
+                                                    static_cast<bf16*>(hsel), static_cast<bf16*>(headin));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_finalize(int* n, int* tok, int tok_stride, const int* Lacc, const int* bonus, int* count_log,
+                            int log_cap, int* step, int B, cudaStream_t s) {
+  finalize_kernel<<<1, ((B + 31) / 32) * 32, 0, s>>>(n, tok, tok_stride, Lacc, bonus, count_log, log_cap, step, B);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_prefill_advance(int dtype, const void* hfin, int d, int rows_per_seq, const int* valid,
+                                   const int* last, int* n, void* headin, int B, cudaStream_t s) {
+  if (dtype == 0)
+    prefill_advance_kernel<float><<<B, 256, 0, s>>>(static_cast<const float*>(hfin), d, rows_per_seq, valid,
+                                                    last, n, static_cast<float*>(headin));
+  else
+    prefill_advance_kernel<bf16><<<B, 256, 0, s>>>(static_cast<const bf16*>(hfin), d, rows_per_seq, valid,
+                                                   last, n, static_cast<bf16*>(headin));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_set_root(const int* n, int* tok, int tok_stride, const int* amax, int B, cudaStream_t s) {
+  set_root_kernel<<<1, ((B + 31) / 32) * 32, 0, s>>>(n, tok, tok_stride, amax, B);
+  return cudaGetLastError();
+}
+
+}  // namespace chimera
