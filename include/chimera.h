@@ -21,8 +21,9 @@
  *     chimera_last_error().  Calls on one context are not thread-safe.
  *   - Weights are caller-owned DEVICE memory that must outlive the context.
  *     Matrices are row-major [out][in] (one output feature per row, y = W x).
- *     dtype 0 = fp32 everywhere; dtype 1 = bf16 weights/activations with fp32
- *     accumulation and an fp32 residual stream.
+ *     dtype 0 = fp32 everywhere; dtype 1 = bf16 weights, fp32 accumulation, an fp32
+ *     residual stream and fp32 projection outputs; `precision` selects how the
+ *     activations that feed the tensor cores and the KV caches are stored.
  *   - The context owns the paged KV caches (blocks of 16 positions), the draft KV
  *     cache, all scratch and the captured CUDA graph of the step.
  *   - Host buffers are caller-owned host memory.  chimera_step / chimera_generate /
@@ -68,6 +69,11 @@ typedef struct {
   int max_batch;        /* sequences per context, 1..64 */
   int max_seq_len;      /* KV slots per sequence (prompt + generated + N tree slots) */
   int kv_block;         /* must be 16 */
+  int precision;        /* bf16 models only.  1: every activation that feeds a tensor-core
+                           GEMM is kept as a hi + lo pair of bf16 values (two MMAs with fp32
+                           accumulation, ~fp32 accuracy) and the KV caches are fp32;
+                           0: activations rounded once to bf16 and bf16 KV caches.
+                           fp32 models ignore it. */
 } chimera_config;
 
 /* One Llama block: RMSNorm gains [d]; wqkv [3d][d] (rows q, then k, then v; head h
@@ -172,13 +178,13 @@ chimera_status chimera_debug_set_root(chimera_ctx* ctx, const int32_t* roots);
 enum {
   CHIMERA_DBG_NODE_TOKENS = 1,    /* int32 [batch][N] tree tokens of the last step */
   CHIMERA_DBG_VERIFY_LOGITS = 2,  /* f32 [batch][N][V] */
-  CHIMERA_DBG_VERIFY_HIDDEN = 3,  /* dtype [batch][N][d] post final norm */
+  CHIMERA_DBG_VERIFY_HIDDEN = 3,  /* f32 [batch][N][d] post final norm (H_LLM rows) */
   CHIMERA_DBG_ARGMAX = 4,         /* int32 [batch][N] */
   CHIMERA_DBG_PATH = 5,           /* int32 [batch][depth+1] accepted node indices */
   CHIMERA_DBG_ACCEPT_LEN = 6,     /* int32 [batch] L (drafted tokens accepted) */
   CHIMERA_DBG_DRAFT_LOGITS = 7,   /* f32 [K][batch][V] residual-head scores */
   CHIMERA_DBG_TOPK = 8,           /* int32 [batch][K][kmax] */
-  CHIMERA_DBG_HFULL = 9,          /* dtype [K][batch][d] full-context outputs */
+  CHIMERA_DBG_HFULL = 9,          /* f32 [K][batch][d] full-context outputs */
   CHIMERA_DBG_N = 10,             /* int32 [batch] committed length n */
   CHIMERA_DBG_TOKENS = 11,        /* int32 [batch][max_seq_len + 1] token history */
   CHIMERA_DBG_PREFILL_LOGITS = 12 /* f32 [batch][V] LM-head scores of the last prompt row
@@ -189,32 +195,34 @@ chimera_status chimera_debug_read(chimera_ctx* ctx, int what, void* host_dst, si
 
 /* Gather KV rows [pos0, pos0+count) of sequence `seq` from the paged cache of base
  * layer `layer` (layer = -1: the draft block's cache) into host buffers
- * k_dst / v_dst of shape [count][H][hd] (dtype of the model). */
+ * k_dst / v_dst of shape [count][H][hd] (fp32 when the caches are fp32, else bf16). */
 chimera_status chimera_debug_read_kv(chimera_ctx* ctx, int layer, int seq, int pos0, int count,
                                      void* k_dst, void* v_dst);
 
 /* ---- kernel-level entry points (stateless; for per-kernel parity tests) ---- */
 
-/* Y[M][N] (epilogue)= X[M][K] . W[N][K]^T on the given stream (NULL: default).
- * dtype 1: X, W bf16 (K, ldx multiples of 8; X, W 16-byte aligned), tcgen05 kernel;
- * dtype 0: everything fp32.  epi 0: Y = acc, 1: Y = SiLU(acc), 2: Y(fp32) += acc.
- * out_f32 selects an fp32 Y for epi 0/1 with dtype 1.  Device pointers.  Uses a
- * per-process workspace allocated on first use. */
+/* Y[M][N] (epilogue)= (X + X_lo)[M][K] . W[N][K]^T on the given stream (NULL: default).
+ * dtype 1: X, X_lo (optional, NULL = none), W bf16 (K, ldx multiples of 8; 16-byte
+ * aligned), tcgen05 kernel; dtype 0: everything fp32, X_lo ignored.  epi 0: Y = acc,
+ * 1: Y = SiLU(acc), 2: Y(fp32) += acc.  out_f32 selects an fp32 Y for epi 0/1 with
+ * dtype 1.  Device pointers.  Uses a per-process workspace allocated on first use. */
 chimera_status chimera_op_linear(int dtype, int epi, int out_f32, int M, int N, int K,
-                                 const void* X, int ldx, const void* W, void* Y, int ldy,
-                                 void* cuda_stream);
+                                 const void* X, const void* X_lo, int ldx, const void* W, void* Y,
+                                 int ldy, void* cuda_stream);
 
-/* Tree-masked attention over a paged KV pool [blocks][H][2][16][hd] (device):
- * q [batch*q_rows][ldq] rotated queries, query i of sequence b at row b*q_rows+i;
+/* Tree-masked attention over a paged KV pool [blocks][H][2][16][hd] (device; fp32
+ * when dtype == 0 or kv_f32, else bf16): q fp32 [batch*q_rows][ldq] rotated queries,
+ * query i of sequence b at row b*q_rows+i;
  * n_ctx (device int32 [batch]) committed rows visible to all; n_local rows follow at
  * slots n_ctx..; query i sees local row j iff bit j of anc[q_local0+i] (device
- * uint64); page_table device int32 [batch][max_pages]; out [batch*q_rows][ldo].
- * nq <= 64, n_local <= 64, hd in {64, 128}. */
-chimera_status chimera_op_attention(int dtype, int batch, int n_heads, int head_dim, int nq,
-                                    int q_local0, int n_local, const void* q, int ldq, int q_rows,
-                                    const void* pool, const int32_t* page_table, int max_pages,
-                                    const int32_t* n_ctx, const uint64_t* anc, void* out, int ldo,
-                                    int splits, void* cuda_stream);
+ * uint64); page_table device int32 [batch][max_pages]; out [batch*q_rows][ldo] in the
+ * model dtype, out_lo (optional, bf16 only) its lo half.  nq <= 64, n_local <= 64,
+ * hd in {64, 128}. */
+chimera_status chimera_op_attention(int dtype, int kv_f32, int batch, int n_heads, int head_dim,
+                                    int nq, int q_local0, int n_local, const float* q, int ldq,
+                                    int q_rows, const void* pool, const int32_t* page_table,
+                                    int max_pages, const int32_t* n_ctx, const uint64_t* anc,
+                                    void* out, void* out_lo, int ldo, int splits, void* cuda_stream);
 
 #ifdef __cplusplus
 }

@@ -37,7 +37,7 @@ class Config(ctypes.Structure):
                 ("dtype", ctypes.c_int), ("rms_eps", ctypes.c_float), ("rope_theta", ctypes.c_float),
                 ("n_draft_heads", ctypes.c_int), ("tree_nodes", ctypes.c_int),
                 ("topk", ctypes.c_int * 8), ("max_batch", ctypes.c_int), ("max_seq_len", ctypes.c_int),
-                ("kv_block", ctypes.c_int)]
+                ("kv_block", ctypes.c_int), ("precision", ctypes.c_int)]
 
 
 class BlockWeights(ctypes.Structure):
@@ -71,12 +71,14 @@ _SIGS = {
     "chimera_debug_read": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p, ctypes.c_size_t]),
     "chimera_debug_read_kv": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                                              ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p]),
-    "chimera_op_linear": (ctypes.c_int, [ctypes.c_int] * 6 + [ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p,
-                                                              ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p]),
-    "chimera_op_attention": (ctypes.c_int, [ctypes.c_int] * 7 + [ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
+    "chimera_op_linear": (ctypes.c_int, [ctypes.c_int] * 6 + [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int,
+                                                              ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int,
+                                                              ctypes.c_void_p]),
+    "chimera_op_attention": (ctypes.c_int, [ctypes.c_int] * 8 + [ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
                                                                  ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int,
                                                                  ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
-                                                                 ctypes.c_int, ctypes.c_int, ctypes.c_void_p]),
+                                                                 ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
+                                                                 ctypes.c_void_p]),
 }
 
 
@@ -107,7 +109,8 @@ def _stream_handle(stream) -> int:
     return int(stream.cuda_stream)
 
 
-def make_config(cfg: dict, max_batch: int | None = None, max_seq_len: int | None = None) -> Config:
+def make_config(cfg: dict, max_batch: int | None = None, max_seq_len: int | None = None,
+                precision: int | None = None) -> Config:
     c = Config()
     c.n_layers, c.d_model, c.n_heads = cfg["n_layers"], cfg["d_model"], cfg["n_heads"]
     c.head_dim, c.ffn_dim, c.vocab = cfg["head_dim"], cfg["ffn_dim"], cfg["vocab"]
@@ -119,6 +122,7 @@ def make_config(cfg: dict, max_batch: int | None = None, max_seq_len: int | None
     c.max_batch = max_batch or cfg["batch"]
     c.max_seq_len = max_seq_len or cfg.get("max_seq_len", 4096)
     c.kv_block = 16
+    c.precision = cfg.get("precision", 1) if precision is None else precision
     return c
 
 
@@ -127,11 +131,12 @@ class Chimera:
     captured step graph live in the library."""
 
     def __init__(self, cfg: dict, weights: dict, max_batch: int | None = None,
-                 max_seq_len: int | None = None, stream=None):
+                 max_seq_len: int | None = None, stream=None, precision: int | None = None):
         self.lib = load()
         self.cfg = cfg
         self._w = weights
-        self.c = make_config(cfg, max_batch, max_seq_len)
+        self.c = make_config(cfg, max_batch, max_seq_len, precision)
+        self.kv_f32 = cfg["dtype"] == "fp32" or self.c.precision == 1
         L, K = cfg["n_layers"], cfg["n_draft_heads"]
 
         def block(prefix):
@@ -236,10 +241,10 @@ class Chimera:
         kmax = max(cfg["topk"])
         fdt = torch.float32 if cfg["dtype"] == "fp32" else torch.bfloat16
         shapes = dict(node_tokens=((B, N), torch.int32), verify_logits=((B, N, V), torch.float32),
-                      verify_hidden=((B, N, d), fdt), argmax=((B, N), torch.int32),
+                      verify_hidden=((B, N, d), torch.float32), argmax=((B, N), torch.int32),
                       path=((B, self.depth + 1), torch.int32), accept_len=((B,), torch.int32),
                       draft_logits=((K, B, V), torch.float32), topk=((B, K, kmax), torch.int32),
-                      hfull=((K, B, d), fdt), n=((B,), torch.int32),
+                      hfull=((K, B, d), torch.float32), n=((B,), torch.int32),
                       tokens=((B, self.c.max_seq_len + 1), torch.int32),
                       prefill_logits=((B, V), torch.float32))
         shape, dt = shapes[what]
@@ -250,7 +255,7 @@ class Chimera:
     def read_kv(self, layer: int, seq: int, pos0: int, count: int):
         import torch
         cfg = self.cfg
-        dt = torch.float32 if cfg["dtype"] == "fp32" else torch.bfloat16
+        dt = torch.float32 if self.kv_f32 else torch.bfloat16
         k = torch.empty((count, cfg["n_heads"], cfg["head_dim"]), dtype=dt)
         v = torch.empty_like(k)
         self._check(self.lib.chimera_debug_read_kv(self.h, layer, seq, pos0, count, k.data_ptr(), v.data_ptr()))
@@ -258,26 +263,29 @@ class Chimera:
 
 
 # ---- kernel-level entry points ----
-def op_linear(X, W, Y, epi: int = 0, out_f32: bool = False, M=None, N=None, K=None, stream=None):
-    """Y (epilogue)= X W^T through chimera_op_linear (X [M][K], W [N][K], Y [M][N] device tensors)."""
+def op_linear(X, W, Y, epi: int = 0, out_f32: bool = False, X_lo=None, stream=None):
+    """Y (epilogue)= (X + X_lo) W^T through chimera_op_linear (X, X_lo [M][K], W [N][K],
+    Y [M][N] device tensors)."""
     lib = load()
-    M = M or X.shape[0]
-    K = K or X.shape[1]
-    N = N or W.shape[0]
-    dtype = 0 if X.dtype.is_floating_point and X.element_size() == 4 else 1
-    st = lib.chimera_op_linear(dtype, epi, int(out_f32), M, N, K, _ptr(X), X.stride(0), _ptr(W), _ptr(Y),
-                               Y.stride(0), _stream_handle(stream))
+    M, K = X.shape
+    N = W.shape[0]
+    dtype = 0 if X.element_size() == 4 else 1
+    st = lib.chimera_op_linear(dtype, epi, int(out_f32), M, N, K, _ptr(X), _ptr(X_lo), X.stride(0), _ptr(W),
+                               _ptr(Y), Y.stride(0), _stream_handle(stream))
     if st != 0:
         raise ChimeraError(st, "chimera_op_linear")
 
 
 def op_attention(q, pool, page_table, n_ctx, anc, out, nq, q_local0, n_local, q_rows, n_heads, head_dim,
-                 splits=1, stream=None):
+                 splits=1, out_lo=None, stream=None):
+    """Tree-masked paged attention through chimera_op_attention (q fp32; pool fp32 or
+    bf16; out fp32 for an fp32 model, else bf16 with an optional lo half)."""
     lib = load()
-    dtype = 0 if q.element_size() == 4 else 1
-    st = lib.chimera_op_attention(dtype, n_ctx.shape[0], n_heads, head_dim, nq, q_local0, n_local, _ptr(q),
-                                  q.stride(0), q_rows, _ptr(pool), _ptr(page_table), page_table.shape[1],
-                                  _ptr(n_ctx), _ptr(anc), _ptr(out), out.stride(0), splits,
+    dtype = 0 if out.element_size() == 4 else 1
+    kv_f32 = int(pool.element_size() == 4)
+    st = lib.chimera_op_attention(dtype, kv_f32, n_ctx.shape[0], n_heads, head_dim, nq, q_local0, n_local,
+                                  _ptr(q), q.stride(0), q_rows, _ptr(pool), _ptr(page_table), page_table.shape[1],
+                                  _ptr(n_ctx), _ptr(anc), _ptr(out), _ptr(out_lo), out.stride(0), splits,
                                   _stream_handle(stream))
     if st != 0:
         raise ChimeraError(st, "chimera_op_attention")

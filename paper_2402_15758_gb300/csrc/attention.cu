@@ -33,7 +33,7 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
-template <typename T, int HD>
+template <typename TKV, typename T, int HD>
 __global__ void __launch_bounds__(WARPS * 32) attn_kernel(const AttnParams p) {
   constexpr int DPL = HD / 32;
   extern __shared__ float sm[];
@@ -52,12 +52,12 @@ __global__ void __launch_bounds__(WARPS * 32) attn_kernel(const AttnParams p) {
   const int tps = (ntiles + p.splits - 1) / p.splits;
   const int t0 = s * tps;
   const int t1 = min(ntiles, t0 + tps);
-  const T* q = static_cast<const T*>(p.q);
-  const T* pool = static_cast<const T*>(p.pool) + static_cast<size_t>(p.layer) * p.pool_layer_stride;
+  const float* q = p.q;
+  const TKV* pool = static_cast<const TKV*>(p.pool) + static_cast<size_t>(p.layer) * p.pool_layer_stride;
 
   for (int idx = threadIdx.x; idx < nq * HD; idx += blockDim.x) {
     const int i = idx / HD, dd = idx % HD;
-    Qs[idx] = to_f(q[static_cast<size_t>(b * p.q_rows + i) * p.ldq + h * HD + dd]);
+    Qs[idx] = q[static_cast<size_t>(b * p.q_rows + i) * p.ldq + h * HD + dd];
   }
 
   float m[QPW], l[QPW], acc[QPW][DPL];
@@ -80,7 +80,7 @@ __global__ void __launch_bounds__(WARPS * 32) attn_kernel(const AttnParams p) {
       float kv = 0.f, vv = 0.f;
       if (key < total) {
         const int page = p.page_table[b * p.max_pages + (key >> 4)];
-        const T* base = pool + (static_cast<size_t>(page) * p.H + h) * 2 * 16 * HD;
+        const TKV* base = pool + (static_cast<size_t>(page) * p.H + h) * 2 * 16 * HD;
         kv = to_f(base[(key & 15) * HD + dd]);
         vv = to_f(base[16 * HD + (key & 15) * HD + dd]);
       }
@@ -120,6 +120,7 @@ __global__ void __launch_bounds__(WARPS * 32) attn_kernel(const AttnParams p) {
   }
 
   T* out = static_cast<T*>(p.out);
+  T* out_lo = static_cast<T*>(p.out_lo);
   if (p.splits == 1) {
 #pragma unroll
     for (int qq = 0; qq < QPW; ++qq) {
@@ -128,8 +129,8 @@ __global__ void __launch_bounds__(WARPS * 32) attn_kernel(const AttnParams p) {
         const float inv = l[qq] > 0.f ? 1.f / l[qq] : 0.f;
 #pragma unroll
         for (int r = 0; r < DPL; ++r)
-          out[static_cast<size_t>(b * p.q_rows + qi) * p.ldo + h * HD + lane + 32 * r] =
-              from_f<T>(acc[qq][r] * inv);
+          store_act(out, out_lo, static_cast<size_t>(b * p.q_rows + qi) * p.ldo + h * HD + lane + 32 * r,
+                    acc[qq][r] * inv);
       }
     }
     return;
@@ -180,21 +181,21 @@ __global__ void __launch_bounds__(WARPS * 32) attn_kernel(const AttnParams p) {
     const float inv = L > 0.f ? 1.f / L : 0.f;
 #pragma unroll
     for (int r = 0; r < DPL; ++r)
-      out[static_cast<size_t>(b * p.q_rows + qi) * p.ldo + h * HD + lane + 32 * r] = from_f<T>(o[r] * inv);
+      store_act(out, out_lo, static_cast<size_t>(b * p.q_rows + qi) * p.ldo + h * HD + lane + 32 * r, o[r] * inv);
   }
   if (threadIdx.x == 0) p.counters[b * p.H + h] = 0;
 }
 
-template <typename T, int HD>
+template <typename TKV, typename T, int HD>
 cudaError_t launch(const AttnParams& p, cudaStream_t s) {
   const size_t smem = (KT * (HD + 1) + KT * HD + static_cast<size_t>(p.nq_max) * HD) * sizeof(float);
   static bool attr = false;
   if (!attr) {
-    cudaFuncSetAttribute(attn_kernel<T, HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+    cudaFuncSetAttribute(attn_kernel<TKV, T, HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
     attr = true;
   }
   dim3 grid(p.splits, p.H, p.B);
-  attn_kernel<T, HD><<<grid, WARPS * 32, smem, s>>>(p);
+  attn_kernel<TKV, T, HD><<<grid, WARPS * 32, smem, s>>>(p);
   return cudaGetLastError();
 }
 
@@ -204,14 +205,17 @@ size_t attn_ws_floats(int B, int H, int splits, int nq_max, int hd) {
   return static_cast<size_t>(B) * H * splits * nq_max * (hd + 2);
 }
 
-cudaError_t attention(const AttnParams& p, int dtype, cudaStream_t s) {
+cudaError_t attention(const AttnParams& p, int dtype, int kv_f32, cudaStream_t s) {
   if (p.nq_max > WARPS * QPW || p.n_local > 64) return cudaErrorInvalidValue;
   if (dtype == 0) {
-    if (p.hd == 64) return launch<float, 64>(p, s);
-    if (p.hd == 128) return launch<float, 128>(p, s);
+    if (p.hd == 64) return launch<float, float, 64>(p, s);
+    if (p.hd == 128) return launch<float, float, 128>(p, s);
+  } else if (kv_f32) {
+    if (p.hd == 64) return launch<float, bf16, 64>(p, s);
+    if (p.hd == 128) return launch<float, bf16, 128>(p, s);
   } else {
-    if (p.hd == 64) return launch<bf16, 64>(p, s);
-    if (p.hd == 128) return launch<bf16, 128>(p, s);
+    if (p.hd == 64) return launch<bf16, bf16, 64>(p, s);
+    if (p.hd == 128) return launch<bf16, bf16, 128>(p, s);
   }
   return cudaErrorInvalidValue;
 }

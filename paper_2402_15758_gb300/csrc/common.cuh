@@ -35,6 +35,16 @@ template <> __device__ __forceinline__ bf16 from_f<bf16>(float v) { return __flo
 
 __device__ __forceinline__ float silu_f(float x) { return x / (1.0f + expf(-x)); }
 
+// Store an activation that feeds a tensor-core GEMM.  bf16 models keep a two-term
+// split x = hi + lo (both bf16, lo = the rounding residual of hi) when `lo` is given,
+// so a pair of bf16 MMAs with fp32 accumulation reproduces x to ~2^-16.
+__device__ __forceinline__ void store_act(float* hi, float* /*lo*/, size_t i, float x) { hi[i] = x; }
+__device__ __forceinline__ void store_act(bf16* hi, bf16* lo, size_t i, float x) {
+  const bf16 h = __float2bfloat16_rn(x);
+  hi[i] = h;
+  if (lo) lo[i] = __float2bfloat16_rn(x - __bfloat162float(h));
+}
+
 __device__ __forceinline__ uint64_t global_timer_ns() {
   uint64_t t;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));

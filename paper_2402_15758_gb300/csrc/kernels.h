@@ -13,6 +13,8 @@ namespace chimera {
 struct TcLinearParams {
   CUtensorMap tmA;   // W: [N][K] bf16, box 128 x 64, 128-byte swizzle
   CUtensorMap tmB;   // X: [M][K] bf16 (row pitch ldx), box BN x 64, 128-byte swizzle
+  CUtensorMap tmB2;  // X_lo (same shape) when the activation is a hi + lo split
+  int has_lo;        // 1: two MMAs per K slice, W.X_hi + W.X_lo into one accumulator
   int M, N, K;
   int BN;            // token tile = UMMA N (multiple of 16, <= 256)
   int tok_tiles, feat_tiles, kblocks;
@@ -21,6 +23,7 @@ struct TcLinearParams {
   int epi;           // EPI_*
   int out_f32;       // Y is fp32 (else bf16) for EPI_STORE / EPI_SILU
   void* Y;
+  void* Y2;          // optional bf16 lo half of Y (EPI_STORE / EPI_SILU, bf16 Y)
   int ldy;
   float* ws;         // split partials: [grid][2][128 * BN] fp32
   int* counters;     // [feat_tiles * tok_tiles], all zero between launches
@@ -44,9 +47,9 @@ int tc_max_tiles();
 // Encode the plan for one call site.  X/W/Y are device pointers; ws/counters are
 // scratch owned by the caller (sizes from tc_ws_floats / tc_max_tiles).
 // Returns 0 on success, otherwise a negative code and a message in `msg`.
-int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, int ldx, const void* W,
-                   void* Y, int ldy, int epi, int out_f32, float* ws, int* counters, int* err,
-                   char* msg, size_t msg_len);
+int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, const void* X_lo, int ldx,
+                   const void* W, void* Y, void* Y_lo, int ldy, int epi, int out_f32, float* ws,
+                   int* counters, int* err, char* msg, size_t msg_len);
 cudaError_t tc_linear_launch(const TcLinearPlan& plan, cudaStream_t s);
 
 // ----------------------------------------------------------------------------
@@ -59,7 +62,7 @@ cudaError_t f32_linear(int M, int N, int K, const float* X, int ldx, const float
 // attention over the paged KV cache with a per-query ancestor bitmask
 // ----------------------------------------------------------------------------
 struct AttnParams {
-  const void* q;          // rotated queries, row (b * q_rows + i), head h at col h*hd
+  const float* q;         // rotated fp32 queries, row (b * q_rows + i), head h at col h*hd
   int ldq, q_rows;
   int nq;                 // queries per sequence
   const int* nq_dev;      // optional per-sequence query count (overrides nq when set)
@@ -73,7 +76,8 @@ struct AttnParams {
   const int* page_table;  // [B][max_pages]
   int max_pages;
   const int* n_ctx;       // [B] committed rows (all visible)
-  void* out;              // [b * q_rows + i][H * hd]
+  void* out;              // [b * q_rows + i][H * hd] (model dtype)
+  void* out_lo;           // optional lo half (bf16 split activations)
   int ldo;
   int B, H, hd;
   float scale;
@@ -82,20 +86,22 @@ struct AttnParams {
   int* counters;          // [B][H], zero between launches
   int nq_max;
 };
-cudaError_t attention(const AttnParams& p, int dtype, cudaStream_t s);
+// dtype: 0 fp32 model; 1 bf16 model.  kv_f32: the KV pool holds fp32 (else bf16).
+cudaError_t attention(const AttnParams& p, int dtype, int kv_f32, cudaStream_t s);
 size_t attn_ws_floats(int B, int H, int splits, int nq_max, int hd);
 
 // ----------------------------------------------------------------------------
 // row-wise / small kernels
 // ----------------------------------------------------------------------------
-cudaError_t rmsnorm(int dtype, int in_f32, const void* X, int ldx, const void* g, void* Y, int ldy,
-                    int rows, int d, float eps, cudaStream_t s);
+// Y (model dtype, plus the optional lo half) and an optional fp32 copy Y32.
+cudaError_t rmsnorm(int dtype, const float* X, int ldx, const void* g, void* Y, void* Y_lo, float* Y32,
+                    int ldy, int rows, int d, float eps, cudaStream_t s);
 
 struct RopeKvParams {
-  const void* qkv;   // [rows][ldqkv]
+  const float* qkv;  // [rows][ldqkv] fp32 projections
   int ldqkv;
   int q_col, k_col, v_col;  // column offsets (q_col < 0: no query output)
-  void* q_out;       // [rows][H*hd]
+  float* q_out;      // [rows][H*hd] fp32
   int ldq;
   void* pool;
   long long pool_layer_stride;
@@ -113,9 +119,9 @@ struct RopeKvParams {
   int B, H, hd;
   int* err;
 };
-cudaError_t rope_kv(const RopeKvParams& p, int dtype, cudaStream_t s);
+cudaError_t rope_kv(const RopeKvParams& p, int kv_f32, cudaStream_t s);
 
-cudaError_t swiglu(int dtype, const void* gu, int ldgu, int F, void* h, int ldh, int rows,
+cudaError_t swiglu(int dtype, const float* gu, int ldgu, int F, void* h, void* h_lo, int ldh, int rows,
                    cudaStream_t s);
 
 // x[r][:] = E[tok(r)] with tok(r) = tokens[r] (mode 0) or tok_hist[b][n[b]+i] for

@@ -46,19 +46,31 @@ __device__ __forceinline__ long long unit_begin(int c, long long U, int G) {
   return static_cast<long long>(c) * U / G;
 }
 
-__device__ __forceinline__ void epi_apply(const TcLinearParams& p, int m, int f, float v) {
-  if (m >= p.M || f >= p.N) return;
-  const size_t idx = static_cast<size_t>(m) * p.ldy + f;
+// Epilogue of 16 consecutive token columns (m0 .. m0+15) of feature row f.  All
+// loads are issued before the stores so they overlap.
+__device__ __forceinline__ void epi_store16(const TcLinearParams& p, int m0, int f, const float (&v)[16]) {
+  if (f >= p.N) return;
   if (p.epi == EPI_RESID) {
     float* y = static_cast<float*>(p.Y);
-    y[idx] += v;
+    float old[16];
+#pragma unroll
+    for (int j = 0; j < 16; ++j)
+      old[j] = (m0 + j < p.M) ? y[static_cast<size_t>(m0 + j) * p.ldy + f] : 0.f;
+#pragma unroll
+    for (int j = 0; j < 16; ++j)
+      if (m0 + j < p.M) y[static_cast<size_t>(m0 + j) * p.ldy + f] = old[j] + v[j];
     return;
   }
-  if (p.epi == EPI_SILU) v = silu_f(v);
-  if (p.out_f32)
-    static_cast<float*>(p.Y)[idx] = v;
-  else
-    static_cast<bf16*>(p.Y)[idx] = __float2bfloat16_rn(v);
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    if (m0 + j >= p.M) break;
+    const float x = (p.epi == EPI_SILU) ? silu_f(v[j]) : v[j];
+    const size_t idx = static_cast<size_t>(m0 + j) * p.ldy + f;
+    if (p.out_f32)
+      static_cast<float*>(p.Y)[idx] = x;
+    else
+      store_act(static_cast<bf16*>(p.Y), static_cast<bf16*>(p.Y2), idx, x);
+  }
 }
 
 __device__ __forceinline__ bool bar_any(int id, int nthreads, bool pred) {
@@ -86,7 +98,8 @@ __global__ void __launch_bounds__(THREADS, 1) tc_linear_kernel(const __grid_cons
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  const int stage_bytes = BM * BK * 2 + p.BN * BK * 2;
+  const int b_bytes = p.BN * BK * 2;
+  const int stage_bytes = BM * BK * 2 + (p.has_lo ? 2 : 1) * b_bytes;
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + p.stages * stage_bytes);
   uint64_t* empty = full + MAX_STAGES;
   uint64_t* tfull = empty + MAX_STAGES;
@@ -116,6 +129,7 @@ __global__ void __launch_bounds__(THREADS, 1) tc_linear_kernel(const __grid_cons
   if (warp == 0 && lane == 0) {
     prefetch_tensormap(&p.tmA);
     prefetch_tensormap(&p.tmB);
+    if (p.has_lo) prefetch_tensormap(&p.tmB2);
   }
   if (warp == 1) tmem_alloc(tmem_slot, p.tmem_cols);
   tc_fence_before();
@@ -150,6 +164,7 @@ __global__ void __launch_bounds__(THREADS, 1) tc_linear_kernel(const __grid_cons
           mbar_arrive_expect_tx(&full[stage], static_cast<uint32_t>(stage_bytes));
           tma_load_2d_hint(sa, &p.tmA, kb * BK, ft * BM, &full[stage], pol_w);
           tma_load_2d(sb, &p.tmB, kb * BK, tt * p.BN, &full[stage]);
+          if (p.has_lo) tma_load_2d(sb + b_bytes, &p.tmB2, kb * BK, tt * p.BN, &full[stage]);
           issued_mask |= 1u << stage;
           issued_par = (issued_par & ~(1u << stage)) | (phase << stage);
           if (++stage == p.stages) {
@@ -186,8 +201,9 @@ __global__ void __launch_bounds__(THREADS, 1) tc_linear_kernel(const __grid_cons
           const uint32_t sb = sa + BM * BK * 2;
 #pragma unroll
           for (int k = 0; k < BK / UK; ++k) {
-            tc_mma_bf16(d_tmem, sw128_desc(sa + k * 32), sw128_desc(sb + k * 32), idesc,
-                        (first && k == 0) ? 0u : 1u);
+            const uint64_t adesc = sw128_desc(sa + k * 32);
+            tc_mma_bf16(d_tmem, adesc, sw128_desc(sb + k * 32), idesc, (first && k == 0) ? 0u : 1u);
+            if (p.has_lo) tc_mma_bf16(d_tmem, adesc, sw128_desc(sb + b_bytes + k * 32), idesc, 1u);
           }
           first = false;
           tc_commit(&empty[stage]);
@@ -231,8 +247,7 @@ __global__ void __launch_bounds__(THREADS, 1) tc_linear_kernel(const __grid_cons
         for (int c0 = 0; c0 < p.BN; c0 += 16) {
           float v[16];
           tmem_ld_16(tbase + c0, v);
-#pragma unroll
-          for (int j = 0; j < 16; ++j) epi_apply(p, m0 + c0 + j, f, v[j]);
+          epi_store16(p, m0 + c0, f, v);
         }
         tc_fence_before();
         mbar_arrive(&tempty[buf]);
@@ -256,14 +271,33 @@ __global__ void __launch_bounds__(THREADS, 1) tc_linear_kernel(const __grid_cons
         named_bar(1, 128);
         if (*s_last) {
           __threadfence();
-          for (int col = 0; col < p.BN; ++col) {
-            if (m0 + col >= p.M) break;
-            float acc = 0.f;
-            for (int cc = c_first; cc <= c_last; ++cc) {
-              const int sl = 2 * cc + ((unit_begin(cc, U, G) / KB == t) ? 0 : 1);
-              acc += __ldcg(&p.ws[static_cast<size_t>(sl) * BM * p.BN + col * BM + row]);
+          for (int c0 = 0; c0 < p.BN; c0 += 16) {
+            if (m0 + c0 >= p.M) break;
+            float acc[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) acc[j] = 0.f;
+            // partials summed in contributor order (deterministic); up to four
+            // contributors' loads in flight at once
+            for (int cc = c_first; cc <= c_last; cc += 4) {
+              float v[4][16];
+#pragma unroll
+              for (int q4 = 0; q4 < 4; ++q4) {
+                if (cc + q4 <= c_last) {
+                  const int c2 = cc + q4;
+                  const int sl = 2 * c2 + ((unit_begin(c2, U, G) / KB == t) ? 0 : 1);
+                  const float* src = p.ws + static_cast<size_t>(sl) * BM * p.BN + static_cast<size_t>(c0) * BM + row;
+#pragma unroll
+                  for (int j = 0; j < 16; ++j) v[q4][j] = __ldcg(src + j * BM);
+                }
+              }
+#pragma unroll
+              for (int q4 = 0; q4 < 4; ++q4)
+                if (cc + q4 <= c_last) {
+#pragma unroll
+                  for (int j = 0; j < 16; ++j) acc[j] += v[q4][j];
+                }
             }
-            epi_apply(p, m0 + col, f, acc);
+            epi_store16(p, m0 + c0, f, acc);
           }
           if (threadIdx.x == 64) p.counters[t] = 0;
         }
@@ -340,9 +374,9 @@ size_t tc_ws_floats(int max_bn) {
 
 int tc_max_tiles() { return MAX_TILES; }
 
-int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, int ldx, const void* W,
-                   void* Y, int ldy, int epi, int out_f32, float* ws, int* counters, int* err,
-                   char* msg, size_t msg_len) {
+int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, const void* X_lo, int ldx,
+                   const void* W, void* Y, void* Y_lo, int ldy, int epi, int out_f32, float* ws,
+                   int* counters, int* err, char* msg, size_t msg_len) {
   auto fail = [&](const char* m) {
     if (msg && msg_len) snprintf(msg, msg_len, "linear(M=%d,N=%d,K=%d): %s", M, N, K, m);
     return -1;
@@ -350,8 +384,9 @@ int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, int l
   if (M < 1 || N < 1 || K < 8) return fail("empty or too-small shape");
   if (K % 8 != 0 || ldx % 8 != 0) return fail("K and the row pitch of X must be multiples of 8");
   if (ldx < K || ldy < N) return fail("row pitch smaller than the row");
-  if ((reinterpret_cast<uintptr_t>(X) & 15) || (reinterpret_cast<uintptr_t>(W) & 15))
-    return fail("X and W must be 16-byte aligned");
+  if ((reinterpret_cast<uintptr_t>(X) & 15) || (reinterpret_cast<uintptr_t>(W) & 15) ||
+      (reinterpret_cast<uintptr_t>(X_lo) & 15))
+    return fail("X, X_lo and W must be 16-byte aligned");
   if (epi == EPI_RESID && !out_f32) return fail("residual epilogue needs an fp32 output");
   TcLinearParams& p = plan->p;
   memset(&p, 0, sizeof(p));
@@ -364,13 +399,15 @@ int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, int l
   p.kblocks = (K + BK - 1) / BK;
   if (static_cast<long long>(p.feat_tiles) * p.tok_tiles > MAX_TILES) return fail("too many tiles");
   p.units = static_cast<long long>(p.feat_tiles) * p.tok_tiles * p.kblocks;
-  const int stage_bytes = BM * BK * 2 + p.BN * BK * 2;
+  p.has_lo = X_lo ? 1 : 0;
+  const int stage_bytes = BM * BK * 2 + (p.has_lo ? 2 : 1) * p.BN * BK * 2;
   p.stages = PIPE_SMEM / stage_bytes;
   if (p.stages > MAX_STAGES) p.stages = MAX_STAGES;
   if (p.stages < 2) return fail("token tile too large");
   p.epi = epi;
   p.out_f32 = out_f32;
   p.Y = Y;
+  p.Y2 = out_f32 ? nullptr : Y_lo;
   p.ldy = ldy;
   p.ws = ws;
   p.counters = counters;
@@ -381,6 +418,7 @@ int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, int l
   if (p.tmem_cols > 512) return fail("accumulators exceed tensor memory");
   if (encode_2d_bf16(&p.tmA, W, K, N, K, BK, BM) != 0) return fail("tensor map of W");
   if (encode_2d_bf16(&p.tmB, X, K, M, ldx, BK, p.BN) != 0) return fail("tensor map of X");
+  if (X_lo && encode_2d_bf16(&p.tmB2, X_lo, K, M, ldx, BK, p.BN) != 0) return fail("tensor map of X_lo");
   const int sms = tc_num_sms();
   plan->grid = static_cast<int>(p.units < sms ? p.units : sms);
   plan->smem = 1024 + static_cast<size_t>(p.stages) * stage_bytes + 2 * MAX_STAGES * 8 + 5 * 8 + 64;

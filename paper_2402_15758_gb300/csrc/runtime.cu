@@ -135,7 +135,10 @@ struct chimera_ctx {
   chimera_config cfg;
   int L = 0, d = 0, H = 0, hd = 0, F = 0, V = 0, K = 0, N = 0, KMAX = 0, D1 = 0, Bmax = 0, cap = 0;
   int dtype = 0;
-  size_t esz = 4;
+  size_t esz = 4;      // weights / GEMM operands
+  int split = 0;       // bf16 GEMM operands kept as hi + lo pairs
+  int kv_f32 = 0;      // KV pools hold fp32
+  size_t kv_esz = 4;
   cudaStream_t stream = nullptr;
   bool own_stream = false;
   int num_sms = 1;
@@ -168,7 +171,10 @@ struct chimera_ctx {
   long long kv_layer_stride = 0;  // elements
   int NB = 0, max_pages = 0;
   int* d_pt = nullptr;
-  std::vector<int> h_pt;
+  int* h_pt = nullptr;  // pinned mirror of the page table
+  size_t h_pt_len = 0;
+  cudaEvent_t pt_event = nullptr;  // last upload of h_pt
+  bool pt_inflight = false;
   std::vector<std::vector<int>> seq_blocks;
   std::vector<int> free_blocks;
   bool pt_dirty = false;
@@ -178,9 +184,15 @@ struct chimera_ctx {
   // activations
   int R = 0;
   float* x = nullptr;
-  void *xn = nullptr, *qkv = nullptr, *qr = nullptr, *ao = nullptr, *gu = nullptr, *hf = nullptr, *hfin = nullptr;
+  // GEMM operands in the model dtype; *_lo = the bf16 rounding residuals (split mode)
+  void *xn = nullptr, *xn_lo = nullptr, *ao = nullptr, *ao_lo = nullptr, *hf = nullptr, *hf_lo = nullptr;
+  void *hfin = nullptr, *hfin_lo = nullptr;
+  float* hfin32 = nullptr;              // post-final-norm hidden states (H_LLM), fp32
+  float* qr = nullptr;                  // rotated queries, fp32
+  float *qkv = nullptr, *gu = nullptr;  // fp32 GEMM outputs feeding RoPE / SwiGLU
   float* logits = nullptr;
-  void *tbuf = nullptr, *ubuf = nullptr, *headin = nullptr, *hfull_log = nullptr, *hsel = nullptr, *kvtmp = nullptr;
+  void *tbuf = nullptr, *ubuf = nullptr, *ubuf_lo = nullptr, *headin = nullptr, *headin_lo = nullptr;
+  float *hfull_log = nullptr, *hsel = nullptr, *kvtmp = nullptr;
   float *dres = nullptr, *hlog = nullptr;
 
   // scratch of the split kernels
@@ -208,6 +220,8 @@ struct chimera_ctx {
   bool prof = false;
   std::vector<ProfEvent> prof_ev;
   size_t prof_used = 0;
+  cudaGraphExec_t prof_graph = nullptr;  // the step with an event pair around every launch
+  size_t prof_count = 0;
   int cur_phase = 0;
 
   std::string err;
@@ -262,10 +276,11 @@ struct Scope {
     ev->kind = kind;
     ev->phase = c->cur_phase;
     ev->bytes = bytes;
-    cudaEventRecord(ev->a, c->stream);
+    // recorded inside a stream capture: external records become event nodes
+    cudaEventRecordWithFlags(ev->a, c->stream, cudaEventRecordExternal);
   }
   ~Scope() {
-    if (ev) cudaEventRecord(ev->b, c->stream);
+    if (ev) cudaEventRecordWithFlags(ev->b, c->stream, cudaEventRecordExternal);
   }
 };
 
@@ -276,8 +291,8 @@ cudaError_t run_lin(chimera_ctx* ctx, const Lin& l) {
                     static_cast<float*>(l.Y), l.ldy, l.epi, ctx->stream);
 }
 
-bool make_lin(chimera_ctx* ctx, Lin* l, int M, int N, int K, const void* X, int ldx, const void* W, void* Y,
-              int ldy, int epi, int out_f32) {
+bool make_lin(chimera_ctx* ctx, Lin* l, int M, int N, int K, const void* X, const void* X_lo, int ldx,
+              const void* W, void* Y, void* Y_lo, int ldy, int epi, int out_f32) {
   l->M = M;
   l->N = N;
   l->K = K;
@@ -292,8 +307,8 @@ bool make_lin(chimera_ctx* ctx, Lin* l, int M, int N, int K, const void* X, int 
   l->tc = ctx->dtype == 1;
   if (!l->tc) return true;
   char msg[256];
-  if (tc_linear_plan(&l->tp, M, N, K, X, ldx, W, Y, ldy, epi, out_f32, ctx->lin_ws, ctx->lin_cnt, ctx->d_err, msg,
-                     sizeof(msg)) != 0) {
+  if (tc_linear_plan(&l->tp, M, N, K, X, X_lo, ldx, W, Y, Y_lo, ldy, epi, out_f32, ctx->lin_ws, ctx->lin_cnt,
+                     ctx->d_err, msg, sizeof(msg)) != 0) {
     ctx->err = msg;
     return false;
   }
@@ -327,6 +342,7 @@ cudaError_t run_attention(chimera_ctx* ctx, bool draft_pool, int layer, int nq, 
   p.max_pages = ctx->max_pages;
   p.n_ctx = ctx->d_n;
   p.out = ctx->ao;
+  p.out_lo = ctx->ao_lo;
   p.ldo = ctx->d;
   p.B = ctx->batch;
   p.H = ctx->H;
@@ -337,10 +353,10 @@ cudaError_t run_attention(chimera_ctx* ctx, bool draft_pool, int layer, int nq, 
   p.counters = ctx->att_cnt;
   p.nq_max = nq_max;
   if (attn_ws_floats(p.B, p.H, splits, nq_max, p.hd) > ctx->att_ws_floats) return cudaErrorInvalidValue;
-  return attention(p, ctx->dtype, ctx->stream);
+  return attention(p, ctx->dtype, ctx->kv_f32, ctx->stream);
 }
 
-cudaError_t run_rope(chimera_ctx* ctx, bool draft_pool, int layer, const void* src, int ldsrc, int q_col, int k_col,
+cudaError_t run_rope(chimera_ctx* ctx, bool draft_pool, int layer, const float* src, int ldsrc, int q_col, int k_col,
                      int v_col, int rows_per_seq, const int* valid, int valid_plus, int pos_base, int slot_base,
                      const int* pos_off) {
   Scope sc(ctx, CHIMERA_KIND_ROPE_KV, 0);
@@ -370,13 +386,21 @@ cudaError_t run_rope(chimera_ctx* ctx, bool draft_pool, int layer, const void* s
   p.H = ctx->H;
   p.hd = ctx->hd;
   p.err = ctx->d_err;
-  return rope_kv(p, ctx->dtype, ctx->stream);
+  return rope_kv(p, ctx->kv_f32, ctx->stream);
 }
 
-cudaError_t run_norm(chimera_ctx* ctx, int in_f32, const void* X, int ldx, const void* g, void* Y, int ldy,
-                     int rows) {
+// RMSNorm of fp32 rows into the GEMM operand buffer xn (+ lo half).
+cudaError_t run_norm(chimera_ctx* ctx, const float* X, const void* g, int rows) {
   Scope sc(ctx, CHIMERA_KIND_NORM, 0);
-  return rmsnorm(ctx->dtype, in_f32, X, ldx, g, Y, ldy, rows, ctx->d, ctx->cfg.rms_eps, ctx->stream);
+  return rmsnorm(ctx->dtype, X, ctx->d, g, ctx->xn, ctx->xn_lo, nullptr, ctx->d, rows, ctx->d, ctx->cfg.rms_eps,
+                 ctx->stream);
+}
+
+// Final norm: H_LLM rows in fp32 plus the LM-head operand (+ lo half).
+cudaError_t run_final_norm(chimera_ctx* ctx, int rows) {
+  Scope sc(ctx, CHIMERA_KIND_NORM, 0);
+  return rmsnorm(ctx->dtype, ctx->x, ctx->d, ctx->final_norm, ctx->hfin, ctx->hfin_lo, ctx->hfin32, ctx->d, rows,
+                 ctx->d, ctx->cfg.rms_eps, ctx->stream);
 }
 
 #define RUN(call)                                            \
@@ -394,18 +418,18 @@ cudaError_t enqueue_layer(chimera_ctx* ctx, int l, const Lin* lin, int rows, int
                           const int* pos_off, const unsigned long long* anc, int splits, double kv_bytes) {
   const chimera_block_weights& w = ctx->layers[l];
   const int d = ctx->d;
-  RUN(run_norm(ctx, 1, ctx->x, d, w.attn_norm, ctx->xn, d, rows));
+  RUN(run_norm(ctx, ctx->x, w.attn_norm, rows));
   RUN(run_lin(ctx, lin[0]));
   RUN(run_rope(ctx, false, l, ctx->qkv, 3 * d, 0, d, 2 * d, rows_per_seq, valid, 0, 0, 0, pos_off));
   RUN(run_attention(ctx, false, l, rows_per_seq, valid, 0, rows_per_seq, valid, anc, rows_per_seq, splits,
                     rows_per_seq, kv_bytes));
   RUN(run_lin(ctx, lin[1]));
-  RUN(run_norm(ctx, 1, ctx->x, d, w.ffn_norm, ctx->xn, d, rows));
+  RUN(run_norm(ctx, ctx->x, w.ffn_norm, rows));
   RUN(run_lin(ctx, lin[2]));
   RUN(run_lin(ctx, lin[3]));
   {
     Scope sc(ctx, CHIMERA_KIND_SWIGLU, 0);
-    RUN(swiglu(ctx->dtype, ctx->gu, 2 * ctx->F, ctx->F, ctx->hf, ctx->F, rows, ctx->stream));
+    RUN(swiglu(ctx->dtype, ctx->gu, 2 * ctx->F, ctx->F, ctx->hf, ctx->hf_lo, ctx->F, rows, ctx->stream));
   }
   RUN(run_lin(ctx, lin[4]));
   return cudaSuccess;
@@ -414,7 +438,8 @@ cudaError_t enqueue_layer(chimera_ctx* ctx, int l, const Lin* lin, int rows, int
 double kv_read_bytes(const chimera_ctx* ctx, int extra_rows, bool draft) {
   double rows = 0;
   for (int b = 0; b < ctx->batch; ++b) rows += ctx->host_n[b] + extra_rows;
-  return rows * 2.0 * ctx->d * ctx->esz * (draft ? 1 : 1);
+  (void)draft;
+  return rows * 2.0 * ctx->d * ctx->kv_esz;
 }
 
 // The whole step on the context stream (graph-capturable: every dynamic value is read
@@ -433,24 +458,24 @@ cudaError_t enqueue_step(chimera_ctx* ctx) {
     }
     RUN(run_lin(ctx, ctx->tri1));
     RUN(run_lin(ctx, ctx->tri2));
-    RUN(run_norm(ctx, 1, ctx->dres, d, ctx->draft.attn_norm, ctx->xn, d, B));
+    RUN(run_norm(ctx, ctx->dres, ctx->draft.attn_norm, B));
     RUN(run_lin(ctx, ctx->dqkv));
     RUN(run_rope(ctx, true, 0, ctx->qkv, 3 * d, 0, d, 2 * d, 1, nullptr, 0, k, k, nullptr));
     RUN(run_attention(ctx, true, 0, 1, nullptr, k, k + 1, nullptr, ctx->d_chain, 1, ctx->att_splits_draft, 1,
                       kv_read_bytes(ctx, k + 1, true)));
     RUN(run_lin(ctx, ctx->dwo));
-    RUN(run_norm(ctx, 1, ctx->dres, d, ctx->draft.ffn_norm, ctx->xn, d, B));
+    RUN(run_norm(ctx, ctx->dres, ctx->draft.ffn_norm, B));
     RUN(run_lin(ctx, ctx->dgate));
     RUN(run_lin(ctx, ctx->dup));
     {
       Scope sc(ctx, CHIMERA_KIND_SWIGLU, 0);
-      RUN(swiglu(ctx->dtype, ctx->gu, 2 * ctx->F, ctx->F, ctx->hf, ctx->F, B, s));
+      RUN(swiglu(ctx->dtype, ctx->gu, 2 * ctx->F, ctx->F, ctx->hf, ctx->hf_lo, ctx->F, B, s));
     }
     RUN(run_lin(ctx, ctx->ddown));
     {
       Scope sc(ctx, CHIMERA_KIND_OTHER, 0);
-      RUN(launch_hfull_store(ctx->dtype, ctx->dres, d, ctx->headin, eoff(ctx, ctx->hfull_log, static_cast<size_t>(k) * B * d),
-                             B, s));
+      RUN(launch_hfull_store(ctx->dtype, ctx->dres, d, ctx->headin, ctx->headin_lo,
+                             ctx->hfull_log + static_cast<size_t>(k) * B * d, B, s));
     }
     RUN(run_lin(ctx, ctx->dhead[k]));
     {
@@ -475,7 +500,7 @@ cudaError_t enqueue_step(chimera_ctx* ctx) {
   const double kvb = kv_read_bytes(ctx, N, false);
   for (int l = 0; l < ctx->L; ++l)
     RUN(enqueue_layer(ctx, l, &ctx->ver[5 * l], B * N, N, nullptr, ctx->d_depth, ctx->d_anc, ctx->att_splits_ver, kvb));
-  RUN(run_norm(ctx, 1, ctx->x, d, ctx->final_norm, ctx->hfin, d, B * N));
+  RUN(run_final_norm(ctx, B * N));
   RUN(run_lin(ctx, ctx->ver_lm));
   {
     Scope sc(ctx, CHIMERA_KIND_ARGMAX, 0);
@@ -490,15 +515,16 @@ cudaError_t enqueue_step(chimera_ctx* ctx) {
   }
   {
     Scope sc(ctx, CHIMERA_KIND_COMPACT, 0);
-    RUN(launch_compact(ctx->kv, ctx->kv_layer_stride * static_cast<long long>(ctx->esz), ctx->L, ctx->H,
-                       static_cast<int>(ctx->hd * ctx->esz), ctx->d_n, ctx->d_path, ctx->d_L, ctx->D1, ctx->d_pt,
+    RUN(launch_compact(ctx->kv, ctx->kv_layer_stride * static_cast<long long>(ctx->kv_esz), ctx->L, ctx->H,
+                       static_cast<int>(ctx->hd * ctx->kv_esz), ctx->d_n, ctx->d_path, ctx->d_L, ctx->D1, ctx->d_pt,
                        ctx->max_pages, B, s));
   }
   {
     Scope sc(ctx, CHIMERA_KIND_OTHER, 0);
-    RUN(launch_gather_hidden(ctx->dtype, ctx->hfin, d, N, ctx->d_path, ctx->d_L, ctx->D1, ctx->hsel, ctx->headin, B, s));
+    RUN(launch_gather_hidden(ctx->dtype, ctx->hfin32, d, N, ctx->d_path, ctx->d_L, ctx->D1, ctx->hsel, ctx->headin,
+                             ctx->headin_lo, B, s));
   }
-  RUN(run_norm(ctx, ctx->dtype == 0 ? 1 : 0, ctx->hsel, d, ctx->draft.attn_norm, ctx->xn, d, B * ctx->D1));
+  RUN(run_norm(ctx, ctx->hsel, ctx->draft.attn_norm, B * ctx->D1));
   RUN(run_lin(ctx, ctx->commit_kv));
   RUN(run_rope(ctx, true, 0, ctx->kvtmp, 2 * d, -1, 0, d, ctx->D1, ctx->d_L, 1, 0, 0, nullptr));
   {
@@ -515,39 +541,49 @@ bool build_plans(chimera_ctx* ctx, int B) {
   const int f32 = 1, tb = ctx->dtype == 0 ? 1 : 0;  // bf16 storage -> out_f32 = 0
   ctx->ver.assign(5 * ctx->L, Lin());
   ctx->pre.assign(5 * ctx->L, Lin());
+  void *xn = ctx->xn, *xl = ctx->xn_lo, *ao = ctx->ao, *al = ctx->ao_lo, *hf = ctx->hf, *hl = ctx->hf_lo;
   auto layer_plans = [&](std::vector<Lin>& v, int M) {
     for (int l = 0; l < ctx->L; ++l) {
       const chimera_block_weights& w = ctx->layers[l];
       Lin* p = &v[5 * l];
-      if (!make_lin(ctx, &p[0], M, 3 * d, d, ctx->xn, d, w.wqkv, ctx->qkv, 3 * d, EPI_STORE, tb)) return false;
-      if (!make_lin(ctx, &p[1], M, d, d, ctx->ao, d, w.wo, ctx->x, d, EPI_RESID, f32)) return false;
-      if (!make_lin(ctx, &p[2], M, F, d, ctx->xn, d, w.w_gate, ctx->gu, 2 * F, EPI_STORE, tb)) return false;
-      if (!make_lin(ctx, &p[3], M, F, d, ctx->xn, d, w.w_up, eoff(ctx, ctx->gu, F), 2 * F, EPI_STORE, tb)) return false;
-      if (!make_lin(ctx, &p[4], M, d, F, ctx->hf, F, w.w_down, ctx->x, d, EPI_RESID, f32)) return false;
+      if (!make_lin(ctx, &p[0], M, 3 * d, d, xn, xl, d, w.wqkv, ctx->qkv, nullptr, 3 * d, EPI_STORE, f32)) return false;
+      if (!make_lin(ctx, &p[1], M, d, d, ao, al, d, w.wo, ctx->x, nullptr, d, EPI_RESID, f32)) return false;
+      if (!make_lin(ctx, &p[2], M, F, d, xn, xl, d, w.w_gate, ctx->gu, nullptr, 2 * F, EPI_STORE, f32)) return false;
+      if (!make_lin(ctx, &p[3], M, F, d, xn, xl, d, w.w_up, ctx->gu + F, nullptr, 2 * F, EPI_STORE, f32)) return false;
+      if (!make_lin(ctx, &p[4], M, d, F, hf, hl, F, w.w_down, ctx->x, nullptr, d, EPI_RESID, f32)) return false;
     }
     return true;
   };
   if (!layer_plans(ctx->ver, B * N)) return false;
   if (!layer_plans(ctx->pre, B * CHUNK)) return false;
-  if (!make_lin(ctx, &ctx->ver_lm, B * N, V, d, ctx->hfin, d, ctx->lm_head, ctx->logits, V, EPI_STORE, f32)) return false;
-  if (!make_lin(ctx, &ctx->pre_lm, B, V, d, ctx->headin, 2 * d, ctx->lm_head, ctx->logits, V, EPI_STORE, f32)) return false;
-  const void* dl_kv = eoff(ctx, const_cast<void*>(ctx->draft.wqkv), static_cast<size_t>(d) * d);
-  if (!make_lin(ctx, &ctx->pre_dkv, B * CHUNK, 2 * d, d, ctx->xn, d, dl_kv, ctx->kvtmp, 2 * d, EPI_STORE, tb)) return false;
-  if (!make_lin(ctx, &ctx->commit_kv, B * ctx->D1, 2 * d, d, ctx->xn, d, dl_kv, ctx->kvtmp, 2 * d, EPI_STORE, tb))
+  if (!make_lin(ctx, &ctx->ver_lm, B * N, V, d, ctx->hfin, ctx->hfin_lo, d, ctx->lm_head, ctx->logits, nullptr, V,
+                EPI_STORE, f32))
     return false;
-  // draft (M = B rows)
-  if (!make_lin(ctx, &ctx->tri1, B, d, 3 * d, ctx->tbuf, 3 * d, ctx->tri_w1, ctx->ubuf, d, EPI_SILU, tb)) return false;
-  if (!make_lin(ctx, &ctx->tri2, B, d, d, ctx->ubuf, d, ctx->tri_w2, ctx->dres, d, EPI_STORE, f32)) return false;
+  if (!make_lin(ctx, &ctx->pre_lm, B, V, d, ctx->headin, ctx->headin_lo, 2 * d, ctx->lm_head, ctx->logits, nullptr, V,
+                EPI_STORE, f32))
+    return false;
+  const void* dl_kv = eoff(ctx, const_cast<void*>(ctx->draft.wqkv), static_cast<size_t>(d) * d);
+  if (!make_lin(ctx, &ctx->pre_dkv, B * CHUNK, 2 * d, d, xn, xl, d, dl_kv, ctx->kvtmp, nullptr, 2 * d, EPI_STORE, f32))
+    return false;
+  if (!make_lin(ctx, &ctx->commit_kv, B * ctx->D1, 2 * d, d, xn, xl, d, dl_kv, ctx->kvtmp, nullptr, 2 * d, EPI_STORE,
+                f32))
+    return false;
+  // draft (M = B rows); the trigram input is a gather of bf16 embeddings: exact, no lo half
+  if (!make_lin(ctx, &ctx->tri1, B, d, 3 * d, ctx->tbuf, nullptr, 3 * d, ctx->tri_w1, ctx->ubuf, ctx->ubuf_lo, d,
+                EPI_SILU, tb))
+    return false;
+  if (!make_lin(ctx, &ctx->tri2, B, d, d, ctx->ubuf, ctx->ubuf_lo, d, ctx->tri_w2, ctx->dres, nullptr, d, EPI_STORE, f32))
+    return false;
   const chimera_block_weights& w = ctx->draft;
-  if (!make_lin(ctx, &ctx->dqkv, B, 3 * d, d, ctx->xn, d, w.wqkv, ctx->qkv, 3 * d, EPI_STORE, tb)) return false;
-  if (!make_lin(ctx, &ctx->dwo, B, d, d, ctx->ao, d, w.wo, ctx->dres, d, EPI_RESID, f32)) return false;
-  if (!make_lin(ctx, &ctx->dgate, B, F, d, ctx->xn, d, w.w_gate, ctx->gu, 2 * F, EPI_STORE, tb)) return false;
-  if (!make_lin(ctx, &ctx->dup, B, F, d, ctx->xn, d, w.w_up, eoff(ctx, ctx->gu, F), 2 * F, EPI_STORE, tb)) return false;
-  if (!make_lin(ctx, &ctx->ddown, B, d, F, ctx->hf, F, w.w_down, ctx->dres, d, EPI_RESID, f32)) return false;
+  if (!make_lin(ctx, &ctx->dqkv, B, 3 * d, d, xn, xl, d, w.wqkv, ctx->qkv, nullptr, 3 * d, EPI_STORE, f32)) return false;
+  if (!make_lin(ctx, &ctx->dwo, B, d, d, ao, al, d, w.wo, ctx->dres, nullptr, d, EPI_RESID, f32)) return false;
+  if (!make_lin(ctx, &ctx->dgate, B, F, d, xn, xl, d, w.w_gate, ctx->gu, nullptr, 2 * F, EPI_STORE, f32)) return false;
+  if (!make_lin(ctx, &ctx->dup, B, F, d, xn, xl, d, w.w_up, ctx->gu + F, nullptr, 2 * F, EPI_STORE, f32)) return false;
+  if (!make_lin(ctx, &ctx->ddown, B, d, F, hf, hl, F, w.w_down, ctx->dres, nullptr, d, EPI_RESID, f32)) return false;
   ctx->dhead.assign(ctx->K, Lin());
   for (int k = 0; k < ctx->K; ++k)
-    if (!make_lin(ctx, &ctx->dhead[k], B, V, 2 * d, ctx->headin, 2 * d, ctx->heads[k],
-                  ctx->hlog + static_cast<size_t>(k) * B * V, V, EPI_STORE, f32))
+    if (!make_lin(ctx, &ctx->dhead[k], B, V, 2 * d, ctx->headin, ctx->headin_lo, 2 * d, ctx->heads[k],
+                  ctx->hlog + static_cast<size_t>(k) * B * V, nullptr, V, EPI_STORE, f32))
       return false;
   ctx->att_splits_ver = att_splits(ctx, B);
   ctx->att_splits_pre = att_splits(ctx, B);
@@ -555,7 +591,16 @@ bool build_plans(chimera_ctx* ctx, int B) {
   return true;
 }
 
+// The pinned mirror may still be read by the last upload: wait for it before editing.
+void pt_wait(chimera_ctx* ctx) {
+  if (ctx->pt_inflight) {
+    cudaEventSynchronize(ctx->pt_event);
+    ctx->pt_inflight = false;
+  }
+}
+
 chimera_status ensure_blocks(chimera_ctx* ctx, int b, int slots) {
+  pt_wait(ctx);
   if (slots > ctx->cap)
     return fail(ctx, CHIMERA_ECAPACITY, "sequence " + std::to_string(b) + " needs " + std::to_string(slots) +
                                             " KV slots > max_seq_len " + std::to_string(ctx->cap));
@@ -573,8 +618,9 @@ chimera_status ensure_blocks(chimera_ctx* ctx, int b, int slots) {
 
 chimera_status flush_page_table(chimera_ctx* ctx) {
   if (!ctx->pt_dirty) return CHIMERA_OK;
-  CK(cudaMemcpyAsync(ctx->d_pt, ctx->h_pt.data(), ctx->h_pt.size() * sizeof(int), cudaMemcpyHostToDevice, ctx->stream));
-  CK(cudaStreamSynchronize(ctx->stream));
+  CK(cudaMemcpyAsync(ctx->d_pt, ctx->h_pt, ctx->h_pt_len * sizeof(int), cudaMemcpyHostToDevice, ctx->stream));
+  CK(cudaEventRecord(ctx->pt_event, ctx->stream));
+  ctx->pt_inflight = true;
   ctx->pt_dirty = false;
   return CHIMERA_OK;
 }
@@ -656,12 +702,15 @@ chimera_status read_new_tokens(chimera_ctx* ctx, int32_t* out_tokens, int per_se
 void free_ctx(chimera_ctx* ctx) {
   if (!ctx) return;
   if (ctx->graph) cudaGraphExecDestroy(ctx->graph);
+  if (ctx->prof_graph) cudaGraphExecDestroy(ctx->prof_graph);
   for (auto& e : ctx->prof_ev) {
     cudaEventDestroy(e.a);
     cudaEventDestroy(e.b);
   }
   for (void* p : ctx->allocs) cudaFree(p);
   if (ctx->h_stage) cudaFreeHost(ctx->h_stage);
+  if (ctx->h_pt) cudaFreeHost(ctx->h_pt);
+  if (ctx->pt_event) cudaEventDestroy(ctx->pt_event);
   if (ctx->own_stream && ctx->stream) cudaStreamDestroy(ctx->stream);
   delete ctx;
 }
@@ -686,7 +735,8 @@ chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
   if (c.n_layers < 1 || c.d_model < 32 || c.n_heads < 1 || c.head_dim * c.n_heads != c.d_model ||
       (c.head_dim != 64 && c.head_dim != 128) || c.ffn_dim < 8 || c.vocab < 8 || (c.dtype != 0 && c.dtype != 1) ||
       c.n_draft_heads < 1 || c.n_draft_heads > 4 || c.tree_nodes < 2 || c.tree_nodes > 64 || c.max_batch < 1 ||
-      c.max_batch > 64 || c.kv_block != 16 || c.max_seq_len < 32 || !(c.rms_eps > 0) || !(c.rope_theta > 0))
+      c.max_batch > 64 || c.kv_block != 16 || c.max_seq_len < 32 || !(c.rms_eps > 0) || !(c.rope_theta > 0) ||
+      (c.precision != 0 && c.precision != 1))
     return CHIMERA_EINVAL;
   if (c.dtype == 1 && (c.d_model % 64 != 0 || c.ffn_dim % 8 != 0)) return CHIMERA_EINVAL;
   for (int k = 0; k < c.n_draft_heads; ++k)
@@ -711,6 +761,9 @@ chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
   ctx->N = c.tree_nodes;
   ctx->dtype = c.dtype;
   ctx->esz = c.dtype == 0 ? 4 : 2;
+  ctx->split = (c.dtype == 1 && c.precision == 1) ? 1 : 0;
+  ctx->kv_f32 = (c.dtype == 0 || c.precision == 1) ? 1 : 0;
+  ctx->kv_esz = ctx->kv_f32 ? 4 : 2;
   ctx->Bmax = c.max_batch;
   ctx->cap = c.max_seq_len;
   ctx->KMAX = 1;
@@ -751,27 +804,36 @@ chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
   ctx->R = B * std::max(N, CHUNK);
   const int Rc = B * std::max(CHUNK, ctx->D1);
   bool ok = true;
-  ok = ok && dalloc_bytes(ctx, &ctx->kv, static_cast<size_t>(ctx->kv_layer_stride) * ctx->L * ctx->esz);
-  ok = ok && dalloc_bytes(ctx, &ctx->dkv, static_cast<size_t>(ctx->kv_layer_stride) * ctx->esz);
+  const size_t Rx = static_cast<size_t>(std::max(ctx->R, Rc));
+  const bool sp = ctx->split != 0;
+  ok = ok && dalloc_bytes(ctx, &ctx->kv, static_cast<size_t>(ctx->kv_layer_stride) * ctx->L * ctx->kv_esz);
+  ok = ok && dalloc_bytes(ctx, &ctx->dkv, static_cast<size_t>(ctx->kv_layer_stride) * ctx->kv_esz);
   ok = ok && dalloc(ctx, &ctx->d_pt, static_cast<size_t>(B) * ctx->max_pages);
   ok = ok && dalloc(ctx, &ctx->d_rope, static_cast<size_t>(ctx->max_pos) * (ctx->hd / 2));
   ok = ok && dalloc(ctx, &ctx->x, static_cast<size_t>(ctx->R) * d);
-  ok = ok && dalloc_bytes(ctx, &ctx->xn, static_cast<size_t>(std::max(ctx->R, Rc)) * d * ctx->esz);
-  ok = ok && dalloc_bytes(ctx, &ctx->qkv, static_cast<size_t>(ctx->R) * 3 * d * ctx->esz);
-  ok = ok && dalloc_bytes(ctx, &ctx->qr, static_cast<size_t>(ctx->R) * d * ctx->esz);
+  ok = ok && dalloc_bytes(ctx, &ctx->xn, Rx * d * ctx->esz);
+  if (sp) ok = ok && dalloc_bytes(ctx, &ctx->xn_lo, Rx * d * ctx->esz);
+  ok = ok && dalloc(ctx, &ctx->qkv, static_cast<size_t>(ctx->R) * 3 * d);
+  ok = ok && dalloc(ctx, &ctx->qr, static_cast<size_t>(ctx->R) * d);
   ok = ok && dalloc_bytes(ctx, &ctx->ao, static_cast<size_t>(ctx->R) * d * ctx->esz);
-  ok = ok && dalloc_bytes(ctx, &ctx->gu, static_cast<size_t>(ctx->R) * 2 * F * ctx->esz);
+  if (sp) ok = ok && dalloc_bytes(ctx, &ctx->ao_lo, static_cast<size_t>(ctx->R) * d * ctx->esz);
+  ok = ok && dalloc(ctx, &ctx->gu, static_cast<size_t>(ctx->R) * 2 * F);
   ok = ok && dalloc_bytes(ctx, &ctx->hf, static_cast<size_t>(ctx->R) * F * ctx->esz);
+  if (sp) ok = ok && dalloc_bytes(ctx, &ctx->hf_lo, static_cast<size_t>(ctx->R) * F * ctx->esz);
   ok = ok && dalloc_bytes(ctx, &ctx->hfin, static_cast<size_t>(ctx->R) * d * ctx->esz);
+  if (sp) ok = ok && dalloc_bytes(ctx, &ctx->hfin_lo, static_cast<size_t>(ctx->R) * d * ctx->esz);
+  ok = ok && dalloc(ctx, &ctx->hfin32, static_cast<size_t>(ctx->R) * d);
   ok = ok && dalloc(ctx, &ctx->logits, static_cast<size_t>(B) * N * V);
   ok = ok && dalloc_bytes(ctx, &ctx->tbuf, static_cast<size_t>(B) * 3 * d * ctx->esz);
   ok = ok && dalloc_bytes(ctx, &ctx->ubuf, static_cast<size_t>(B) * d * ctx->esz);
+  if (sp) ok = ok && dalloc_bytes(ctx, &ctx->ubuf_lo, static_cast<size_t>(B) * d * ctx->esz);
   ok = ok && dalloc(ctx, &ctx->dres, static_cast<size_t>(B) * d);
   ok = ok && dalloc_bytes(ctx, &ctx->headin, static_cast<size_t>(B) * 2 * d * ctx->esz);
-  ok = ok && dalloc_bytes(ctx, &ctx->hfull_log, static_cast<size_t>(K) * B * d * ctx->esz);
+  if (sp) ok = ok && dalloc_bytes(ctx, &ctx->headin_lo, static_cast<size_t>(B) * 2 * d * ctx->esz);
+  ok = ok && dalloc(ctx, &ctx->hfull_log, static_cast<size_t>(K) * B * d);
   ok = ok && dalloc(ctx, &ctx->hlog, static_cast<size_t>(K) * B * V);
-  ok = ok && dalloc_bytes(ctx, &ctx->hsel, static_cast<size_t>(B) * ctx->D1 * d * ctx->esz);
-  ok = ok && dalloc_bytes(ctx, &ctx->kvtmp, static_cast<size_t>(Rc) * 2 * d * ctx->esz);
+  ok = ok && dalloc(ctx, &ctx->hsel, static_cast<size_t>(B) * ctx->D1 * d);
+  ok = ok && dalloc(ctx, &ctx->kvtmp, static_cast<size_t>(Rc) * 2 * d);
   ok = ok && dalloc(ctx, &ctx->d_n, B);
   ok = ok && dalloc(ctx, &ctx->d_tok, static_cast<size_t>(B) * ctx->tok_stride);
   ok = ok && dalloc(ctx, &ctx->d_node_tok, static_cast<size_t>(B) * N);
@@ -802,6 +864,9 @@ chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
   ok = ok && dalloc(ctx, &ctx->att_ws, ctx->att_ws_floats);
   ok = ok && dalloc(ctx, &ctx->att_cnt, static_cast<size_t>(B) * ctx->H);
   if (ok && cudaMallocHost(reinterpret_cast<void**>(&ctx->h_stage), 4096 * sizeof(int)) != cudaSuccess) ok = false;
+  ctx->h_pt_len = static_cast<size_t>(B) * ctx->max_pages;
+  if (ok && cudaMallocHost(reinterpret_cast<void**>(&ctx->h_pt), ctx->h_pt_len * sizeof(int)) != cudaSuccess) ok = false;
+  if (ok && cudaEventCreateWithFlags(&ctx->pt_event, cudaEventDisableTiming) != cudaSuccess) ok = false;
   if (!ok) {
     free_ctx(ctx);
     return CHIMERA_ENOMEM;
@@ -811,8 +876,8 @@ chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
   // zero-initialised state and scratch
   cudaStream_t s = ctx->stream;
   bool zok = true;
-  zok = zok && cudaMemsetAsync(ctx->kv, 0, static_cast<size_t>(ctx->kv_layer_stride) * ctx->L * ctx->esz, s) == cudaSuccess;
-  zok = zok && cudaMemsetAsync(ctx->dkv, 0, static_cast<size_t>(ctx->kv_layer_stride) * ctx->esz, s) == cudaSuccess;
+  zok = zok && cudaMemsetAsync(ctx->kv, 0, static_cast<size_t>(ctx->kv_layer_stride) * ctx->L * ctx->kv_esz, s) == cudaSuccess;
+  zok = zok && cudaMemsetAsync(ctx->dkv, 0, static_cast<size_t>(ctx->kv_layer_stride) * ctx->kv_esz, s) == cudaSuccess;
   zok = zok && cudaMemsetAsync(ctx->att_cnt, 0, static_cast<size_t>(B) * ctx->H * sizeof(int), s) == cudaSuccess;
   if (ctx->lin_cnt)
     zok = zok && cudaMemsetAsync(ctx->lin_cnt, 0, static_cast<size_t>(tc_max_tiles()) * sizeof(int), s) == cudaSuccess;
@@ -821,6 +886,8 @@ chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
   zok = zok && cudaMemsetAsync(ctx->d_step, 0, sizeof(int), s) == cudaSuccess;
   zok = zok && cudaMemsetAsync(ctx->d_topk, 0, static_cast<size_t>(B) * K * ctx->KMAX * sizeof(int), s) == cudaSuccess;
   zok = zok && cudaMemsetAsync(ctx->headin, 0, static_cast<size_t>(B) * 2 * d * ctx->esz, s) == cudaSuccess;
+  if (ctx->headin_lo)
+    zok = zok && cudaMemsetAsync(ctx->headin_lo, 0, static_cast<size_t>(B) * 2 * d * ctx->esz, s) == cudaSuccess;
   zok = zok && cudaMemsetAsync(ctx->x, 0, static_cast<size_t>(ctx->R) * d * sizeof(float), s) == cudaSuccess;
 
   // tree, chain masks and the RoPE table (fp64 on the host, rounded to fp32)
@@ -848,7 +915,7 @@ chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
     free_ctx(ctx);
     return CHIMERA_ECUDA;
   }
-  ctx->h_pt.assign(static_cast<size_t>(B) * ctx->max_pages, 0);
+  std::fill(ctx->h_pt, ctx->h_pt + ctx->h_pt_len, 0);
   ctx->seq_blocks.assign(B, {});
   ctx->free_blocks.clear();
   for (int i = ctx->NB - 1; i >= 0; --i) ctx->free_blocks.push_back(i);
@@ -874,15 +941,20 @@ chimera_status chimera_prefill(chimera_ctx* ctx, int batch, const int32_t* token
 
   // reset: free every block, rebuild plans for this batch, drop the step graph
   ctx->prefilled = false;
+  pt_wait(ctx);
   for (auto& blocks : ctx->seq_blocks) {
     for (int blk : blocks) ctx->free_blocks.push_back(blk);
     blocks.clear();
   }
-  std::fill(ctx->h_pt.begin(), ctx->h_pt.end(), 0);
+  std::fill(ctx->h_pt, ctx->h_pt + ctx->h_pt_len, 0);
   ctx->pt_dirty = true;
   if (ctx->graph) {
     cudaGraphExecDestroy(ctx->graph);
     ctx->graph = nullptr;
+  }
+  if (ctx->prof_graph) {
+    cudaGraphExecDestroy(ctx->prof_graph);
+    ctx->prof_graph = nullptr;
   }
   ctx->batch = batch;
   if (!build_plans(ctx, batch)) return CHIMERA_EINVAL;
@@ -927,12 +999,13 @@ chimera_status chimera_prefill(chimera_ctx* ctx, int batch, const int32_t* token
     for (int l = 0; l < ctx->L; ++l)
       CK(enqueue_layer(ctx, l, &ctx->pre[5 * l], B * CHUNK, CHUNK, ctx->d_valid, nullptr, ctx->d_chain,
                        ctx->att_splits_pre, 0));
-    CK(rmsnorm(ctx->dtype, 1, ctx->x, d, ctx->final_norm, ctx->hfin, d, B * CHUNK, d, ctx->cfg.rms_eps, s));
+    CK(run_final_norm(ctx, B * CHUNK));
     // draft-layer K/V of the chunk's H_LLM rows
-    CK(rmsnorm(ctx->dtype, ctx->dtype == 0 ? 1 : 0, ctx->hfin, d, dl_norm, ctx->xn, d, B * CHUNK, d, ctx->cfg.rms_eps, s));
+    CK(run_norm(ctx, ctx->hfin32, dl_norm, B * CHUNK));
     CK(run_lin(ctx, ctx->pre_dkv));
     CK(run_rope(ctx, true, 0, ctx->kvtmp, 2 * d, -1, 0, d, CHUNK, ctx->d_valid, 0, 0, 0, nullptr));
-    CK(launch_prefill_advance(ctx->dtype, ctx->hfin, d, CHUNK, ctx->d_valid, ctx->d_last, ctx->d_n, ctx->headin, B, s));
+    CK(launch_prefill_advance(ctx->dtype, ctx->hfin32, d, CHUNK, ctx->d_valid, ctx->d_last, ctx->d_n, ctx->headin,
+                              ctx->headin_lo, B, s));
     CK(cudaStreamSynchronize(s));  // the staging buffer is reused by the next chunk
   }
   // root = greedy next token of each prompt (eq. 1)
@@ -1011,13 +1084,36 @@ chimera_status chimera_profile_step(chimera_ctx* ctx, int max, int32_t* kinds, i
   if (!count) return fail(ctx, CHIMERA_EINVAL, "NULL count");
   chimera_status st = steps_prepare(ctx, 1);
   if (st != CHIMERA_OK) return st;
-  ctx->prof = true;
-  ctx->prof_used = 0;
-  cudaError_t e = enqueue_step(ctx);
-  ctx->prof = false;
-  if (e != cudaSuccess) return fail(ctx, CHIMERA_ECUDA, std::string("profiled step: ") + cudaGetErrorString(e));
+  if (!ctx->prof_graph) {
+    ctx->prof_ev.reserve(8192);
+    ctx->prof = true;
+    ctx->prof_used = 0;
+    cudaGraph_t g = nullptr;
+    CK(cudaStreamBeginCapture(ctx->stream, cudaStreamCaptureModeThreadLocal));
+    cudaError_t e = enqueue_step(ctx);
+    cudaError_t e2 = cudaStreamEndCapture(ctx->stream, &g);
+    ctx->prof = false;
+    if (e != cudaSuccess || e2 != cudaSuccess) {
+      if (g) cudaGraphDestroy(g);
+      return fail(ctx, CHIMERA_ECUDA, std::string("capturing the profiled step: ") +
+                                          cudaGetErrorString(e != cudaSuccess ? e : e2));
+    }
+    e = cudaGraphInstantiate(&ctx->prof_graph, g, 0);
+    cudaGraphDestroy(g);
+    if (e != cudaSuccess) return fail(ctx, CHIMERA_ECUDA, std::string("instantiating: ") + cudaGetErrorString(e));
+    ctx->prof_count = ctx->prof_used;
+  }
+  if (ctx->ovr_pending) {
+    const int one = 1;
+    CK(cudaMemcpyAsync(ctx->d_ovr_flag, &one, sizeof(int), cudaMemcpyHostToDevice, ctx->stream));
+  }
+  CK(cudaGraphLaunch(ctx->prof_graph, ctx->stream));
+  if (ctx->ovr_pending) {
+    CK(cudaMemsetAsync(ctx->d_ovr_flag, 0, sizeof(int), ctx->stream));
+    ctx->ovr_pending = false;
+  }
   CK(cudaStreamSynchronize(ctx->stream));
-  const int n = static_cast<int>(ctx->prof_used);
+  const int n = static_cast<int>(ctx->prof_count);
   for (int i = 0; i < n && i < max; ++i) {
     float t = 0;
     cudaEventElapsedTime(&t, ctx->prof_ev[i].a, ctx->prof_ev[i].b);
@@ -1064,13 +1160,13 @@ chimera_status chimera_debug_read(chimera_ctx* ctx, int what, void* dst, size_t 
   switch (what) {
     case CHIMERA_DBG_NODE_TOKENS: src = ctx->d_node_tok; need = B * N * 4; break;
     case CHIMERA_DBG_VERIFY_LOGITS: src = ctx->logits; need = B * N * V * 4; break;
-    case CHIMERA_DBG_VERIFY_HIDDEN: src = ctx->hfin; need = B * N * d * ctx->esz; break;
+    case CHIMERA_DBG_VERIFY_HIDDEN: src = ctx->hfin32; need = B * N * d * 4; break;
     case CHIMERA_DBG_ARGMAX: src = ctx->d_amax; need = B * N * 4; break;
     case CHIMERA_DBG_PATH: src = ctx->d_path; need = B * ctx->D1 * 4; break;
     case CHIMERA_DBG_ACCEPT_LEN: src = ctx->d_L; need = B * 4; break;
     case CHIMERA_DBG_DRAFT_LOGITS: src = ctx->hlog; need = K * B * V * 4; break;
     case CHIMERA_DBG_TOPK: src = ctx->d_topk; need = B * K * ctx->KMAX * 4; break;
-    case CHIMERA_DBG_HFULL: src = ctx->hfull_log; need = K * B * d * ctx->esz; break;
+    case CHIMERA_DBG_HFULL: src = ctx->hfull_log; need = K * B * d * 4; break;
     case CHIMERA_DBG_N: src = ctx->d_n; need = B * 4; break;
     case CHIMERA_DBG_TOKENS: src = ctx->d_tok; need = B * ctx->tok_stride * 4; break;
     case CHIMERA_DBG_PREFILL_LOGITS: src = ctx->logits; need = B * V * 4; break;
@@ -1090,9 +1186,9 @@ chimera_status chimera_debug_read_kv(chimera_ctx* ctx, int layer, int seq, int p
       pos0 + count > static_cast<int>(ctx->seq_blocks[seq].size()) * 16 || !k_dst || !v_dst)
     return fail(ctx, CHIMERA_EINVAL, "bad KV read");
   CK(cudaStreamSynchronize(ctx->stream));
-  const size_t row = static_cast<size_t>(ctx->hd) * ctx->esz;
+  const size_t row = static_cast<size_t>(ctx->hd) * ctx->kv_esz;
   const char* pool = static_cast<const char*>(layer < 0 ? ctx->dkv : ctx->kv) +
-                     (layer < 0 ? 0 : static_cast<size_t>(layer) * ctx->kv_layer_stride * ctx->esz);
+                     (layer < 0 ? 0 : static_cast<size_t>(layer) * ctx->kv_layer_stride * ctx->kv_esz);
   for (int i = 0; i < count; ++i) {
     const int slot = pos0 + i;
     const int page = ctx->h_pt[seq * ctx->max_pages + slot / 16];
@@ -1144,8 +1240,8 @@ bool op_scratch() {
 }
 }  // namespace
 
-chimera_status chimera_op_linear(int dtype, int epi, int out_f32, int M, int N, int K, const void* X, int ldx,
-                                 const void* W, void* Y, int ldy, void* cuda_stream) {
+chimera_status chimera_op_linear(int dtype, int epi, int out_f32, int M, int N, int K, const void* X,
+                                 const void* X_lo, int ldx, const void* W, void* Y, int ldy, void* cuda_stream) {
   if ((dtype != 0 && dtype != 1) || epi < 0 || epi > 2 || M < 1 || N < 1 || K < 1 || !X || !W || !Y || ldx < K ||
       ldy < N)
     return CHIMERA_EINVAL;
@@ -1158,16 +1254,16 @@ chimera_status chimera_op_linear(int dtype, int epi, int out_f32, int M, int N, 
   if (!op_scratch()) return CHIMERA_ENOMEM;
   TcLinearPlan plan;
   char msg[256];
-  if (tc_linear_plan(&plan, M, N, K, X, ldx, W, Y, ldy, epi, epi == EPI_RESID ? 1 : out_f32, g_op.lin_ws, g_op.lin_cnt,
-                     g_op.err, msg, sizeof(msg)) != 0)
+  if (tc_linear_plan(&plan, M, N, K, X, X_lo, ldx, W, Y, nullptr, ldy, epi, epi == EPI_RESID ? 1 : out_f32, g_op.lin_ws,
+                     g_op.lin_cnt, g_op.err, msg, sizeof(msg)) != 0)
     return CHIMERA_EINVAL;
   return tc_linear_launch(plan, s) == cudaSuccess ? CHIMERA_OK : CHIMERA_ECUDA;
 }
 
-chimera_status chimera_op_attention(int dtype, int batch, int n_heads, int head_dim, int nq, int q_local0, int n_local,
-                                    const void* q, int ldq, int q_rows, const void* pool, const int32_t* page_table,
-                                    int max_pages, const int32_t* n_ctx, const uint64_t* anc, void* out, int ldo,
-                                    int splits, void* cuda_stream) {
+chimera_status chimera_op_attention(int dtype, int kv_f32, int batch, int n_heads, int head_dim, int nq, int q_local0,
+                                    int n_local, const float* q, int ldq, int q_rows, const void* pool,
+                                    const int32_t* page_table, int max_pages, const int32_t* n_ctx, const uint64_t* anc,
+                                    void* out, void* out_lo, int ldo, int splits, void* cuda_stream) {
   if ((dtype != 0 && dtype != 1) || batch < 1 || n_heads < 1 || (head_dim != 64 && head_dim != 128) || nq < 1 ||
       nq > 64 || n_local < 0 || n_local > 64 || q_local0 < 0 || !q || !pool || !page_table || !n_ctx || !anc || !out ||
       splits < 1 || splits > 64 || batch * n_heads > 64 * 256)
@@ -1187,6 +1283,7 @@ chimera_status chimera_op_attention(int dtype, int batch, int n_heads, int head_
   p.max_pages = max_pages;
   p.n_ctx = n_ctx;
   p.out = out;
+  p.out_lo = out_lo;
   p.ldo = ldo;
   p.B = batch;
   p.H = n_heads;
@@ -1197,7 +1294,9 @@ chimera_status chimera_op_attention(int dtype, int batch, int n_heads, int head_
   p.counters = g_op.att_cnt;
   p.nq_max = nq;
   if (attn_ws_floats(batch, n_heads, splits, nq, head_dim) > g_op.att_floats) return CHIMERA_EINVAL;
-  return attention(p, dtype, static_cast<cudaStream_t>(cuda_stream)) == cudaSuccess ? CHIMERA_OK : CHIMERA_ECUDA;
+  return attention(p, dtype, dtype == 0 ? 1 : kv_f32, static_cast<cudaStream_t>(cuda_stream)) == cudaSuccess
+             ? CHIMERA_OK
+             : CHIMERA_ECUDA;
 }
 
 }  // extern "C"

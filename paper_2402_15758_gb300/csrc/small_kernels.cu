@@ -28,24 +28,28 @@ __device__ float block_sum(float v, float* red) {
   return r;
 }
 
-// RMSNorm (Llama): y = x / sqrt(mean(x^2) + eps) * g.
-template <typename Tin, typename T>
-__global__ void rmsnorm_kernel(const Tin* __restrict__ X, int ldx, const T* __restrict__ g,
-                               T* __restrict__ Y, int ldy, int d, float eps) {
+// RMSNorm (Llama): y = x / sqrt(mean(x^2) + eps) * g, from the fp32 residual stream.
+// Writes the GEMM operand (model dtype, optional lo half) and an optional fp32 copy.
+template <typename T>
+__global__ void rmsnorm_kernel(const float* __restrict__ X, int ldx, const T* __restrict__ g,
+                               T* __restrict__ Y, T* __restrict__ Y_lo, float* __restrict__ Y32,
+                               int ldy, int d, float eps) {
   __shared__ float red[33];
-  const Tin* x = X + static_cast<size_t>(blockIdx.x) * ldx;
+  const float* x = X + static_cast<size_t>(blockIdx.x) * ldx;
   float ss = 0.f;
-  for (int i = threadIdx.x; i < d; i += blockDim.x) {
-    const float v = to_f(x[i]);
-    ss = fmaf(v, v, ss);
-  }
+  for (int i = threadIdx.x; i < d; i += blockDim.x) ss = fmaf(x[i], x[i], ss);
   ss = block_sum(ss, red);
   const float r = rsqrtf(ss / static_cast<float>(d) + eps);
-  T* y = Y + static_cast<size_t>(blockIdx.x) * ldy;
-  for (int i = threadIdx.x; i < d; i += blockDim.x) y[i] = from_f<T>(to_f(x[i]) * r * to_f(g[i]));
+  const size_t row = static_cast<size_t>(blockIdx.x) * ldy;
+  for (int i = threadIdx.x; i < d; i += blockDim.x) {
+    const float v = x[i] * r * to_f(g[i]);
+    store_act(Y, Y_lo, row + i, v);
+    if (Y32) Y32[row + i] = v;
+  }
 }
 
-// Rotate-half RoPE of q and k, plus the write of k and v into the paged cache.
+// Rotate-half RoPE of q and k, plus the write of k and v into the paged cache
+// (T = element type of the cache).
 template <typename T>
 __global__ void rope_kv_kernel(const RopeKvParams p) {
   const int row = blockIdx.x;
@@ -69,37 +73,38 @@ __global__ void rope_kv_kernel(const RopeKvParams p) {
       page = p.page_table[b * p.max_pages + pi];
     }
   }
-  const T* src = static_cast<const T*>(p.qkv) + static_cast<size_t>(row) * p.ldqkv;
+  const float* src = p.qkv + static_cast<size_t>(row) * p.ldqkv;
   T* pool = static_cast<T*>(p.pool) + static_cast<size_t>(p.layer) * p.pool_layer_stride;
   for (int idx = threadIdx.x; idx < p.H * half; idx += blockDim.x) {
     const int h = idx / half, j = idx % half;
     const float2 cs = p.rope[static_cast<size_t>(pos) * half + j];
     if (p.q_col >= 0) {
-      const float x1 = to_f(src[p.q_col + h * p.hd + j]);
-      const float x2 = to_f(src[p.q_col + h * p.hd + j + half]);
-      T* qo = static_cast<T*>(p.q_out) + static_cast<size_t>(row) * p.ldq + h * p.hd;
-      qo[j] = from_f<T>(x1 * cs.x - x2 * cs.y);
-      qo[j + half] = from_f<T>(x2 * cs.x + x1 * cs.y);
+      const float x1 = src[p.q_col + h * p.hd + j];
+      const float x2 = src[p.q_col + h * p.hd + j + half];
+      float* qo = p.q_out + static_cast<size_t>(row) * p.ldq + h * p.hd;
+      qo[j] = x1 * cs.x - x2 * cs.y;
+      qo[j + half] = x2 * cs.x + x1 * cs.y;
     }
     if (page >= 0) {
       T* base = pool + (static_cast<size_t>(page) * p.H + h) * 2 * 16 * p.hd + (slot & 15) * p.hd;
-      const float k1 = to_f(src[p.k_col + h * p.hd + j]);
-      const float k2 = to_f(src[p.k_col + h * p.hd + j + half]);
+      const float k1 = src[p.k_col + h * p.hd + j];
+      const float k2 = src[p.k_col + h * p.hd + j + half];
       base[j] = from_f<T>(k1 * cs.x - k2 * cs.y);
       base[j + half] = from_f<T>(k2 * cs.x + k1 * cs.y);
-      base[16 * p.hd + j] = src[p.v_col + h * p.hd + j];
-      base[16 * p.hd + j + half] = src[p.v_col + h * p.hd + j + half];
+      base[16 * p.hd + j] = from_f<T>(src[p.v_col + h * p.hd + j]);
+      base[16 * p.hd + j + half] = from_f<T>(src[p.v_col + h * p.hd + j + half]);
     }
   }
 }
 
 // SwiGLU: h = SiLU(gate) * up, gate in columns [0, F), up in [F, 2F).
 template <typename T>
-__global__ void swiglu_kernel(const T* __restrict__ gu, int ldgu, int F, T* __restrict__ h, int ldh) {
-  const T* g = gu + static_cast<size_t>(blockIdx.y) * ldgu;
-  T* o = h + static_cast<size_t>(blockIdx.y) * ldh;
+__global__ void swiglu_kernel(const float* __restrict__ gu, int ldgu, int F, T* __restrict__ h,
+                              T* __restrict__ h_lo, int ldh) {
+  const float* g = gu + static_cast<size_t>(blockIdx.y) * ldgu;
+  const size_t row = static_cast<size_t>(blockIdx.y) * ldh;
   for (int f = blockIdx.x * blockDim.x + threadIdx.x; f < F; f += gridDim.x * blockDim.x)
-    o[f] = from_f<T>(silu_f(to_f(g[f])) * to_f(g[F + f]));
+    store_act(h, h_lo, row + f, silu_f(g[f]) * g[F + f]);
 }
 
 template <typename T>
@@ -260,44 +265,36 @@ __global__ void topk_kernel(const float* __restrict__ logits, int V, int k, int*
 
 }  // namespace
 
-cudaError_t rmsnorm(int dtype, int in_f32, const void* X, int ldx, const void* g, void* Y, int ldy,
-                    int rows, int d, float eps, cudaStream_t s) {
+cudaError_t rmsnorm(int dtype, const float* X, int ldx, const void* g, void* Y, void* Y_lo, float* Y32,
+                    int ldy, int rows, int d, float eps, cudaStream_t s) {
   if (rows <= 0) return cudaSuccess;
   if (dtype == 0)
-    rmsnorm_kernel<float, float><<<rows, 256, 0, s>>>(static_cast<const float*>(X), ldx,
-                                                       static_cast<const float*>(g),
-                                                       static_cast<float*>(Y), ldy, d, eps);
-  else if (in_f32)
-    rmsnorm_kernel<float, bf16><<<rows, 256, 0, s>>>(static_cast<const float*>(X), ldx,
-                                                      static_cast<const bf16*>(g),
-                                                      static_cast<bf16*>(Y), ldy, d, eps);
+    rmsnorm_kernel<float><<<rows, 256, 0, s>>>(X, ldx, static_cast<const float*>(g), static_cast<float*>(Y),
+                                               nullptr, Y32, ldy, d, eps);
   else
-    rmsnorm_kernel<bf16, bf16><<<rows, 256, 0, s>>>(static_cast<const bf16*>(X), ldx,
-                                                     static_cast<const bf16*>(g),
-                                                     static_cast<bf16*>(Y), ldy, d, eps);
+    rmsnorm_kernel<bf16><<<rows, 256, 0, s>>>(X, ldx, static_cast<const bf16*>(g), static_cast<bf16*>(Y),
+                                              static_cast<bf16*>(Y_lo), Y32, ldy, d, eps);
   return cudaGetLastError();
 }
 
-cudaError_t rope_kv(const RopeKvParams& p, int dtype, cudaStream_t s) {
+cudaError_t rope_kv(const RopeKvParams& p, int kv_f32, cudaStream_t s) {
   const int rows = p.B * p.rows_per_seq;
   if (rows <= 0) return cudaSuccess;
-  if (dtype == 0)
+  if (kv_f32)
     rope_kv_kernel<float><<<rows, 256, 0, s>>>(p);
   else
     rope_kv_kernel<bf16><<<rows, 256, 0, s>>>(p);
   return cudaGetLastError();
 }
 
-cudaError_t swiglu(int dtype, const void* gu, int ldgu, int F, void* h, int ldh, int rows,
+cudaError_t swiglu(int dtype, const float* gu, int ldgu, int F, void* h, void* h_lo, int ldh, int rows,
                    cudaStream_t s) {
   if (rows <= 0) return cudaSuccess;
   dim3 grid((F + 255) / 256, rows);
   if (dtype == 0)
-    swiglu_kernel<float><<<grid, 256, 0, s>>>(static_cast<const float*>(gu), ldgu, F,
-                                              static_cast<float*>(h), ldh);
+    swiglu_kernel<float><<<grid, 256, 0, s>>>(gu, ldgu, F, static_cast<float*>(h), nullptr, ldh);
   else
-    swiglu_kernel<bf16><<<grid, 256, 0, s>>>(static_cast<const bf16*>(gu), ldgu, F,
-                                             static_cast<bf16*>(h), ldh);
+    swiglu_kernel<bf16><<<grid, 256, 0, s>>>(gu, ldgu, F, static_cast<bf16*>(h), static_cast<bf16*>(h_lo), ldh);
   return cudaGetLastError();
 }
 

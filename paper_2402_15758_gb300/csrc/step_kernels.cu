@@ -33,11 +33,11 @@ __global__ void trigram_gather_kernel(const T* __restrict__ E, int d, int V, con
 // headin[b][d..2d) = h_full (the draft block output), kept per head for debugging.
 template <typename T>
 __global__ void hfull_store_kernel(const float* __restrict__ dres, int d, T* __restrict__ headin,
-                                   T* __restrict__ hlog) {
+                                   T* __restrict__ headin_lo, float* __restrict__ hlog) {
   const int b = blockIdx.x;
   for (int c = threadIdx.x; c < d; c += blockDim.x) {
-    const T v = from_f<T>(dres[static_cast<size_t>(b) * d + c]);
-    headin[static_cast<size_t>(b) * 2 * d + d + c] = v;
+    const float v = dres[static_cast<size_t>(b) * d + c];
+    store_act(headin, headin_lo, static_cast<size_t>(b) * 2 * d + d + c, v);
     hlog[static_cast<size_t>(b) * d + c] = v;
   }
 }
@@ -119,21 +119,21 @@ __global__ void compact_kernel(char* pool, long long layer_stride_bytes, int H, 
   if (active) *row_ptr(n + j) = v;
 }
 
-// hsel[b][j] = verify hidden of path node j (j <= L; later rows repeat the last);
-// headin[b][0..d) = hidden of the last accepted node (h_LLM of the new prefix end).
+// hsel[b][j] = verify hidden (fp32) of path node j (j <= L; later rows repeat the
+// last); headin[b][0..d) = hidden of the last accepted node (h_LLM of the new prefix end).
 template <typename T>
-__global__ void gather_hidden_kernel(const T* __restrict__ hfin, int d, int N, const int* path,
-                                     const int* Lacc, int D1, T* __restrict__ hsel,
-                                     T* __restrict__ headin) {
+__global__ void gather_hidden_kernel(const float* __restrict__ hfin, int d, int N, const int* path,
+                                     const int* Lacc, int D1, float* __restrict__ hsel,
+                                     T* __restrict__ headin, T* __restrict__ headin_lo) {
   const int b = blockIdx.x, j = blockIdx.y;
   const int L = Lacc[b];
   const int node = path[b * D1 + (j <= L ? j : L)];
-  const T* src = hfin + static_cast<size_t>(b * N + node) * d;
-  T* dst = hsel + static_cast<size_t>(b * D1 + j) * d;
+  const float* src = hfin + static_cast<size_t>(b * N + node) * d;
+  float* dst = hsel + static_cast<size_t>(b * D1 + j) * d;
   for (int c = threadIdx.x; c < d; c += blockDim.x) {
-    const T v = src[c];
+    const float v = src[c];
     dst[c] = v;
-    if (j == L) headin[static_cast<size_t>(b) * 2 * d + c] = v;
+    if (j == L) store_act(headin, headin_lo, static_cast<size_t>(b) * 2 * d + c, v);
   }
 }
 
@@ -156,14 +156,15 @@ __global__ void finalize_kernel(int* n_arr, int* tok, int tok_stride, const int*
 
 // Prefill chunk bookkeeping: keep h_LLM of the last prompt row, advance n.
 template <typename T>
-__global__ void prefill_advance_kernel(const T* __restrict__ hfin, int d, int rows_per_seq,
+__global__ void prefill_advance_kernel(const float* __restrict__ hfin, int d, int rows_per_seq,
                                        const int* valid, const int* last, int* n_arr,
-                                       T* __restrict__ headin) {
+                                       T* __restrict__ headin, T* __restrict__ headin_lo) {
   const int b = blockIdx.x;
   const int li = last[b];
   if (li >= 0) {
-    const T* src = hfin + static_cast<size_t>(b * rows_per_seq + li) * d;
-    for (int c = threadIdx.x; c < d; c += blockDim.x) headin[static_cast<size_t>(b) * 2 * d + c] = src[c];
+    const float* src = hfin + static_cast<size_t>(b * rows_per_seq + li) * d;
+    for (int c = threadIdx.x; c < d; c += blockDim.x)
+      store_act(headin, headin_lo, static_cast<size_t>(b) * 2 * d + c, src[c]);
   }
   if (threadIdx.x == 0) n_arr[b] += valid[b];
 }
@@ -187,12 +188,13 @@ cudaError_t launch_trigram_gather(int dtype, const void* E, int d, int V, const 
   return cudaGetLastError();
 }
 
-cudaError_t launch_hfull_store(int dtype, const float* dres, int d, void* headin, void* hlog, int B,
-                               cudaStream_t s) {
+cudaError_t launch_hfull_store(int dtype, const float* dres, int d, void* headin, void* headin_lo, float* hlog,
+                               int B, cudaStream_t s) {
   if (dtype == 0)
-    hfull_store_kernel<float><<<B, 256, 0, s>>>(dres, d, static_cast<float*>(headin), static_cast<float*>(hlog));
+    hfull_store_kernel<float><<<B, 256, 0, s>>>(dres, d, static_cast<float*>(headin), nullptr, hlog);
   else
-    hfull_store_kernel<bf16><<<B, 256, 0, s>>>(dres, d, static_cast<bf16*>(headin), static_cast<bf16*>(hlog));
+    hfull_store_kernel<bf16><<<B, 256, 0, s>>>(dres, d, static_cast<bf16*>(headin), static_cast<bf16*>(headin_lo),
+                                               hlog);
   return cudaGetLastError();
 }
 
@@ -222,15 +224,15 @@ cudaError_t launch_compact(void* pool, long long layer_stride_bytes, int n_layer
   return cudaGetLastError();
 }
 
-cudaError_t launch_gather_hidden(int dtype, const void* hfin, int d, int N, const int* path, const int* Lacc,
-                                 int D1, void* hsel, void* headin, int B, cudaStream_t s) {
+cudaError_t launch_gather_hidden(int dtype, const float* hfin, int d, int N, const int* path, const int* Lacc,
+                                 int D1, float* hsel, void* headin, void* headin_lo, int B, cudaStream_t s) {
   dim3 grid(B, D1);
   if (dtype == 0)
-    gather_hidden_kernel<float><<<grid, 256, 0, s>>>(static_cast<const float*>(hfin), d, N, path, Lacc, D1,
-                                                     static_cast<float*>(hsel), static_cast<float*>(headin));
+    gather_hidden_kernel<float><<<grid, 256, 0, s>>>(hfin, d, N, path, Lacc, D1, hsel, static_cast<float*>(headin),
+                                                     nullptr);
   else
-    gather_hidden_kernel<bf16><<<grid, 256, 0, s>>>(static_cast<const bf16*>(hfin), d, N, path, Lacc, D1,
-                                                    static_cast<bf16*>(hsel), static_cast<bf16*>(headin));
+    gather_hidden_kernel<bf16><<<grid, 256, 0, s>>>(hfin, d, N, path, Lacc, D1, hsel, static_cast<bf16*>(headin),
+                                                    static_cast<bf16*>(headin_lo));
   return cudaGetLastError();
 }
 
@@ -240,14 +242,14 @@ cudaError_t launch_finalize(int* n, int* tok, int tok_stride, const int* Lacc, c
   return cudaGetLastError();
 }
 
-cudaError_t launch_prefill_advance(int dtype, const void* hfin, int d, int rows_per_seq, const int* valid,
-                                   const int* last, int* n, void* headin, int B, cudaStream_t s) {
+cudaError_t launch_prefill_advance(int dtype, const float* hfin, int d, int rows_per_seq, const int* valid,
+                                   const int* last, int* n, void* headin, void* headin_lo, int B, cudaStream_t s) {
   if (dtype == 0)
-    prefill_advance_kernel<float><<<B, 256, 0, s>>>(static_cast<const float*>(hfin), d, rows_per_seq, valid,
-                                                    last, n, static_cast<float*>(headin));
+    prefill_advance_kernel<float><<<B, 256, 0, s>>>(hfin, d, rows_per_seq, valid, last, n,
+                                                    static_cast<float*>(headin), nullptr);
   else
-    prefill_advance_kernel<bf16><<<B, 256, 0, s>>>(static_cast<const bf16*>(hfin), d, rows_per_seq, valid,
-                                                   last, n, static_cast<bf16*>(headin));
+    prefill_advance_kernel<bf16><<<B, 256, 0, s>>>(hfin, d, rows_per_seq, valid, last, n,
+                                                   static_cast<bf16*>(headin), static_cast<bf16*>(headin_lo));
   return cudaGetLastError();
 }
 

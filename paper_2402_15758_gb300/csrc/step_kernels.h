@@ -8,8 +8,8 @@ namespace chimera {
 cudaError_t launch_trigram_gather(int dtype, const void* E, int d, int V, const int* n, const int* tok,
                                   int tok_stride, const int* topk, int K, int KMAX, int k, void* out,
                                   int B, int* err, cudaStream_t s);
-cudaError_t launch_hfull_store(int dtype, const float* dres, int d, void* headin, void* hlog, int B,
-                               cudaStream_t s);
+cudaError_t launch_hfull_store(int dtype, const float* dres, int d, void* headin, void* headin_lo, float* hlog,
+                               int B, cudaStream_t s);
 cudaError_t launch_tree_expand(const int* n, const int* tok, int tok_stride, const int* topk, int K, int KMAX,
                                const int* depth, const int* rank, int N, const int* ovr_flag, const int* ovr,
                                int* node_tok, int B, cudaStream_t s);
@@ -19,12 +19,12 @@ cudaError_t launch_accept(const int* n, int* tok, int tok_stride, const int* nod
 cudaError_t launch_compact(void* pool, long long layer_stride_bytes, int n_layers, int H, int row_bytes,
                            const int* n, const int* path, const int* Lacc, int D1, const int* page_table,
                            int max_pages, int B, cudaStream_t s);
-cudaError_t launch_gather_hidden(int dtype, const void* hfin, int d, int N, const int* path, const int* Lacc,
-                                 int D1, void* hsel, void* headin, int B, cudaStream_t s);
+cudaError_t launch_gather_hidden(int dtype, const float* hfin, int d, int N, const int* path, const int* Lacc,
+                                 int D1, float* hsel, void* headin, void* headin_lo, int B, cudaStream_t s);
 cudaError_t launch_finalize(int* n, int* tok, int tok_stride, const int* Lacc, const int* bonus, int* count_log,
                             int log_cap, int* step, int B, cudaStream_t s);
-cudaError_t launch_prefill_advance(int dtype, const void* hfin, int d, int rows_per_seq, const int* valid,
-                                   const int* last, int* n, void* headin, int B, cudaStream_t s);
+cudaError_t launch_prefill_advance(int dtype, const float* hfin, int d, int rows_per_seq, const int* valid,
+                                   const int* last, int* n, void* headin, void* headin_lo, int B, cudaStream_t s);
 cudaError_t launch_set_root(const int* n, int* tok, int tok_stride, const int* amax, int B, cudaStream_t s);
 
 }  // namespace chimera

@@ -59,6 +59,25 @@ def test_linear_bf16_epilogues(M, N, K):
     assert _rel_rows(R.cpu().numpy(), R0.double().numpy() + ref) <= 1e-5
 
 
+@pytest.mark.parametrize("M,N,K", [(1, 256, 512), (64, 1536, 1024), (100, 384, 4096)])
+def test_linear_bf16_split_operand(M, N, K):
+    # X = hi + lo (two bf16 halves): W (hi + lo) reproduces the fp32 activation
+    g = torch.Generator().manual_seed(3 * M + K)
+    X32 = torch.randn(M, K, generator=g)
+    hi = X32.to(torch.bfloat16)
+    lo = (X32 - hi.float()).to(torch.bfloat16)
+    W = (torch.randn(N, K, generator=g) * 0.05).to(torch.bfloat16)
+    Y = torch.zeros(M, N, dtype=torch.float32, device="cuda")
+    pkg.op_linear(hi.cuda(), W.cuda(), Y, epi=0, out_f32=True, X_lo=lo.cuda())
+    torch.cuda.synchronize()
+    ref = X32.double().numpy() @ W.double().numpy().T
+    assert _rel_rows(Y.cpu().numpy(), ref) <= 2e-5
+    # without the lo half the error is the bf16 rounding of X
+    pkg.op_linear(hi.cuda(), W.cuda(), Y, epi=0, out_f32=True)
+    torch.cuda.synchronize()
+    assert _rel_rows(Y.cpu().numpy(), ref) > 1e-4
+
+
 def test_linear_deterministic():
     g = torch.Generator().manual_seed(5)
     X = torch.randn(64, 4096, generator=g).to(torch.bfloat16).cuda()
@@ -104,26 +123,30 @@ ATT_CASES = [
 ]
 
 
-@pytest.mark.parametrize("dtype", ["fp32", "bf16"])
+@pytest.mark.parametrize("dtype", ["fp32", "bf16", "bf16_kv32"])
 @pytest.mark.parametrize("case", range(len(ATT_CASES)))
 def test_attention_tree_masked_paged(dtype, case):
     B, H, hd, nctx, n_local, nq, q0, splits = ATT_CASES[case]
     rng = np.random.default_rng(case)
-    tdt = torch.float32 if dtype == "fp32" else torch.bfloat16
+    tdt = torch.float32 if dtype != "bf16" else torch.bfloat16  # KV pool element type
+    odt = torch.float32 if dtype == "fp32" else torch.bfloat16  # output type
     max_pages = (max(nctx) + n_local + 15) // 16 + 1
     n_blocks = B * max_pages + 3
     perm = rng.permutation(n_blocks)[: B * max_pages].reshape(B, max_pages).astype(np.int32)
     assert perm.max() < n_blocks
     pool = torch.randn(n_blocks, H, 2, 16, hd, generator=torch.Generator().manual_seed(case)).to(tdt)
-    q = torch.randn(B * nq, H * hd, generator=torch.Generator().manual_seed(100 + case)).to(tdt)
+    q = torch.randn(B * nq, H * hd, generator=torch.Generator().manual_seed(100 + case))
     anc = _random_tree_anc(n_local, rng) if q0 == 0 else [(1 << (i + 1)) - 1 for i in range(n_local)]
-    out = torch.zeros(B * nq, H * hd, dtype=tdt, device="cuda")
+    out = torch.zeros(B * nq, H * hd, dtype=odt, device="cuda")
+    out_lo = torch.zeros_like(out) if odt == torch.bfloat16 else None
     anc_t = torch.tensor(np.array(anc, dtype=np.uint64).view(np.int64), device="cuda")
     pkg.op_attention(q.cuda(), pool.cuda(), torch.tensor(perm, device="cuda"),
                      torch.tensor(nctx, dtype=torch.int32, device="cuda"), anc_t, out, nq=nq, q_local0=q0,
-                     n_local=n_local, q_rows=nq, n_heads=H, head_dim=hd, splits=splits)
+                     n_local=n_local, q_rows=nq, n_heads=H, head_dim=hd, splits=splits, out_lo=out_lo)
     torch.cuda.synchronize()
     got = out.float().cpu().numpy().reshape(B, nq, H, hd)
+    if out_lo is not None:
+        got = got + out_lo.float().cpu().numpy().reshape(B, nq, H, hd)
     P = pool.double().numpy()
     Q = q.double().numpy().reshape(B, nq, H, hd)
 
@@ -131,7 +154,7 @@ def test_attention_tree_masked_paged(dtype, case):
         blk = perm[b, slot // 16]
         return P[blk, :, 0, slot % 16], P[blk, :, 1, slot % 16]
 
-    tol = 1e-5 if dtype == "fp32" else 1e-2
+    tol = 1e-5
     for b in range(B):
         for i in range(nq):
             m = anc[q0 + i]

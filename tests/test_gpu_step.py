@@ -148,7 +148,7 @@ def _force_chain(W, cfg, st, tree, toks, L):
     return toks
 
 
-def _run_bf16(name, n_steps, forced_seq, device_gen="cpu", max_seq=None):
+def _run_bf16(name, n_steps, forced_seq, device_gen="cpu", max_seq=None, precision=1):
     cfg, w_cpu, w_dev = _setup(name, device_gen)
     W = co.OracleWeights(w_cpu, cache=(name != "7b"))
     prompts = synth.make_prompts(cfg)
@@ -156,7 +156,7 @@ def _run_bf16(name, n_steps, forced_seq, device_gen="cpu", max_seq=None):
     cap = max(len(p) for p in prompts) + n_steps * 5 + cfg["tree_nodes"] + 16
     cap = max_seq or ((cap + 15) // 16) * 16
     tree = ot.build_tree(cfg["topk"], cfg["tree_nodes"])
-    ctx = pkg.Chimera(cfg, w_dev, max_batch=B, max_seq_len=cap)
+    ctx = pkg.Chimera(cfg, w_dev, max_batch=B, max_seq_len=cap, precision=precision)
     _tree_equal(ctx, tree)
     states = [co.prefill(W, cfg, p, cap + 8) for p in prompts]
     ctx.prefill(prompts)
@@ -228,7 +228,7 @@ def _run_bf16(name, n_steps, forced_seq, device_gen="cpu", max_seq=None):
         ctx.set_root([s.tokens[s.n] for s in states])
         assert ctx.read("n").tolist() == [s.n for s in states]
     ctx.close()
-    print(f"{name}: {n_steps} steps x {B} seqs, accepted {accepted}, flags {flags}, "
+    print(f"{name} (precision {precision}): {n_steps} steps x {B} seqs, accepted {accepted}, flags {flags}, "
           f"draft heads skipped {skipped}, resyncs {resync}")
     return accepted
 
@@ -236,6 +236,11 @@ def _run_bf16(name, n_steps, forced_seq, device_gen="cpu", max_seq=None):
 def test_mini_bf16_steps():
     acc = _run_bf16("mini", 6, [0, 4, 2, 1, 3])
     assert max(acc) >= 3
+
+
+def test_mini_bf16_plain_precision():
+    # activations rounded once to bf16 and bf16 KV caches (precision 0)
+    _run_bf16("mini", 3, [4, 2, 0], precision=0)
 
 
 def test_mini_b4_ragged_batch():
