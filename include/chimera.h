@@ -69,10 +69,11 @@ typedef struct {
   int max_batch;        /* sequences per context, 1..64 */
   int max_seq_len;      /* KV slots per sequence (prompt + generated + N tree slots) */
   int kv_block;         /* must be 16 */
-  int precision;        /* bf16 models only.  1: every activation that feeds a tensor-core
-                           GEMM is kept as a hi + lo pair of bf16 values (two MMAs with fp32
-                           accumulation, ~fp32 accuracy) and the KV caches are fp32;
-                           0: activations rounded once to bf16 and bf16 KV caches.
+  int precision;        /* bf16 models only.  1: every activation that feeds a tensor core
+                           (GEMM operands, attention queries and probabilities) and every
+                           KV-cache entry is kept as a hi + lo pair of bf16 values, products
+                           taken term by term with fp32 accumulation (~fp32 accuracy);
+                           0: activations and KV entries rounded once to bf16.
                            fp32 models ignore it. */
 } chimera_config;
 
@@ -195,7 +196,8 @@ chimera_status chimera_debug_read(chimera_ctx* ctx, int what, void* host_dst, si
 
 /* Gather KV rows [pos0, pos0+count) of sequence `seq` from the paged cache of base
  * layer `layer` (layer = -1: the draft block's cache) into host buffers
- * k_dst / v_dst of shape [count][H][hd] (fp32 when the caches are fp32, else bf16). */
+ * k_dst / v_dst of shape [count][H][hd]: fp32 for fp32 models and for bf16 models with
+ * precision 1 (hi + lo), bf16 for precision 0. */
 chimera_status chimera_debug_read_kv(chimera_ctx* ctx, int layer, int seq, int pos0, int count,
                                      void* k_dst, void* v_dst);
 
@@ -210,15 +212,16 @@ chimera_status chimera_op_linear(int dtype, int epi, int out_f32, int M, int N, 
                                  const void* X, const void* X_lo, int ldx, const void* W, void* Y,
                                  int ldy, void* cuda_stream);
 
-/* Tree-masked attention over a paged KV pool [blocks][H][2][16][hd] (device; fp32
- * when dtype == 0 or kv_f32, else bf16): q fp32 [batch*q_rows][ldq] rotated queries,
+/* Tree-masked attention over a paged KV pool [blocks][H][planes][16][hd] (device):
+ * dtype 0: fp32 planes K, V; dtype 1: bf16 planes K, V, or with kv_split the two-term
+ * split K_hi, K_lo, V_hi, V_lo.  q fp32 [batch*q_rows][ldq] rotated queries,
  * query i of sequence b at row b*q_rows+i;
  * n_ctx (device int32 [batch]) committed rows visible to all; n_local rows follow at
  * slots n_ctx..; query i sees local row j iff bit j of anc[q_local0+i] (device
  * uint64); page_table device int32 [batch][max_pages]; out [batch*q_rows][ldo] in the
  * model dtype, out_lo (optional, bf16 only) its lo half.  nq <= 64, n_local <= 64,
  * hd in {64, 128}. */
-chimera_status chimera_op_attention(int dtype, int kv_f32, int batch, int n_heads, int head_dim,
+chimera_status chimera_op_attention(int dtype, int kv_split, int batch, int n_heads, int head_dim,
                                     int nq, int q_local0, int n_local, const float* q, int ldq,
                                     int q_rows, const void* pool, const int32_t* page_table,
                                     int max_pages, const int32_t* n_ctx, const uint64_t* anc,

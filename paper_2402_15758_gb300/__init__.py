@@ -278,12 +278,14 @@ def op_linear(X, W, Y, epi: int = 0, out_f32: bool = False, X_lo=None, stream=No
 
 def op_attention(q, pool, page_table, n_ctx, anc, out, nq, q_local0, n_local, q_rows, n_heads, head_dim,
                  splits=1, out_lo=None, stream=None):
-    """Tree-masked paged attention through chimera_op_attention (q fp32; pool fp32 or
-    bf16; out fp32 for an fp32 model, else bf16 with an optional lo half)."""
+    """Tree-masked paged attention through chimera_op_attention.  q fp32; pool
+    [blocks][H][planes][16][hd]: fp32 K, V planes (fp32 model, out fp32) or bf16 planes
+    (bf16 model, out bf16 + optional lo half): 2 planes K, V or 4 planes K_hi, K_lo,
+    V_hi, V_lo."""
     lib = load()
     dtype = 0 if out.element_size() == 4 else 1
-    kv_f32 = int(pool.element_size() == 4)
-    st = lib.chimera_op_attention(dtype, kv_f32, n_ctx.shape[0], n_heads, head_dim, nq, q_local0, n_local,
+    kv_split = int(pool.shape[2] == 4)
+    st = lib.chimera_op_attention(dtype, kv_split, n_ctx.shape[0], n_heads, head_dim, nq, q_local0, n_local,
                                   _ptr(q), q.stride(0), q_rows, _ptr(pool), _ptr(page_table), page_table.shape[1],
                                   _ptr(n_ctx), _ptr(anc), _ptr(out), _ptr(out_lo), out.stride(0), splits,
                                   _stream_handle(stream))

@@ -23,7 +23,8 @@ enum : int {
 enum : int {
   EPI_STORE = 0,   // Y = acc                      (Y bf16 or fp32)
   EPI_SILU = 1,    // Y = SiLU(acc)                (trigram encoder, first linear)
-  EPI_RESID = 2,   // Y(fp32) += acc               (residual stream update)
+  EPI_RESID = 2,   // Y(fp32) += acc, split-K partials added with red.global.add in any
+                   // order: residual updates, and fp32 outputs zeroed by an earlier kernel
 };
 
 template <typename T> __device__ __forceinline__ float to_f(T v);

@@ -70,7 +70,8 @@ struct AttnParams {
   int n_local;            // local rows at slots n..n+n_local-1
   const int* n_local_dev; // optional per-sequence local count
   const unsigned long long* anc;  // [q_local0 + nq] ancestor-or-self masks over local rows
-  const void* pool;       // [blocks][H][2][16][hd]
+  const void* pool;       // [blocks][H][planes][16][hd], element type of the model
+  int planes;             // 2: K, V;  4: K_hi, K_lo, V_hi, V_lo (bf16 two-term split)
   long long pool_layer_stride;  // elements between layers (0 for the draft pool)
   int layer;
   const int* page_table;  // [B][max_pages]
@@ -82,20 +83,21 @@ struct AttnParams {
   int B, H, hd;
   float scale;
   int splits;             // KV splits per (b, h)
-  float* ws;              // [B][H][splits][nq_max][hd + 2]
+  float* ws;              // [B][H][splits][nq_max][hd + 4] (output, max, sum, pad)
   int* counters;          // [B][H], zero between launches
   int nq_max;
 };
-// dtype: 0 fp32 model; 1 bf16 model.  kv_f32: the KV pool holds fp32 (else bf16).
-cudaError_t attention(const AttnParams& p, int dtype, int kv_f32, cudaStream_t s);
+// dtype: 0 fp32 model (fp32 KV), 1 bf16 model (bf16 KV planes).
+cudaError_t attention(const AttnParams& p, int dtype, cudaStream_t s);
 size_t attn_ws_floats(int B, int H, int splits, int nq_max, int hd);
 
 // ----------------------------------------------------------------------------
 // row-wise / small kernels
 // ----------------------------------------------------------------------------
-// Y (model dtype, plus the optional lo half) and an optional fp32 copy Y32.
+// Y (model dtype, plus the optional lo half) and an optional fp32 copy Y32; also zeroes
+// rows [0, rows) x [0, zcols) of Z when given (zcols, ldz multiples of 4).
 cudaError_t rmsnorm(int dtype, const float* X, int ldx, const void* g, void* Y, void* Y_lo, float* Y32,
-                    int ldy, int rows, int d, float eps, cudaStream_t s);
+                    int ldy, int rows, int d, float eps, float* Z, int ldz, int zcols, cudaStream_t s);
 
 struct RopeKvParams {
   const float* qkv;  // [rows][ldqkv] fp32 projections
@@ -103,7 +105,8 @@ struct RopeKvParams {
   int q_col, k_col, v_col;  // column offsets (q_col < 0: no query output)
   float* q_out;      // [rows][H*hd] fp32
   int ldq;
-  void* pool;
+  void* pool;          // [blocks][H][planes][16][hd]
+  int planes;          // 2 or 4 (split hi/lo planes, bf16 models)
   long long pool_layer_stride;
   int layer;
   const int* page_table;
@@ -119,7 +122,7 @@ struct RopeKvParams {
   int B, H, hd;
   int* err;
 };
-cudaError_t rope_kv(const RopeKvParams& p, int kv_f32, cudaStream_t s);
+cudaError_t rope_kv(const RopeKvParams& p, int dtype, cudaStream_t s);
 
 cudaError_t swiglu(int dtype, const float* gu, int ldgu, int F, void* h, void* h_lo, int ldh, int rows,
                    cudaStream_t s);
@@ -131,7 +134,10 @@ cudaError_t embed(int dtype, const void* E, int d, int V, float* x, int rows, in
                   const int* valid, int* err, cudaStream_t s);
 
 cudaError_t argmax_rows(const float* logits, int V, int rows, int* out, cudaStream_t s);
-cudaError_t topk_rows(const float* logits, int V, int rows, int k, int* idx, float* val,
-                      int out_stride, cudaStream_t s);
+// Top-k (k <= 8) of each row, larger score first, then smaller index.  Scratch:
+// ws_v / ws_i [rows][TOPK_MAX_BLOCKS][8], counters [rows] (zero between launches).
+constexpr int TOPK_MAX_BLOCKS = 64;  // V <= 64 * 2048
+cudaError_t topk_rows(const float* logits, int V, int rows, int k, int* idx, float* val, int out_stride,
+                      float* ws_v, int* ws_i, int* counters, cudaStream_t s);
 
 }  // namespace chimera

@@ -30,21 +30,41 @@
 namespace chimera {
 namespace {
 
+// Pipeline shape (compile-time; the defaults are the tuned values).
+#ifndef CHIMERA_LIN_CTAS_PER_SM
+#define CHIMERA_LIN_CTAS_PER_SM 1
+#endif
+#ifndef CHIMERA_LIN_PIPE_KB
+#define CHIMERA_LIN_PIPE_KB 200
+#endif
+#ifndef CHIMERA_LIN_BK_ATOMS
+#define CHIMERA_LIN_BK_ATOMS 1
+#endif
 constexpr int BM = 128;   // weight rows per tile (UMMA M)
-constexpr int BK = 64;    // K per stage: one 128-byte swizzle atom of bf16
+constexpr int ATOM = 64;  // one 128-byte swizzle atom of bf16 along K
+constexpr int BKA = CHIMERA_LIN_BK_ATOMS;  // atoms per pipeline stage
+constexpr int BK = ATOM * BKA;             // K per stage
 constexpr int UK = 16;    // UMMA K for 16-bit inputs
 constexpr int MAX_STAGES = 12;
 constexpr int THREADS = 192;
-constexpr int PIPE_SMEM = 200 * 1024;
+constexpr int CTAS_PER_SM = CHIMERA_LIN_CTAS_PER_SM;
+constexpr int PIPE_SMEM = CHIMERA_LIN_PIPE_KB * 1024;
 constexpr int MAX_BN = 256;
 constexpr int MAX_TILES = 8192;
 
-__device__ __forceinline__ int cta_of_unit(long long u, long long U, int G) {
+#ifdef CHIMERA_LIN_TRACE
+// Per-CTA timestamps of one launch (instrumented builds only).
+__device__ unsigned long long g_lin_trace[1024][8];
+#define TRACE(i) g_lin_trace[blockIdx.x][i] = global_timer_ns()
+#else
+#define TRACE(i)
+#endif
+
+// Stream-K partition in 32-bit arithmetic (the host checks units * grid < 2^32).
+__device__ __forceinline__ int cta_of_unit(uint32_t u, uint32_t U, uint32_t G) {
   return static_cast<int>(((u + 1) * G - 1) / U);
 }
-__device__ __forceinline__ long long unit_begin(int c, long long U, int G) {
-  return static_cast<long long>(c) * U / G;
-}
+__device__ __forceinline__ uint32_t unit_begin(uint32_t c, uint32_t U, uint32_t G) { return c * U / G; }
 
 // Epilogue of 16 consecutive token columns (m0 .. m0+15) of feature row f.  All
 // loads are issued before the stores so they overlap.
@@ -52,13 +72,9 @@ __device__ __forceinline__ void epi_store16(const TcLinearParams& p, int m0, int
   if (f >= p.N) return;
   if (p.epi == EPI_RESID) {
     float* y = static_cast<float*>(p.Y);
-    float old[16];
 #pragma unroll
     for (int j = 0; j < 16; ++j)
-      old[j] = (m0 + j < p.M) ? y[static_cast<size_t>(m0 + j) * p.ldy + f] : 0.f;
-#pragma unroll
-    for (int j = 0; j < 16; ++j)
-      if (m0 + j < p.M) y[static_cast<size_t>(m0 + j) * p.ldy + f] = old[j] + v[j];
+      if (m0 + j < p.M) atomicAdd(y + static_cast<size_t>(m0 + j) * p.ldy + f, v[j]);  // red.global.add
     return;
   }
 #pragma unroll
@@ -94,12 +110,14 @@ __device__ __forceinline__ bool mbar_wait_plain(uint64_t* bar, uint32_t parity, 
   return true;
 }
 
-__global__ void __launch_bounds__(THREADS, 1) tc_linear_kernel(const __grid_constant__ TcLinearParams p) {
+__global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const __grid_constant__ TcLinearParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  const int b_bytes = p.BN * BK * 2;
-  const int stage_bytes = BM * BK * 2 + (p.has_lo ? 2 : 1) * b_bytes;
+  const int a_atom = BM * ATOM * 2;     // one 128 x 64 weight box
+  const int b_atom = p.BN * ATOM * 2;  // one BN x 64 activation box
+  const int b_bytes = b_atom * BKA;
+  const int stage_bytes = a_atom * BKA + (p.has_lo ? 2 : 1) * b_bytes;
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + p.stages * stage_bytes);
   uint64_t* empty = full + MAX_STAGES;
   uint64_t* tfull = empty + MAX_STAGES;
@@ -136,13 +154,14 @@ __global__ void __launch_bounds__(THREADS, 1) tc_linear_kernel(const __grid_cons
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  if (threadIdx.x == 0) TRACE(0);
 
-  const long long U = p.units;
-  const int G = gridDim.x;
+  const uint32_t U = static_cast<uint32_t>(p.units);
+  const uint32_t G = gridDim.x;
   const int cta = blockIdx.x;
-  const long long u_begin = unit_begin(cta, U, G);
-  const long long u_end = unit_begin(cta + 1, U, G);
-  const int KB = p.kblocks;
+  const uint32_t u_begin = unit_begin(cta, U, G);
+  const uint32_t u_end = unit_begin(cta + 1, U, G);
+  const uint32_t KB = p.kblocks;
   volatile int* abort = s_abort;
 
   if (warp == 0) {
@@ -152,19 +171,23 @@ __global__ void __launch_bounds__(THREADS, 1) tc_linear_kernel(const __grid_cons
       int stage = 0;
       uint32_t phase = 0;
       uint32_t issued_mask = 0, issued_par = 0;
-      for (long long u = u_begin; u < u_end && !*abort;) {
+      for (uint32_t u = u_begin; u < u_end && !*abort;) {
         const int t = static_cast<int>(u / KB);
         int kb = static_cast<int>(u % KB);
-        const long long seg_end = min(u_end, static_cast<long long>(t + 1) * KB);
+        const uint32_t seg_end = min(u_end, static_cast<uint32_t>(t + 1) * KB);
         const int ft = t / p.tok_tiles, tt = t % p.tok_tiles;
         for (; u < seg_end; ++u, ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1u, abort)) break;
           uint8_t* sa = smem + stage * stage_bytes;
-          uint8_t* sb = sa + BM * BK * 2;
+          uint8_t* sb = sa + a_atom * BKA;
           mbar_arrive_expect_tx(&full[stage], static_cast<uint32_t>(stage_bytes));
-          tma_load_2d_hint(sa, &p.tmA, kb * BK, ft * BM, &full[stage], pol_w);
-          tma_load_2d(sb, &p.tmB, kb * BK, tt * p.BN, &full[stage]);
-          if (p.has_lo) tma_load_2d(sb + b_bytes, &p.tmB2, kb * BK, tt * p.BN, &full[stage]);
+          if (u == u_begin) TRACE(1);
+#pragma unroll
+          for (int a = 0; a < BKA; ++a) {
+            tma_load_2d_hint(sa + a * a_atom, &p.tmA, kb * BK + a * ATOM, ft * BM, &full[stage], pol_w);
+            tma_load_2d(sb + a * b_atom, &p.tmB, kb * BK + a * ATOM, tt * p.BN, &full[stage]);
+            if (p.has_lo) tma_load_2d(sb + b_bytes + a * b_atom, &p.tmB2, kb * BK + a * ATOM, tt * p.BN, &full[stage]);
+          }
           issued_mask |= 1u << stage;
           issued_par = (issued_par & ~(1u << stage)) | (phase << stage);
           if (++stage == p.stages) {
@@ -187,23 +210,28 @@ __global__ void __launch_bounds__(THREADS, 1) tc_linear_kernel(const __grid_cons
       uint32_t phase = 0;
       int buf = 0;
       uint32_t aphase = 0;
-      for (long long u = u_begin; u < u_end && !*abort;) {
+      for (uint32_t u = u_begin; u < u_end && !*abort;) {
         const int t = static_cast<int>(u / KB);
-        const long long seg_end = min(u_end, static_cast<long long>(t + 1) * KB);
+        const uint32_t seg_end = min(u_end, static_cast<uint32_t>(t + 1) * KB);
         if (!mbar_wait(&tempty[buf], aphase ^ 1u, abort)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + buf * p.acc_stride;
         bool first = true;
         for (; u < seg_end; ++u) {
           if (!mbar_wait(&full[stage], phase, abort)) break;
+          if (u == u_begin) TRACE(2);
           tc_fence_after();
           const uint32_t sa = smem_u32(smem + stage * stage_bytes);
-          const uint32_t sb = sa + BM * BK * 2;
+          const uint32_t sb = sa + a_atom * BKA;
 #pragma unroll
-          for (int k = 0; k < BK / UK; ++k) {
-            const uint64_t adesc = sw128_desc(sa + k * 32);
-            tc_mma_bf16(d_tmem, adesc, sw128_desc(sb + k * 32), idesc, (first && k == 0) ? 0u : 1u);
-            if (p.has_lo) tc_mma_bf16(d_tmem, adesc, sw128_desc(sb + b_bytes + k * 32), idesc, 1u);
+          for (int a = 0; a < BKA; ++a) {
+#pragma unroll
+            for (int k = 0; k < ATOM / UK; ++k) {
+              const uint64_t adesc = sw128_desc(sa + a * a_atom + k * 32);
+              tc_mma_bf16(d_tmem, adesc, sw128_desc(sb + a * b_atom + k * 32), idesc,
+                          (first && a == 0 && k == 0) ? 0u : 1u);
+              if (p.has_lo) tc_mma_bf16(d_tmem, adesc, sw128_desc(sb + b_bytes + a * b_atom + k * 32), idesc, 1u);
+            }
           }
           first = false;
           tc_commit(&empty[stage]);
@@ -213,6 +241,7 @@ __global__ void __launch_bounds__(THREADS, 1) tc_linear_kernel(const __grid_cons
           }
         }
         tc_commit(&tfull[buf]);
+        TRACE(3);
         buf ^= 1;
         if (buf == 0) aphase ^= 1u;
       }
@@ -228,22 +257,23 @@ __global__ void __launch_bounds__(THREADS, 1) tc_linear_kernel(const __grid_cons
     const int row = q * 32 + lane;
     int buf = 0;
     uint32_t aphase = 0;
-    for (long long u = u_begin; u < u_end;) {
+    for (uint32_t u = u_begin; u < u_end;) {
       const int t = static_cast<int>(u / KB);
-      const long long seg_end = min(u_end, static_cast<long long>(t + 1) * KB);
+      const uint32_t seg_end = min(u_end, static_cast<uint32_t>(t + 1) * KB);
       u = seg_end;
       const bool ok = mbar_wait(&tfull[buf], aphase, abort);
       if (bar_any(1, 128, !ok)) break;
+      if (threadIdx.x == 64) TRACE(4);
       tc_fence_after();
       const int ft = t / p.tok_tiles, tt = t % p.tok_tiles;
-      const long long tu0 = static_cast<long long>(t) * KB;
+      const uint32_t tu0 = static_cast<uint32_t>(t) * KB;
       const int c_first = cta_of_unit(tu0, U, G);
       const int c_last = cta_of_unit(tu0 + KB - 1, U, G);
       const int nparts = c_last - c_first + 1;
       const int f = ft * BM + row;
       const int m0 = tt * p.BN;
       const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + buf * p.acc_stride;
-      if (nparts == 1) {
+      if (nparts == 1 || p.epi == EPI_RESID) {
         for (int c0 = 0; c0 < p.BN; c0 += 16) {
           float v[16];
           tmem_ld_16(tbase + c0, v);
@@ -252,7 +282,7 @@ __global__ void __launch_bounds__(THREADS, 1) tc_linear_kernel(const __grid_cons
         tc_fence_before();
         mbar_arrive(&tempty[buf]);
       } else {
-        const int my_slot = 2 * cta + ((u_begin / KB == t) ? 0 : 1);
+        const int my_slot = 2 * cta + ((u_begin / KB == static_cast<uint32_t>(t)) ? 0 : 1);
         float* wsp = p.ws + static_cast<size_t>(my_slot) * BM * p.BN;
         for (int c0 = 0; c0 < p.BN; c0 += 16) {
           float v[16];
@@ -269,8 +299,12 @@ __global__ void __launch_bounds__(THREADS, 1) tc_linear_kernel(const __grid_cons
           *s_last = (old == nparts - 1) ? 1 : 0;
         }
         named_bar(1, 128);
+        if (threadIdx.x == 64) TRACE(5);
         if (*s_last) {
           __threadfence();
+          // slot of every contributor, computed once (contributor c2 > c_first starts
+          // inside tile t, so only c_first can hold the tile in its second slot)
+          const int slot_first = 2 * c_first + ((unit_begin(c_first, U, G) / KB == static_cast<uint32_t>(t)) ? 0 : 1);
           for (int c0 = 0; c0 < p.BN; c0 += 16) {
             if (m0 + c0 >= p.M) break;
             float acc[16];
@@ -284,7 +318,7 @@ __global__ void __launch_bounds__(THREADS, 1) tc_linear_kernel(const __grid_cons
               for (int q4 = 0; q4 < 4; ++q4) {
                 if (cc + q4 <= c_last) {
                   const int c2 = cc + q4;
-                  const int sl = 2 * c2 + ((unit_begin(c2, U, G) / KB == t) ? 0 : 1);
+                  const int sl = c2 == c_first ? slot_first : 2 * c2;
                   const float* src = p.ws + static_cast<size_t>(sl) * BM * p.BN + static_cast<size_t>(c0) * BM + row;
 #pragma unroll
                   for (int j = 0; j < 16; ++j) v[q4][j] = __ldcg(src + j * BM);
@@ -300,6 +334,7 @@ __global__ void __launch_bounds__(THREADS, 1) tc_linear_kernel(const __grid_cons
             epi_store16(p, m0 + c0, f, acc);
           }
           if (threadIdx.x == 64) p.counters[t] = 0;
+          if (threadIdx.x == 64) TRACE(6);
         }
         named_bar(1, 128);
       }
@@ -315,6 +350,7 @@ __global__ void __launch_bounds__(THREADS, 1) tc_linear_kernel(const __grid_cons
     tmem_dealloc(tmem_base, p.tmem_cols);
   }
   if (threadIdx.x == 0 && *abort) atomicOr(p.err, ERR_TIMEOUT);
+  if (threadIdx.x == 0) TRACE(7);
 }
 
 // ----------------------------------------------------------------------------
@@ -369,10 +405,19 @@ int tc_num_sms() {
 }
 
 size_t tc_ws_floats(int max_bn) {
-  return static_cast<size_t>(tc_num_sms()) * 2 * BM * static_cast<size_t>(max_bn);
+  return static_cast<size_t>(tc_num_sms()) * CTAS_PER_SM * 2 * BM * static_cast<size_t>(max_bn);
 }
 
 int tc_max_tiles() { return MAX_TILES; }
+
+#ifdef CHIMERA_LIN_TRACE
+extern "C" int chimera_lin_trace(unsigned long long* host, int ctas) {
+  return cudaMemcpyFromSymbol(host, g_lin_trace, static_cast<size_t>(ctas) * 8 * sizeof(unsigned long long)) ==
+                 cudaSuccess
+             ? 0
+             : -1;
+}
+#endif
 
 int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, const void* X_lo, int ldx,
                    const void* W, void* Y, void* Y_lo, int ldy, int epi, int out_f32, float* ws,
@@ -387,7 +432,7 @@ int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, const
   if ((reinterpret_cast<uintptr_t>(X) & 15) || (reinterpret_cast<uintptr_t>(W) & 15) ||
       (reinterpret_cast<uintptr_t>(X_lo) & 15))
     return fail("X, X_lo and W must be 16-byte aligned");
-  if (epi == EPI_RESID && !out_f32) return fail("residual epilogue needs an fp32 output");
+  if (epi == EPI_RESID && !out_f32) return fail("accumulating epilogue needs an fp32 output");
   TcLinearParams& p = plan->p;
   memset(&p, 0, sizeof(p));
   p.M = M;
@@ -399,6 +444,7 @@ int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, const
   p.kblocks = (K + BK - 1) / BK;
   if (static_cast<long long>(p.feat_tiles) * p.tok_tiles > MAX_TILES) return fail("too many tiles");
   p.units = static_cast<long long>(p.feat_tiles) * p.tok_tiles * p.kblocks;
+  if (p.units * (tc_num_sms() * CTAS_PER_SM + 1) >= (1ll << 32)) return fail("too many work units");
   p.has_lo = X_lo ? 1 : 0;
   const int stage_bytes = BM * BK * 2 + (p.has_lo ? 2 : 1) * p.BN * BK * 2;
   p.stages = PIPE_SMEM / stage_bytes;
@@ -416,10 +462,10 @@ int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, const
   p.tmem_cols = pow2ceil(2 * p.acc_stride);
   if (p.tmem_cols < 32) p.tmem_cols = 32;
   if (p.tmem_cols > 512) return fail("accumulators exceed tensor memory");
-  if (encode_2d_bf16(&p.tmA, W, K, N, K, BK, BM) != 0) return fail("tensor map of W");
-  if (encode_2d_bf16(&p.tmB, X, K, M, ldx, BK, p.BN) != 0) return fail("tensor map of X");
-  if (X_lo && encode_2d_bf16(&p.tmB2, X_lo, K, M, ldx, BK, p.BN) != 0) return fail("tensor map of X_lo");
-  const int sms = tc_num_sms();
+  if (encode_2d_bf16(&p.tmA, W, K, N, K, ATOM, BM) != 0) return fail("tensor map of W");
+  if (encode_2d_bf16(&p.tmB, X, K, M, ldx, ATOM, p.BN) != 0) return fail("tensor map of X");
+  if (X_lo && encode_2d_bf16(&p.tmB2, X_lo, K, M, ldx, ATOM, p.BN) != 0) return fail("tensor map of X_lo");
+  const int sms = tc_num_sms() * CTAS_PER_SM;
   plan->grid = static_cast<int>(p.units < sms ? p.units : sms);
   plan->smem = 1024 + static_cast<size_t>(p.stages) * stage_bytes + 2 * MAX_STAGES * 8 + 5 * 8 + 64;
   plan->weight_bytes = 2.0 * N * K;

@@ -137,8 +137,8 @@ struct chimera_ctx {
   int dtype = 0;
   size_t esz = 4;      // weights / GEMM operands
   int split = 0;       // bf16 GEMM operands kept as hi + lo pairs
-  int kv_f32 = 0;      // KV pools hold fp32
-  size_t kv_esz = 4;
+  int kv_planes = 2;   // KV planes per (block, head): K, V or K_hi, K_lo, V_hi, V_lo
+  size_t kv_esz = 4;   // element size of the KV pools (the model dtype)
   cudaStream_t stream = nullptr;
   bool own_stream = false;
   int num_sms = 1;
@@ -201,6 +201,9 @@ struct chimera_ctx {
   float* att_ws = nullptr;
   size_t att_ws_floats = 0;
   int* att_cnt = nullptr;
+  float* topk_ws_v = nullptr;
+  int* topk_ws_i = nullptr;
+  int* topk_cnt = nullptr;
 
   // plan of the current batch
   int batch = 0;
@@ -209,6 +212,7 @@ struct chimera_ctx {
   Lin ver_lm, pre_lm, pre_dkv, tri1, tri2, dqkv, dwo, dgate, dup, ddown, commit_kv;
   std::vector<Lin> dhead;
   int att_splits_ver = 1, att_splits_pre = 1, att_splits_draft = 1;
+  int plan_keys = 0;  // longest prompt of the batch (sizes the attention splits)
   cudaGraphExec_t graph = nullptr;
   bool prefilled = false;
   bool ovr_pending = false;
@@ -315,9 +319,13 @@ bool make_lin(chimera_ctx* ctx, Lin* l, int M, int N, int K, const void* X, cons
   return true;
 }
 
-int att_splits(const chimera_ctx* ctx, int B) {
+// KV splits per (sequence, head): enough CTAs to cover the SMs for single-query
+// attention (the draft), and about three 64-key tiles per split for tree queries so
+// the per-split partials stay few (their merge is latency-bound).
+int att_splits(const chimera_ctx* ctx, int B, int nq, int n_keys) {
   const int target = 2 * ctx->num_sms;
   int s = (target + B * ctx->H - 1) / (B * ctx->H);
+  if (nq > 1) s = std::min(s, (n_keys + 191) / 192);
   return std::max(1, std::min(16, s));
 }
 
@@ -336,6 +344,7 @@ cudaError_t run_attention(chimera_ctx* ctx, bool draft_pool, int layer, int nq, 
   p.n_local_dev = n_local_dev;
   p.anc = anc;
   p.pool = draft_pool ? ctx->dkv : ctx->kv;
+  p.planes = ctx->kv_planes;
   p.pool_layer_stride = draft_pool ? 0 : ctx->kv_layer_stride;
   p.layer = draft_pool ? 0 : layer;
   p.page_table = ctx->d_pt;
@@ -353,7 +362,7 @@ cudaError_t run_attention(chimera_ctx* ctx, bool draft_pool, int layer, int nq, 
   p.counters = ctx->att_cnt;
   p.nq_max = nq_max;
   if (attn_ws_floats(p.B, p.H, splits, nq_max, p.hd) > ctx->att_ws_floats) return cudaErrorInvalidValue;
-  return attention(p, ctx->dtype, ctx->kv_f32, ctx->stream);
+  return attention(p, ctx->dtype, ctx->stream);
 }
 
 cudaError_t run_rope(chimera_ctx* ctx, bool draft_pool, int layer, const float* src, int ldsrc, int q_col, int k_col,
@@ -369,6 +378,7 @@ cudaError_t run_rope(chimera_ctx* ctx, bool draft_pool, int layer, const float* 
   p.q_out = ctx->qr;
   p.ldq = ctx->d;
   p.pool = draft_pool ? ctx->dkv : ctx->kv;
+  p.planes = ctx->kv_planes;
   p.pool_layer_stride = draft_pool ? 0 : ctx->kv_layer_stride;
   p.layer = draft_pool ? 0 : layer;
   p.page_table = ctx->d_pt;
@@ -386,21 +396,23 @@ cudaError_t run_rope(chimera_ctx* ctx, bool draft_pool, int layer, const float* 
   p.H = ctx->H;
   p.hd = ctx->hd;
   p.err = ctx->d_err;
-  return rope_kv(p, ctx->kv_f32, ctx->stream);
+  return rope_kv(p, ctx->dtype, ctx->stream);
 }
 
-// RMSNorm of fp32 rows into the GEMM operand buffer xn (+ lo half).
-cudaError_t run_norm(chimera_ctx* ctx, const float* X, const void* g, int rows) {
+// RMSNorm of fp32 rows into the GEMM operand buffer xn (+ lo half); zeroes the rows of
+// Z (zcols floats, pitch zcols) that the following linear accumulates into.
+cudaError_t run_norm(chimera_ctx* ctx, const float* X, const void* g, int rows, float* Z, int zcols) {
   Scope sc(ctx, CHIMERA_KIND_NORM, 0);
-  return rmsnorm(ctx->dtype, X, ctx->d, g, ctx->xn, ctx->xn_lo, nullptr, ctx->d, rows, ctx->d, ctx->cfg.rms_eps,
-                 ctx->stream);
+  return rmsnorm(ctx->dtype, X, ctx->d, g, ctx->xn, ctx->xn_lo, nullptr, ctx->d, rows, ctx->d, ctx->cfg.rms_eps, Z,
+                 zcols, zcols, ctx->stream);
 }
 
-// Final norm: H_LLM rows in fp32 plus the LM-head operand (+ lo half).
-cudaError_t run_final_norm(chimera_ctx* ctx, int rows) {
+// Final norm: H_LLM rows in fp32 plus the LM-head operand (+ lo half); zeroes the
+// logits rows when the LM head follows.
+cudaError_t run_final_norm(chimera_ctx* ctx, int rows, bool zero_logits) {
   Scope sc(ctx, CHIMERA_KIND_NORM, 0);
   return rmsnorm(ctx->dtype, ctx->x, ctx->d, ctx->final_norm, ctx->hfin, ctx->hfin_lo, ctx->hfin32, ctx->d, rows,
-                 ctx->d, ctx->cfg.rms_eps, ctx->stream);
+                 ctx->d, ctx->cfg.rms_eps, zero_logits ? ctx->logits : nullptr, ctx->V, ctx->V, ctx->stream);
 }
 
 #define RUN(call)                                            \
@@ -418,13 +430,13 @@ cudaError_t enqueue_layer(chimera_ctx* ctx, int l, const Lin* lin, int rows, int
                           const int* pos_off, const unsigned long long* anc, int splits, double kv_bytes) {
   const chimera_block_weights& w = ctx->layers[l];
   const int d = ctx->d;
-  RUN(run_norm(ctx, ctx->x, w.attn_norm, rows));
+  RUN(run_norm(ctx, ctx->x, w.attn_norm, rows, ctx->qkv, 3 * d));
   RUN(run_lin(ctx, lin[0]));
   RUN(run_rope(ctx, false, l, ctx->qkv, 3 * d, 0, d, 2 * d, rows_per_seq, valid, 0, 0, 0, pos_off));
   RUN(run_attention(ctx, false, l, rows_per_seq, valid, 0, rows_per_seq, valid, anc, rows_per_seq, splits,
                     rows_per_seq, kv_bytes));
   RUN(run_lin(ctx, lin[1]));
-  RUN(run_norm(ctx, ctx->x, w.ffn_norm, rows));
+  RUN(run_norm(ctx, ctx->x, w.ffn_norm, rows, ctx->gu, 2 * ctx->F));
   RUN(run_lin(ctx, lin[2]));
   RUN(run_lin(ctx, lin[3]));
   {
@@ -439,7 +451,7 @@ double kv_read_bytes(const chimera_ctx* ctx, int extra_rows, bool draft) {
   double rows = 0;
   for (int b = 0; b < ctx->batch; ++b) rows += ctx->host_n[b] + extra_rows;
   (void)draft;
-  return rows * 2.0 * ctx->d * ctx->kv_esz;
+  return rows * ctx->kv_planes * static_cast<double>(ctx->d) * ctx->kv_esz;
 }
 
 // The whole step on the context stream (graph-capturable: every dynamic value is read
@@ -454,17 +466,17 @@ cudaError_t enqueue_step(chimera_ctx* ctx) {
     {
       Scope sc(ctx, CHIMERA_KIND_EMBED, 0);
       RUN(launch_trigram_gather(ctx->dtype, ctx->embed, d, V, ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_topk, K,
-                                ctx->KMAX, k, ctx->tbuf, B, ctx->d_err, s));
+                                ctx->KMAX, k, ctx->tbuf, B, ctx->d_err, ctx->dres, s));
     }
     RUN(run_lin(ctx, ctx->tri1));
     RUN(run_lin(ctx, ctx->tri2));
-    RUN(run_norm(ctx, ctx->dres, ctx->draft.attn_norm, B));
+    RUN(run_norm(ctx, ctx->dres, ctx->draft.attn_norm, B, ctx->qkv, 3 * d));
     RUN(run_lin(ctx, ctx->dqkv));
     RUN(run_rope(ctx, true, 0, ctx->qkv, 3 * d, 0, d, 2 * d, 1, nullptr, 0, k, k, nullptr));
     RUN(run_attention(ctx, true, 0, 1, nullptr, k, k + 1, nullptr, ctx->d_chain, 1, ctx->att_splits_draft, 1,
                       kv_read_bytes(ctx, k + 1, true)));
     RUN(run_lin(ctx, ctx->dwo));
-    RUN(run_norm(ctx, ctx->dres, ctx->draft.ffn_norm, B));
+    RUN(run_norm(ctx, ctx->dres, ctx->draft.ffn_norm, B, ctx->gu, 2 * ctx->F));
     RUN(run_lin(ctx, ctx->dgate));
     RUN(run_lin(ctx, ctx->dup));
     {
@@ -475,13 +487,15 @@ cudaError_t enqueue_step(chimera_ctx* ctx) {
     {
       Scope sc(ctx, CHIMERA_KIND_OTHER, 0);
       RUN(launch_hfull_store(ctx->dtype, ctx->dres, d, ctx->headin, ctx->headin_lo,
-                             ctx->hfull_log + static_cast<size_t>(k) * B * d, B, s));
+                             ctx->hfull_log + static_cast<size_t>(k) * B * d, ctx->hlog + static_cast<size_t>(k) * B * V,
+                             V, B, s));
     }
     RUN(run_lin(ctx, ctx->dhead[k]));
     {
       Scope sc(ctx, CHIMERA_KIND_TOPK, 0);
       RUN(topk_rows(ctx->hlog + static_cast<size_t>(k) * B * V, V, B, ctx->KMAX, ctx->d_topk + k * ctx->KMAX,
-                    ctx->d_topk_val + k * ctx->KMAX, K * ctx->KMAX, s));
+                    ctx->d_topk_val + k * ctx->KMAX, K * ctx->KMAX, ctx->topk_ws_v, ctx->topk_ws_i,
+                    ctx->topk_cnt, s));
     }
   }
   // ---- tree ----
@@ -500,7 +514,7 @@ cudaError_t enqueue_step(chimera_ctx* ctx) {
   const double kvb = kv_read_bytes(ctx, N, false);
   for (int l = 0; l < ctx->L; ++l)
     RUN(enqueue_layer(ctx, l, &ctx->ver[5 * l], B * N, N, nullptr, ctx->d_depth, ctx->d_anc, ctx->att_splits_ver, kvb));
-  RUN(run_final_norm(ctx, B * N));
+  RUN(run_final_norm(ctx, B * N, true));
   RUN(run_lin(ctx, ctx->ver_lm));
   {
     Scope sc(ctx, CHIMERA_KIND_ARGMAX, 0);
@@ -516,15 +530,15 @@ cudaError_t enqueue_step(chimera_ctx* ctx) {
   {
     Scope sc(ctx, CHIMERA_KIND_COMPACT, 0);
     RUN(launch_compact(ctx->kv, ctx->kv_layer_stride * static_cast<long long>(ctx->kv_esz), ctx->L, ctx->H,
-                       static_cast<int>(ctx->hd * ctx->kv_esz), ctx->d_n, ctx->d_path, ctx->d_L, ctx->D1, ctx->d_pt,
-                       ctx->max_pages, B, s));
+                       ctx->kv_planes, static_cast<int>(ctx->hd * ctx->kv_esz), ctx->d_n, ctx->d_path, ctx->d_L,
+                       ctx->D1, ctx->d_pt, ctx->max_pages, B, s));
   }
   {
     Scope sc(ctx, CHIMERA_KIND_OTHER, 0);
     RUN(launch_gather_hidden(ctx->dtype, ctx->hfin32, d, N, ctx->d_path, ctx->d_L, ctx->D1, ctx->hsel, ctx->headin,
                              ctx->headin_lo, B, s));
   }
-  RUN(run_norm(ctx, ctx->hsel, ctx->draft.attn_norm, B * ctx->D1));
+  RUN(run_norm(ctx, ctx->hsel, ctx->draft.attn_norm, B * ctx->D1, ctx->kvtmp, 2 * d));
   RUN(run_lin(ctx, ctx->commit_kv));
   RUN(run_rope(ctx, true, 0, ctx->kvtmp, 2 * d, -1, 0, d, ctx->D1, ctx->d_L, 1, 0, 0, nullptr));
   {
@@ -541,53 +555,56 @@ bool build_plans(chimera_ctx* ctx, int B) {
   const int f32 = 1, tb = ctx->dtype == 0 ? 1 : 0;  // bf16 storage -> out_f32 = 0
   ctx->ver.assign(5 * ctx->L, Lin());
   ctx->pre.assign(5 * ctx->L, Lin());
+  // fp32 outputs accumulate (split-K partials added atomically) into buffers that the
+  // preceding kernel zeroed, or into the residual stream itself
+  constexpr int ACC = EPI_RESID;
   void *xn = ctx->xn, *xl = ctx->xn_lo, *ao = ctx->ao, *al = ctx->ao_lo, *hf = ctx->hf, *hl = ctx->hf_lo;
   auto layer_plans = [&](std::vector<Lin>& v, int M) {
     for (int l = 0; l < ctx->L; ++l) {
       const chimera_block_weights& w = ctx->layers[l];
       Lin* p = &v[5 * l];
-      if (!make_lin(ctx, &p[0], M, 3 * d, d, xn, xl, d, w.wqkv, ctx->qkv, nullptr, 3 * d, EPI_STORE, f32)) return false;
-      if (!make_lin(ctx, &p[1], M, d, d, ao, al, d, w.wo, ctx->x, nullptr, d, EPI_RESID, f32)) return false;
-      if (!make_lin(ctx, &p[2], M, F, d, xn, xl, d, w.w_gate, ctx->gu, nullptr, 2 * F, EPI_STORE, f32)) return false;
-      if (!make_lin(ctx, &p[3], M, F, d, xn, xl, d, w.w_up, ctx->gu + F, nullptr, 2 * F, EPI_STORE, f32)) return false;
-      if (!make_lin(ctx, &p[4], M, d, F, hf, hl, F, w.w_down, ctx->x, nullptr, d, EPI_RESID, f32)) return false;
+      if (!make_lin(ctx, &p[0], M, 3 * d, d, xn, xl, d, w.wqkv, ctx->qkv, nullptr, 3 * d, ACC, f32)) return false;
+      if (!make_lin(ctx, &p[1], M, d, d, ao, al, d, w.wo, ctx->x, nullptr, d, ACC, f32)) return false;
+      if (!make_lin(ctx, &p[2], M, F, d, xn, xl, d, w.w_gate, ctx->gu, nullptr, 2 * F, ACC, f32)) return false;
+      if (!make_lin(ctx, &p[3], M, F, d, xn, xl, d, w.w_up, ctx->gu + F, nullptr, 2 * F, ACC, f32)) return false;
+      if (!make_lin(ctx, &p[4], M, d, F, hf, hl, F, w.w_down, ctx->x, nullptr, d, ACC, f32)) return false;
     }
     return true;
   };
   if (!layer_plans(ctx->ver, B * N)) return false;
   if (!layer_plans(ctx->pre, B * CHUNK)) return false;
   if (!make_lin(ctx, &ctx->ver_lm, B * N, V, d, ctx->hfin, ctx->hfin_lo, d, ctx->lm_head, ctx->logits, nullptr, V,
-                EPI_STORE, f32))
+                ACC, f32))
     return false;
   if (!make_lin(ctx, &ctx->pre_lm, B, V, d, ctx->headin, ctx->headin_lo, 2 * d, ctx->lm_head, ctx->logits, nullptr, V,
-                EPI_STORE, f32))
+                ACC, f32))
     return false;
   const void* dl_kv = eoff(ctx, const_cast<void*>(ctx->draft.wqkv), static_cast<size_t>(d) * d);
-  if (!make_lin(ctx, &ctx->pre_dkv, B * CHUNK, 2 * d, d, xn, xl, d, dl_kv, ctx->kvtmp, nullptr, 2 * d, EPI_STORE, f32))
+  if (!make_lin(ctx, &ctx->pre_dkv, B * CHUNK, 2 * d, d, xn, xl, d, dl_kv, ctx->kvtmp, nullptr, 2 * d, ACC, f32))
     return false;
-  if (!make_lin(ctx, &ctx->commit_kv, B * ctx->D1, 2 * d, d, xn, xl, d, dl_kv, ctx->kvtmp, nullptr, 2 * d, EPI_STORE,
+  if (!make_lin(ctx, &ctx->commit_kv, B * ctx->D1, 2 * d, d, xn, xl, d, dl_kv, ctx->kvtmp, nullptr, 2 * d, ACC,
                 f32))
     return false;
   // draft (M = B rows); the trigram input is a gather of bf16 embeddings: exact, no lo half
   if (!make_lin(ctx, &ctx->tri1, B, d, 3 * d, ctx->tbuf, nullptr, 3 * d, ctx->tri_w1, ctx->ubuf, ctx->ubuf_lo, d,
                 EPI_SILU, tb))
     return false;
-  if (!make_lin(ctx, &ctx->tri2, B, d, d, ctx->ubuf, ctx->ubuf_lo, d, ctx->tri_w2, ctx->dres, nullptr, d, EPI_STORE, f32))
+  if (!make_lin(ctx, &ctx->tri2, B, d, d, ctx->ubuf, ctx->ubuf_lo, d, ctx->tri_w2, ctx->dres, nullptr, d, ACC, f32))
     return false;
   const chimera_block_weights& w = ctx->draft;
-  if (!make_lin(ctx, &ctx->dqkv, B, 3 * d, d, xn, xl, d, w.wqkv, ctx->qkv, nullptr, 3 * d, EPI_STORE, f32)) return false;
-  if (!make_lin(ctx, &ctx->dwo, B, d, d, ao, al, d, w.wo, ctx->dres, nullptr, d, EPI_RESID, f32)) return false;
-  if (!make_lin(ctx, &ctx->dgate, B, F, d, xn, xl, d, w.w_gate, ctx->gu, nullptr, 2 * F, EPI_STORE, f32)) return false;
-  if (!make_lin(ctx, &ctx->dup, B, F, d, xn, xl, d, w.w_up, ctx->gu + F, nullptr, 2 * F, EPI_STORE, f32)) return false;
-  if (!make_lin(ctx, &ctx->ddown, B, d, F, hf, hl, F, w.w_down, ctx->dres, nullptr, d, EPI_RESID, f32)) return false;
+  if (!make_lin(ctx, &ctx->dqkv, B, 3 * d, d, xn, xl, d, w.wqkv, ctx->qkv, nullptr, 3 * d, ACC, f32)) return false;
+  if (!make_lin(ctx, &ctx->dwo, B, d, d, ao, al, d, w.wo, ctx->dres, nullptr, d, ACC, f32)) return false;
+  if (!make_lin(ctx, &ctx->dgate, B, F, d, xn, xl, d, w.w_gate, ctx->gu, nullptr, 2 * F, ACC, f32)) return false;
+  if (!make_lin(ctx, &ctx->dup, B, F, d, xn, xl, d, w.w_up, ctx->gu + F, nullptr, 2 * F, ACC, f32)) return false;
+  if (!make_lin(ctx, &ctx->ddown, B, d, F, hf, hl, F, w.w_down, ctx->dres, nullptr, d, ACC, f32)) return false;
   ctx->dhead.assign(ctx->K, Lin());
   for (int k = 0; k < ctx->K; ++k)
     if (!make_lin(ctx, &ctx->dhead[k], B, V, 2 * d, ctx->headin, ctx->headin_lo, 2 * d, ctx->heads[k],
-                  ctx->hlog + static_cast<size_t>(k) * B * V, nullptr, V, EPI_STORE, f32))
+                  ctx->hlog + static_cast<size_t>(k) * B * V, nullptr, V, ACC, f32))
       return false;
-  ctx->att_splits_ver = att_splits(ctx, B);
-  ctx->att_splits_pre = att_splits(ctx, B);
-  ctx->att_splits_draft = att_splits(ctx, B);
+  ctx->att_splits_ver = att_splits(ctx, B, N, ctx->plan_keys + N);
+  ctx->att_splits_pre = att_splits(ctx, B, CHUNK, ctx->plan_keys);
+  ctx->att_splits_draft = att_splits(ctx, B, 1, ctx->plan_keys);
   return true;
 }
 
@@ -739,6 +756,8 @@ chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
       (c.precision != 0 && c.precision != 1))
     return CHIMERA_EINVAL;
   if (c.dtype == 1 && (c.d_model % 64 != 0 || c.ffn_dim % 8 != 0)) return CHIMERA_EINVAL;
+  // row kernels read 16-byte vectors; the top-k covers at most 64 slices of 2048 scores
+  if ((c.d_model & 3) || (c.ffn_dim & 3) || (c.vocab & 3) || c.vocab > TOPK_MAX_BLOCKS * 2048) return CHIMERA_EINVAL;
   for (int k = 0; k < c.n_draft_heads; ++k)
     if (c.topk[k] < 1 || c.topk[k] > MAX_KMAX) return CHIMERA_EINVAL;
   if (!w->embed || !w->layers || !w->final_norm || !w->lm_head || !w->tri_w1 || !w->tri_w2 || !w->heads ||
@@ -762,8 +781,8 @@ chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
   ctx->dtype = c.dtype;
   ctx->esz = c.dtype == 0 ? 4 : 2;
   ctx->split = (c.dtype == 1 && c.precision == 1) ? 1 : 0;
-  ctx->kv_f32 = (c.dtype == 0 || c.precision == 1) ? 1 : 0;
-  ctx->kv_esz = ctx->kv_f32 ? 4 : 2;
+  ctx->kv_planes = ctx->split ? 4 : 2;
+  ctx->kv_esz = ctx->esz;
   ctx->Bmax = c.max_batch;
   ctx->cap = c.max_seq_len;
   ctx->KMAX = 1;
@@ -799,7 +818,7 @@ chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
   ctx->tok_stride = ctx->cap + 1;
   ctx->max_pages = (ctx->cap + 15) / 16;
   ctx->NB = B * ctx->max_pages;
-  ctx->kv_layer_stride = static_cast<long long>(ctx->NB) * ctx->H * 2 * 16 * ctx->hd;
+  ctx->kv_layer_stride = static_cast<long long>(ctx->NB) * ctx->H * ctx->kv_planes * 16 * ctx->hd;
   ctx->max_pos = ctx->cap + 64;
   ctx->R = B * std::max(N, CHUNK);
   const int Rc = B * std::max(CHUNK, ctx->D1);
@@ -863,6 +882,9 @@ chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
   ctx->att_ws_floats = attn_ws_floats(B, ctx->H, 16, std::max(N, CHUNK), ctx->hd);
   ok = ok && dalloc(ctx, &ctx->att_ws, ctx->att_ws_floats);
   ok = ok && dalloc(ctx, &ctx->att_cnt, static_cast<size_t>(B) * ctx->H);
+  ok = ok && dalloc(ctx, &ctx->topk_ws_v, static_cast<size_t>(B) * TOPK_MAX_BLOCKS * 8);
+  ok = ok && dalloc(ctx, &ctx->topk_ws_i, static_cast<size_t>(B) * TOPK_MAX_BLOCKS * 8);
+  ok = ok && dalloc(ctx, &ctx->topk_cnt, static_cast<size_t>(B));
   if (ok && cudaMallocHost(reinterpret_cast<void**>(&ctx->h_stage), 4096 * sizeof(int)) != cudaSuccess) ok = false;
   ctx->h_pt_len = static_cast<size_t>(B) * ctx->max_pages;
   if (ok && cudaMallocHost(reinterpret_cast<void**>(&ctx->h_pt), ctx->h_pt_len * sizeof(int)) != cudaSuccess) ok = false;
@@ -879,6 +901,7 @@ chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
   zok = zok && cudaMemsetAsync(ctx->kv, 0, static_cast<size_t>(ctx->kv_layer_stride) * ctx->L * ctx->kv_esz, s) == cudaSuccess;
   zok = zok && cudaMemsetAsync(ctx->dkv, 0, static_cast<size_t>(ctx->kv_layer_stride) * ctx->kv_esz, s) == cudaSuccess;
   zok = zok && cudaMemsetAsync(ctx->att_cnt, 0, static_cast<size_t>(B) * ctx->H * sizeof(int), s) == cudaSuccess;
+  zok = zok && cudaMemsetAsync(ctx->topk_cnt, 0, static_cast<size_t>(B) * sizeof(int), s) == cudaSuccess;
   if (ctx->lin_cnt)
     zok = zok && cudaMemsetAsync(ctx->lin_cnt, 0, static_cast<size_t>(tc_max_tiles()) * sizeof(int), s) == cudaSuccess;
   zok = zok && cudaMemsetAsync(ctx->d_err, 0, sizeof(int), s) == cudaSuccess;
@@ -957,6 +980,7 @@ chimera_status chimera_prefill(chimera_ctx* ctx, int batch, const int32_t* token
     ctx->prof_graph = nullptr;
   }
   ctx->batch = batch;
+  ctx->plan_keys = max_len;
   if (!build_plans(ctx, batch)) return CHIMERA_EINVAL;
   for (int b = 0; b < batch; ++b) {
     chimera_status st = ensure_blocks(ctx, b, lens[b] + need);
@@ -999,9 +1023,9 @@ chimera_status chimera_prefill(chimera_ctx* ctx, int batch, const int32_t* token
     for (int l = 0; l < ctx->L; ++l)
       CK(enqueue_layer(ctx, l, &ctx->pre[5 * l], B * CHUNK, CHUNK, ctx->d_valid, nullptr, ctx->d_chain,
                        ctx->att_splits_pre, 0));
-    CK(run_final_norm(ctx, B * CHUNK));
+    CK(run_final_norm(ctx, B * CHUNK, false));
     // draft-layer K/V of the chunk's H_LLM rows
-    CK(run_norm(ctx, ctx->hfin32, dl_norm, B * CHUNK));
+    CK(run_norm(ctx, ctx->hfin32, dl_norm, B * CHUNK, ctx->kvtmp, 2 * d));
     CK(run_lin(ctx, ctx->pre_dkv));
     CK(run_rope(ctx, true, 0, ctx->kvtmp, 2 * d, -1, 0, d, CHUNK, ctx->d_valid, 0, 0, 0, nullptr));
     CK(launch_prefill_advance(ctx->dtype, ctx->hfin32, d, CHUNK, ctx->d_valid, ctx->d_last, ctx->d_n, ctx->headin,
@@ -1009,6 +1033,7 @@ chimera_status chimera_prefill(chimera_ctx* ctx, int batch, const int32_t* token
     CK(cudaStreamSynchronize(s));  // the staging buffer is reused by the next chunk
   }
   // root = greedy next token of each prompt (eq. 1)
+  CK(cudaMemsetAsync(ctx->logits, 0, static_cast<size_t>(B) * ctx->V * sizeof(float), s));
   CK(run_lin(ctx, ctx->pre_lm));
   CK(argmax_rows(ctx->logits, ctx->V, B, ctx->d_amax, s));
   CK(launch_set_root(ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_amax, B, s));
@@ -1186,18 +1211,36 @@ chimera_status chimera_debug_read_kv(chimera_ctx* ctx, int layer, int seq, int p
       pos0 + count > static_cast<int>(ctx->seq_blocks[seq].size()) * 16 || !k_dst || !v_dst)
     return fail(ctx, CHIMERA_EINVAL, "bad KV read");
   CK(cudaStreamSynchronize(ctx->stream));
-  const size_t row = static_cast<size_t>(ctx->hd) * ctx->kv_esz;
+  const int P = ctx->kv_planes, hd = ctx->hd;
+  const size_t row = static_cast<size_t>(hd) * ctx->kv_esz;
   const char* pool = static_cast<const char*>(layer < 0 ? ctx->dkv : ctx->kv) +
                      (layer < 0 ? 0 : static_cast<size_t>(layer) * ctx->kv_layer_stride * ctx->kv_esz);
+  std::vector<uint16_t> tmp(static_cast<size_t>(P) * hd);
   for (int i = 0; i < count; ++i) {
     const int slot = pos0 + i;
     const int page = ctx->h_pt[seq * ctx->max_pages + slot / 16];
     for (int h = 0; h < ctx->H; ++h) {
-      const char* base = pool + ((static_cast<size_t>(page) * ctx->H + h) * 2) * 16 * row + (slot % 16) * row;
-      CK(cudaMemcpy(static_cast<char*>(k_dst) + (static_cast<size_t>(i) * ctx->H + h) * row, base, row,
-                    cudaMemcpyDeviceToHost));
-      CK(cudaMemcpy(static_cast<char*>(v_dst) + (static_cast<size_t>(i) * ctx->H + h) * row, base + 16 * row, row,
-                    cudaMemcpyDeviceToHost));
+      const char* base = pool + ((static_cast<size_t>(page) * ctx->H + h) * P) * 16 * row + (slot % 16) * row;
+      const size_t o = (static_cast<size_t>(i) * ctx->H + h);
+      if (P == 2) {
+        CK(cudaMemcpy(static_cast<char*>(k_dst) + o * row, base, row, cudaMemcpyDeviceToHost));
+        CK(cudaMemcpy(static_cast<char*>(v_dst) + o * row, base + 16 * row, row, cudaMemcpyDeviceToHost));
+      } else {  // split planes: return hi + lo as fp32
+        for (int pl = 0; pl < 4; ++pl)
+          CK(cudaMemcpy(tmp.data() + pl * hd, base + pl * 16 * row, row, cudaMemcpyDeviceToHost));
+        float* kd = static_cast<float*>(k_dst) + o * hd;
+        float* vd = static_cast<float*>(v_dst) + o * hd;
+        auto bf = [](uint16_t u) {
+          uint32_t x = static_cast<uint32_t>(u) << 16;
+          float f;
+          memcpy(&f, &x, 4);
+          return f;
+        };
+        for (int j = 0; j < hd; ++j) {
+          kd[j] = bf(tmp[j]) + bf(tmp[hd + j]);
+          vd[j] = bf(tmp[2 * hd + j]) + bf(tmp[3 * hd + j]);
+        }
+      }
     }
   }
   return CHIMERA_OK;
@@ -1260,7 +1303,7 @@ chimera_status chimera_op_linear(int dtype, int epi, int out_f32, int M, int N, 
   return tc_linear_launch(plan, s) == cudaSuccess ? CHIMERA_OK : CHIMERA_ECUDA;
 }
 
-chimera_status chimera_op_attention(int dtype, int kv_f32, int batch, int n_heads, int head_dim, int nq, int q_local0,
+chimera_status chimera_op_attention(int dtype, int kv_split, int batch, int n_heads, int head_dim, int nq, int q_local0,
                                     int n_local, const float* q, int ldq, int q_rows, const void* pool,
                                     const int32_t* page_table, int max_pages, const int32_t* n_ctx, const uint64_t* anc,
                                     void* out, void* out_lo, int ldo, int splits, void* cuda_stream) {
@@ -1279,6 +1322,7 @@ chimera_status chimera_op_attention(int dtype, int kv_f32, int batch, int n_head
   p.n_local = n_local;
   p.anc = reinterpret_cast<const unsigned long long*>(anc);
   p.pool = pool;
+  p.planes = (dtype == 1 && kv_split) ? 4 : 2;
   p.page_table = page_table;
   p.max_pages = max_pages;
   p.n_ctx = n_ctx;
@@ -1294,7 +1338,7 @@ chimera_status chimera_op_attention(int dtype, int kv_f32, int batch, int n_head
   p.counters = g_op.att_cnt;
   p.nq_max = nq;
   if (attn_ws_floats(batch, n_heads, splits, nq, head_dim) > g_op.att_floats) return CHIMERA_EINVAL;
-  return attention(p, dtype, dtype == 0 ? 1 : kv_f32, static_cast<cudaStream_t>(cuda_stream)) == cudaSuccess
+  return attention(p, dtype, static_cast<cudaStream_t>(cuda_stream)) == cudaSuccess
              ? CHIMERA_OK
              : CHIMERA_ECUDA;
 }

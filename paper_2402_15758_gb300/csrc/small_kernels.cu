@@ -30,26 +30,110 @@ __device__ float block_sum(float v, float* red) {
 
 // RMSNorm (Llama): y = x / sqrt(mean(x^2) + eps) * g, from the fp32 residual stream.
 // Writes the GEMM operand (model dtype, optional lo half) and an optional fp32 copy.
+// Side job: zero row r of Z (the fp32 output that the next linear accumulates into).
+constexpr int NORM_THREADS = 256;
+constexpr int NORM_VEC = 8;  // float4 per thread: d <= 8192
+
 template <typename T>
-__global__ void rmsnorm_kernel(const float* __restrict__ X, int ldx, const T* __restrict__ g,
-                               T* __restrict__ Y, T* __restrict__ Y_lo, float* __restrict__ Y32,
-                               int ldy, int d, float eps) {
+__device__ __forceinline__ void store_act4(T* hi, T* lo, size_t i, float4 v) {
+  store_act(hi, lo, i, v.x);
+  store_act(hi, lo, i + 1, v.y);
+  store_act(hi, lo, i + 2, v.z);
+  store_act(hi, lo, i + 3, v.w);
+}
+
+template <typename T>
+__device__ __forceinline__ float4 load_g4(const T* g, int i);
+template <>
+__device__ __forceinline__ float4 load_g4<float>(const float* g, int i) {
+  return *reinterpret_cast<const float4*>(g + i);
+}
+template <>
+__device__ __forceinline__ float4 load_g4<bf16>(const bf16* g, int i) {
+  const uint2 u = *reinterpret_cast<const uint2*>(g + i);
+  const bf16* h = reinterpret_cast<const bf16*>(&u);
+  return make_float4(__bfloat162float(h[0]), __bfloat162float(h[1]), __bfloat162float(h[2]), __bfloat162float(h[3]));
+}
+
+// One block per row; every thread loads its (<= NORM_VEC) float4 of the row at once.
+template <typename T>
+__global__ void __launch_bounds__(NORM_THREADS) rmsnorm_kernel(const float* __restrict__ X, int ldx,
+                                                               const T* __restrict__ g, T* __restrict__ Y,
+                                                               T* __restrict__ Y_lo, float* __restrict__ Y32,
+                                                               int ldy, int d, float eps, float* __restrict__ Z,
+                                                               int ldz, int zcols) {
   __shared__ float red[33];
   const float* x = X + static_cast<size_t>(blockIdx.x) * ldx;
+  float4 v[NORM_VEC];
   float ss = 0.f;
-  for (int i = threadIdx.x; i < d; i += blockDim.x) ss = fmaf(x[i], x[i], ss);
+#pragma unroll
+  for (int k = 0; k < NORM_VEC; ++k) {
+    const int i = (threadIdx.x + k * NORM_THREADS) * 4;
+    v[k] = i < d ? *reinterpret_cast<const float4*>(x + i) : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+#pragma unroll
+  for (int k = 0; k < NORM_VEC; ++k) ss += v[k].x * v[k].x + v[k].y * v[k].y + v[k].z * v[k].z + v[k].w * v[k].w;
+  if (Z) {
+    float4* z = reinterpret_cast<float4*>(Z + static_cast<size_t>(blockIdx.x) * ldz);
+    for (int i = threadIdx.x; i < zcols / 4; i += NORM_THREADS) z[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+  }
   ss = block_sum(ss, red);
   const float r = rsqrtf(ss / static_cast<float>(d) + eps);
   const size_t row = static_cast<size_t>(blockIdx.x) * ldy;
-  for (int i = threadIdx.x; i < d; i += blockDim.x) {
-    const float v = x[i] * r * to_f(g[i]);
-    store_act(Y, Y_lo, row + i, v);
-    if (Y32) Y32[row + i] = v;
+#pragma unroll
+  for (int k = 0; k < NORM_VEC; ++k) {
+    const int i = (threadIdx.x + k * NORM_THREADS) * 4;
+    if (i < d) {
+      const float4 gg = load_g4(g, i);
+      const float4 y = make_float4(v[k].x * r * gg.x, v[k].y * r * gg.y, v[k].z * r * gg.z, v[k].w * r * gg.w);
+      store_act4(Y, Y_lo, row + i, y);
+      if (Y32) *reinterpret_cast<float4*>(Y32 + row + i) = y;
+    }
   }
 }
 
 // Rotate-half RoPE of q and k, plus the write of k and v into the paged cache
-// (T = element type of the cache).
+// (T = element type of the cache).  One block per row; an item is 4 consecutive
+// pair indices j..j+3 of one head (pairs (j, j + hd/2)).
+template <typename T>
+__device__ __forceinline__ void store4(T* dst, float4 v);
+template <>
+__device__ __forceinline__ void store4<float>(float* dst, float4 v) { *reinterpret_cast<float4*>(dst) = v; }
+template <>
+__device__ __forceinline__ void store4<bf16>(bf16* dst, float4 v) {
+  __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y), b = __floats2bfloat162_rn(v.z, v.w);
+  uint2 u;
+  u.x = *reinterpret_cast<uint32_t*>(&a);
+  u.y = *reinterpret_cast<uint32_t*>(&b);
+  *reinterpret_cast<uint2*>(dst) = u;
+}
+
+// Two-term bf16 split of 4 values into a hi plane and a lo plane.
+template <typename T>
+__device__ __forceinline__ void store4_split(T* hi, T* lo, float4 v) {
+  store4<T>(hi, v);
+}
+template <>
+__device__ __forceinline__ void store4_split<bf16>(bf16* hi, bf16* lo, float4 v) {
+  __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y), b = __floats2bfloat162_rn(v.z, v.w);
+  const float2 fa = __bfloat1622float2(a), fb = __bfloat1622float2(b);
+  __nv_bfloat162 la = __floats2bfloat162_rn(v.x - fa.x, v.y - fa.y), lb = __floats2bfloat162_rn(v.z - fb.x, v.w - fb.y);
+  uint2 u, w;
+  u.x = *reinterpret_cast<uint32_t*>(&a);
+  u.y = *reinterpret_cast<uint32_t*>(&b);
+  w.x = *reinterpret_cast<uint32_t*>(&la);
+  w.y = *reinterpret_cast<uint32_t*>(&lb);
+  *reinterpret_cast<uint2*>(hi) = u;
+  *reinterpret_cast<uint2*>(lo) = w;
+}
+
+__device__ __forceinline__ float4 rot_lo(float4 x1, float4 x2, float4 c, float4 s) {
+  return make_float4(x1.x * c.x - x2.x * s.x, x1.y * c.y - x2.y * s.y, x1.z * c.z - x2.z * s.z, x1.w * c.w - x2.w * s.w);
+}
+__device__ __forceinline__ float4 rot_hi(float4 x1, float4 x2, float4 c, float4 s) {
+  return make_float4(x2.x * c.x + x1.x * s.x, x2.y * c.y + x1.y * s.y, x2.z * c.z + x1.z * s.z, x2.w * c.w + x1.w * s.w);
+}
+
 template <typename T>
 __global__ void rope_kv_kernel(const RopeKvParams p) {
   const int row = blockIdx.x;
@@ -75,24 +159,46 @@ __global__ void rope_kv_kernel(const RopeKvParams p) {
   }
   const float* src = p.qkv + static_cast<size_t>(row) * p.ldqkv;
   T* pool = static_cast<T*>(p.pool) + static_cast<size_t>(p.layer) * p.pool_layer_stride;
-  for (int idx = threadIdx.x; idx < p.H * half; idx += blockDim.x) {
-    const int h = idx / half, j = idx % half;
-    const float2 cs = p.rope[static_cast<size_t>(pos) * half + j];
+  const float2* tab = p.rope + static_cast<size_t>(pos) * half;
+  const int per_head = half / 4;
+  for (int it = threadIdx.x; it < p.H * per_head; it += blockDim.x) {
+    const int h = it / per_head, j = (it % per_head) * 4;
+    const float4 cs01 = *reinterpret_cast<const float4*>(tab + j);
+    const float4 cs23 = *reinterpret_cast<const float4*>(tab + j + 2);
+    const float4 c = make_float4(cs01.x, cs01.z, cs23.x, cs23.z);
+    const float4 sn = make_float4(cs01.y, cs01.w, cs23.y, cs23.w);
+    const int hb = h * p.hd + j;
+    float4 q1, q2, k1, k2, v1, v2;
     if (p.q_col >= 0) {
-      const float x1 = src[p.q_col + h * p.hd + j];
-      const float x2 = src[p.q_col + h * p.hd + j + half];
-      float* qo = p.q_out + static_cast<size_t>(row) * p.ldq + h * p.hd;
-      qo[j] = x1 * cs.x - x2 * cs.y;
-      qo[j + half] = x2 * cs.x + x1 * cs.y;
+      q1 = *reinterpret_cast<const float4*>(src + p.q_col + hb);
+      q2 = *reinterpret_cast<const float4*>(src + p.q_col + hb + half);
     }
     if (page >= 0) {
-      T* base = pool + (static_cast<size_t>(page) * p.H + h) * 2 * 16 * p.hd + (slot & 15) * p.hd;
-      const float k1 = src[p.k_col + h * p.hd + j];
-      const float k2 = src[p.k_col + h * p.hd + j + half];
-      base[j] = from_f<T>(k1 * cs.x - k2 * cs.y);
-      base[j + half] = from_f<T>(k2 * cs.x + k1 * cs.y);
-      base[16 * p.hd + j] = from_f<T>(src[p.v_col + h * p.hd + j]);
-      base[16 * p.hd + j + half] = from_f<T>(src[p.v_col + h * p.hd + j + half]);
+      k1 = *reinterpret_cast<const float4*>(src + p.k_col + hb);
+      k2 = *reinterpret_cast<const float4*>(src + p.k_col + hb + half);
+      v1 = *reinterpret_cast<const float4*>(src + p.v_col + hb);
+      v2 = *reinterpret_cast<const float4*>(src + p.v_col + hb + half);
+    }
+    if (p.q_col >= 0) {
+      float* qo = p.q_out + static_cast<size_t>(row) * p.ldq + hb;
+      *reinterpret_cast<float4*>(qo) = rot_lo(q1, q2, c, sn);
+      *reinterpret_cast<float4*>(qo + half) = rot_hi(q1, q2, c, sn);
+    }
+    if (page >= 0) {
+      T* base = pool + (static_cast<size_t>(page) * p.H + h) * p.planes * 16 * p.hd + (slot & 15) * p.hd + j;
+      const size_t plane = 16 * static_cast<size_t>(p.hd);
+      const float4 ka = rot_lo(k1, k2, c, sn), kb = rot_hi(k1, k2, c, sn);
+      if (p.planes == 4) {  // K_hi, K_lo, V_hi, V_lo
+        store4_split(base, base + plane, ka);
+        store4_split(base + half, base + plane + half, kb);
+        store4_split(base + 2 * plane, base + 3 * plane, v1);
+        store4_split(base + 2 * plane + half, base + 3 * plane + half, v2);
+      } else {
+        store4<T>(base, ka);
+        store4<T>(base + half, kb);
+        store4<T>(base + plane, v1);
+        store4<T>(base + plane + half, v2);
+      }
     }
   }
 }
@@ -103,8 +209,11 @@ __global__ void swiglu_kernel(const float* __restrict__ gu, int ldgu, int F, T* 
                               T* __restrict__ h_lo, int ldh) {
   const float* g = gu + static_cast<size_t>(blockIdx.y) * ldgu;
   const size_t row = static_cast<size_t>(blockIdx.y) * ldh;
-  for (int f = blockIdx.x * blockDim.x + threadIdx.x; f < F; f += gridDim.x * blockDim.x)
-    store_act(h, h_lo, row + f, silu_f(g[f]) * g[F + f]);
+  const int f = (blockIdx.x * blockDim.x + threadIdx.x) * 4;
+  if (f >= F) return;
+  const float4 a = *reinterpret_cast<const float4*>(g + f);
+  const float4 u = *reinterpret_cast<const float4*>(g + F + f);
+  store_act4(h, h_lo, row + f, make_float4(silu_f(a.x) * u.x, silu_f(a.y) * u.y, silu_f(a.z) * u.z, silu_f(a.w) * u.w));
 }
 
 template <typename T>
@@ -125,7 +234,7 @@ __global__ void embed_kernel(const T* __restrict__ E, int d, int V, float* __res
   }
   const T* e = E + static_cast<size_t>(tok) * d;
   float* y = x + static_cast<size_t>(r) * d;
-  for (int i = threadIdx.x; i < d; i += blockDim.x) y[i] = to_f(e[i]);
+  for (int i = threadIdx.x * 4; i < d; i += blockDim.x * 4) *reinterpret_cast<float4*>(y + i) = load_g4(e, i);
 }
 
 // (value, index) order of the method: larger value first, then smaller index.
@@ -133,19 +242,32 @@ __device__ __forceinline__ bool better(float v, int i, float bv, int bi) {
   return v > bv || (v == bv && i < bi);
 }
 
-__global__ void argmax_kernel(const float* __restrict__ logits, int V, int* __restrict__ out) {
+__global__ void __launch_bounds__(512) argmax_kernel(const float* __restrict__ logits, int V, int* __restrict__ out) {
   __shared__ float sv[32];
   __shared__ int si[32];
   const float* z = logits + static_cast<size_t>(blockIdx.x) * V;
   float bv = -INFINITY;
   int bi = 0x7fffffff;
-  for (int i = threadIdx.x; i < V; i += blockDim.x) {
-    const float v = z[i];
-    if (better(v, i, bv, bi)) {
-      bv = v;
-      bi = i;
+  const int V4 = V / 4;
+  for (int base = threadIdx.x; base < V4; base += 4 * blockDim.x) {
+    float4 v[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int i4 = base + u * blockDim.x;
+      v[u] = i4 < V4 ? *reinterpret_cast<const float4*>(z + 4 * i4) : make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      if (base + u * static_cast<int>(blockDim.x) >= V4) break;
+      const int i = 4 * (base + u * blockDim.x);
+      if (better(v[u].x, i, bv, bi)) { bv = v[u].x; bi = i; }
+      if (better(v[u].y, i + 1, bv, bi)) { bv = v[u].y; bi = i + 1; }
+      if (better(v[u].z, i + 2, bv, bi)) { bv = v[u].z; bi = i + 2; }
+      if (better(v[u].w, i + 3, bv, bi)) { bv = v[u].w; bi = i + 3; }
     }
   }
+  for (int i = 4 * V4 + threadIdx.x; i < V; i += blockDim.x)
+    if (better(z[i], i, bv, bi)) { bv = z[i]; bi = i; }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
@@ -180,37 +302,33 @@ __global__ void argmax_kernel(const float* __restrict__ logits, int V, int* __re
 
 constexpr int TOPK_MAX = 8;
 
-// Top-k of a row: every thread keeps a sorted list of its strided elements; then k
-// rounds of a block-wide arg-best over the list heads.
-__global__ void topk_kernel(const float* __restrict__ logits, int V, int k, int* __restrict__ idx,
-                            float* __restrict__ val, int out_stride) {
+// Top-k of a row in two levels: each block selects the top-k of a 2048-score slice
+// (every thread keeps a sorted register list of its 8 scores, then k rounds of a
+// block-wide arg-best), writes its k candidates, and the last block of the row to
+// finish merges the candidates (counter per row, reset by the merger).
+constexpr int TOPK_THREADS = 256;
+constexpr int TOPK_SLICE = TOPK_THREADS * 8;
+
+__device__ __forceinline__ void topk_insert(float (&lv)[TOPK_MAX], int (&li)[TOPK_MAX], int k, float v, int ii) {
+#pragma unroll
+  for (int j = 0; j < TOPK_MAX; ++j) {
+    if (j < k && better(v, ii, lv[j], li[j])) {
+      const float sv2 = lv[j];
+      const int si2 = li[j];
+      lv[j] = v;
+      li[j] = ii;
+      v = sv2;
+      ii = si2;
+    }
+  }
+}
+
+// k rounds of block-wide arg-best over the heads of the per-thread sorted lists;
+// round r's winner is written to (out_v[r], out_i[r]) by thread 0.
+__device__ void topk_block_select(float (&lv)[TOPK_MAX], int (&li)[TOPK_MAX], int k, float* out_v, int* out_i) {
   __shared__ float sv[32];
   __shared__ int si[32];
   __shared__ int s_win;
-  const float* z = logits + static_cast<size_t>(blockIdx.x) * V;
-  float lv[TOPK_MAX];
-  int li[TOPK_MAX];
-#pragma unroll
-  for (int j = 0; j < TOPK_MAX; ++j) {
-    lv[j] = -INFINITY;
-    li[j] = 0x7fffffff;
-  }
-  for (int i = threadIdx.x; i < V; i += blockDim.x) {
-    float v = z[i];
-    int ii = i;
-    if (!better(v, ii, lv[k - 1], li[k - 1])) continue;
-#pragma unroll
-    for (int j = 0; j < TOPK_MAX; ++j) {
-      if (j < k && better(v, ii, lv[j], li[j])) {
-        const float tv = lv[j];
-        const int ti = li[j];
-        lv[j] = v;
-        li[j] = ii;
-        v = tv;
-        ii = ti;
-      }
-    }
-  }
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   int head = 0;
   for (int r = 0; r < k; ++r) {
@@ -253,8 +371,8 @@ __global__ void topk_kernel(const float* __restrict__ logits, int V, int k, int*
       }
       if (lane == 0) {
         s_win = ci;
-        idx[static_cast<size_t>(blockIdx.x) * out_stride + r] = ci < V ? ci : 0;
-        if (val) val[static_cast<size_t>(blockIdx.x) * out_stride + r] = cv;
+        out_v[r] = cv;
+        out_i[r] = ci;
       }
     }
     __syncthreads();
@@ -263,24 +381,98 @@ __global__ void topk_kernel(const float* __restrict__ logits, int V, int k, int*
   }
 }
 
+__global__ void __launch_bounds__(TOPK_THREADS) topk_kernel(const float* __restrict__ logits, int V, int k,
+                                                            int* __restrict__ idx, float* __restrict__ val,
+                                                            int out_stride, float* __restrict__ ws_v,
+                                                            int* __restrict__ ws_i, int* __restrict__ counters) {
+  __shared__ float s_bv[TOPK_MAX];
+  __shared__ int s_bi[TOPK_MAX];
+  __shared__ int s_last;
+  const int row = blockIdx.y, blk = blockIdx.x, nblk = gridDim.x;
+  const float* z = logits + static_cast<size_t>(row) * V;
+  float lv[TOPK_MAX];
+  int li[TOPK_MAX];
+#pragma unroll
+  for (int j = 0; j < TOPK_MAX; ++j) {
+    lv[j] = -INFINITY;
+    li[j] = 0x7fffffff;
+  }
+  // this thread's 8 scores: two float4 of the slice (V is a multiple of 4)
+  const int s0 = blk * TOPK_SLICE;
+  float4 v[2];
+  int i0[2];
+#pragma unroll
+  for (int u = 0; u < 2; ++u) {
+    i0[u] = s0 + (threadIdx.x + u * TOPK_THREADS) * 4;
+    v[u] = i0[u] < V ? *reinterpret_cast<const float4*>(z + i0[u]) : make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+  }
+#pragma unroll
+  for (int u = 0; u < 2; ++u) {
+    if (i0[u] >= V) continue;
+    topk_insert(lv, li, k, v[u].x, i0[u]);
+    topk_insert(lv, li, k, v[u].y, i0[u] + 1);
+    topk_insert(lv, li, k, v[u].z, i0[u] + 2);
+    topk_insert(lv, li, k, v[u].w, i0[u] + 3);
+  }
+  const size_t wbase = (static_cast<size_t>(row) * nblk + blk) * TOPK_MAX;
+  if (nblk == 1) {
+    topk_block_select(lv, li, k, s_bv, s_bi);
+  } else {
+    topk_block_select(lv, li, k, ws_v + wbase, ws_i + wbase);
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      const int old = atomicAdd(&counters[row], 1);
+      s_last = (old == nblk - 1) ? 1 : 0;
+    }
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();
+    // merge: thread t holds candidates t, t + 256, ... of the nblk * k list
+#pragma unroll
+    for (int j = 0; j < TOPK_MAX; ++j) {
+      lv[j] = -INFINITY;
+      li[j] = 0x7fffffff;
+    }
+    const int ncand = nblk * k;
+    for (int c = threadIdx.x; c < ncand; c += TOPK_THREADS) {
+      const size_t o = static_cast<size_t>(row) * nblk * TOPK_MAX + (c / k) * TOPK_MAX + (c % k);
+      topk_insert(lv, li, k, __ldcg(ws_v + o), __ldcg(ws_i + o));
+    }
+    topk_block_select(lv, li, k, s_bv, s_bi);
+    if (threadIdx.x == 0) counters[row] = 0;
+  }
+  if (threadIdx.x < k) {
+    const int ci = s_bi[threadIdx.x];
+    idx[static_cast<size_t>(row) * out_stride + threadIdx.x] = ci < V ? ci : 0;
+    if (val) val[static_cast<size_t>(row) * out_stride + threadIdx.x] = s_bv[threadIdx.x];
+  }
+}
+
 }  // namespace
 
 cudaError_t rmsnorm(int dtype, const float* X, int ldx, const void* g, void* Y, void* Y_lo, float* Y32,
-                    int ldy, int rows, int d, float eps, cudaStream_t s) {
+                    int ldy, int rows, int d, float eps, float* Z, int ldz, int zcols, cudaStream_t s) {
   if (rows <= 0) return cudaSuccess;
+  if (Z && ((zcols & 3) || (ldz & 3) || (reinterpret_cast<uintptr_t>(Z) & 15))) return cudaErrorInvalidValue;
+  if ((d & 3) || (ldx & 3) || (ldy & 3) || d > NORM_THREADS * NORM_VEC * 4) return cudaErrorInvalidValue;
   if (dtype == 0)
-    rmsnorm_kernel<float><<<rows, 256, 0, s>>>(X, ldx, static_cast<const float*>(g), static_cast<float*>(Y),
-                                               nullptr, Y32, ldy, d, eps);
+    rmsnorm_kernel<float><<<rows, NORM_THREADS, 0, s>>>(X, ldx, static_cast<const float*>(g), static_cast<float*>(Y),
+                                               nullptr, Y32, ldy, d, eps, Z, ldz, zcols);
   else
-    rmsnorm_kernel<bf16><<<rows, 256, 0, s>>>(X, ldx, static_cast<const bf16*>(g), static_cast<bf16*>(Y),
-                                              static_cast<bf16*>(Y_lo), Y32, ldy, d, eps);
+    rmsnorm_kernel<bf16><<<rows, NORM_THREADS, 0, s>>>(X, ldx, static_cast<const bf16*>(g), static_cast<bf16*>(Y),
+                                              static_cast<bf16*>(Y_lo), Y32, ldy, d, eps, Z, ldz, zcols);
   return cudaGetLastError();
 }
 
-cudaError_t rope_kv(const RopeKvParams& p, int kv_f32, cudaStream_t s) {
+cudaError_t rope_kv(const RopeKvParams& p, int dtype, cudaStream_t s) {
   const int rows = p.B * p.rows_per_seq;
   if (rows <= 0) return cudaSuccess;
-  if (kv_f32)
+  if ((p.hd & 15) || (p.ldqkv & 3) || (p.ldq & 3) || (p.q_col >= 0 && (p.q_col & 3)) || (p.k_col & 3) ||
+      (p.v_col & 3))
+    return cudaErrorInvalidValue;
+  if (p.planes != 2 && !(p.planes == 4 && dtype == 1)) return cudaErrorInvalidValue;
+  if (dtype == 0)
     rope_kv_kernel<float><<<rows, 256, 0, s>>>(p);
   else
     rope_kv_kernel<bf16><<<rows, 256, 0, s>>>(p);
@@ -290,7 +482,8 @@ cudaError_t rope_kv(const RopeKvParams& p, int kv_f32, cudaStream_t s) {
 cudaError_t swiglu(int dtype, const float* gu, int ldgu, int F, void* h, void* h_lo, int ldh, int rows,
                    cudaStream_t s) {
   if (rows <= 0) return cudaSuccess;
-  dim3 grid((F + 255) / 256, rows);
+  if ((F & 3) || (ldh & 3)) return cudaErrorInvalidValue;
+  dim3 grid((F / 4 + 255) / 256, rows);
   if (dtype == 0)
     swiglu_kernel<float><<<grid, 256, 0, s>>>(gu, ldgu, F, static_cast<float*>(h), nullptr, ldh);
   else
@@ -313,15 +506,19 @@ cudaError_t embed(int dtype, const void* E, int d, int V, float* x, int rows, in
 
 cudaError_t argmax_rows(const float* logits, int V, int rows, int* out, cudaStream_t s) {
   if (rows <= 0) return cudaSuccess;
+  if (V & 3) return cudaErrorInvalidValue;  // rows are read as float4
   argmax_kernel<<<rows, 512, 0, s>>>(logits, V, out);
   return cudaGetLastError();
 }
 
-cudaError_t topk_rows(const float* logits, int V, int rows, int k, int* idx, float* val,
-                      int out_stride, cudaStream_t s) {
+cudaError_t topk_rows(const float* logits, int V, int rows, int k, int* idx, float* val, int out_stride,
+                      float* ws_v, int* ws_i, int* counters, cudaStream_t s) {
   if (rows <= 0) return cudaSuccess;
-  if (k < 1 || k > TOPK_MAX) return cudaErrorInvalidValue;
-  topk_kernel<<<rows, 512, 0, s>>>(logits, V, k, idx, val, out_stride);
+  if (k < 1 || k > TOPK_MAX || (V & 3)) return cudaErrorInvalidValue;
+  const int nblk = (V + TOPK_SLICE - 1) / TOPK_SLICE;
+  if (nblk > TOPK_MAX_BLOCKS) return cudaErrorInvalidValue;
+  dim3 grid(nblk, rows);
+  topk_kernel<<<grid, TOPK_THREADS, 0, s>>>(logits, V, k, idx, val, out_stride, ws_v, ws_i, counters);
   return cudaGetLastError();
 }
 

@@ -9,12 +9,15 @@ namespace {
 // Trigram input of draft sub-step k (eq. trigram_calculations): the embeddings of
 // x[n-2+k], x[n-1+k], x[n+k], where x[n] is the root and x[n+1+j] is head j's top-1.
 // A position before the start of the sequence contributes a zero block.
+// Also zeroes row b of `zero` (d floats): the draft residual that W2 accumulates into.
 template <typename T>
 __global__ void trigram_gather_kernel(const T* __restrict__ E, int d, int V, const int* n_arr,
                                       const int* tok, int tok_stride, const int* topk, int K,
-                                      int KMAX, int k, T* __restrict__ out, int* err) {
+                                      int KMAX, int k, T* __restrict__ out, int* err, float* __restrict__ zero) {
   const int b = blockIdx.x;
   const int n = n_arr[b];
+  for (int c = threadIdx.x * 4; c < d; c += blockDim.x * 4)
+    *reinterpret_cast<float4*>(zero + static_cast<size_t>(b) * d + c) = make_float4(0.f, 0.f, 0.f, 0.f);
   for (int t = 0; t < 3; ++t) {
     const int i = n - 2 + k + t;
     int id = -1;
@@ -26,19 +29,30 @@ __global__ void trigram_gather_kernel(const T* __restrict__ E, int d, int V, con
     }
     T* o = out + static_cast<size_t>(b) * 3 * d + t * d;
     const T* e = E + static_cast<size_t>(id < 0 ? 0 : id) * d;
-    for (int c = threadIdx.x; c < d; c += blockDim.x) o[c] = id < 0 ? from_f<T>(0.f) : e[c];
+    // 16-byte chunks (d * sizeof(T) is a multiple of 16)
+    constexpr int PER = 16 / sizeof(T);
+    for (int c = threadIdx.x * PER; c < d; c += blockDim.x * PER)
+      *reinterpret_cast<uint4*>(o + c) = id < 0 ? make_uint4(0, 0, 0, 0) : *reinterpret_cast<const uint4*>(e + c);
   }
 }
 
-// headin[b][d..2d) = h_full (the draft block output), kept per head for debugging.
+// headin[b][d..2d) = h_full (the draft block output), kept per head for debugging;
+// also zeroes row b of the head's score buffer (V floats) that its linear accumulates into.
 template <typename T>
 __global__ void hfull_store_kernel(const float* __restrict__ dres, int d, T* __restrict__ headin,
-                                   T* __restrict__ headin_lo, float* __restrict__ hlog) {
+                                   T* __restrict__ headin_lo, float* __restrict__ hlog,
+                                   float* __restrict__ zero, int V) {
   const int b = blockIdx.x;
-  for (int c = threadIdx.x; c < d; c += blockDim.x) {
-    const float v = dres[static_cast<size_t>(b) * d + c];
-    store_act(headin, headin_lo, static_cast<size_t>(b) * 2 * d + d + c, v);
-    hlog[static_cast<size_t>(b) * d + c] = v;
+  for (int c = threadIdx.x * 4; c < V; c += blockDim.x * 4)
+    *reinterpret_cast<float4*>(zero + static_cast<size_t>(b) * V + c) = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int c = threadIdx.x * 4; c < d; c += blockDim.x * 4) {
+    const float4 v = *reinterpret_cast<const float4*>(dres + static_cast<size_t>(b) * d + c);
+    const size_t o = static_cast<size_t>(b) * 2 * d + d + c;
+    store_act(headin, headin_lo, o, v.x);
+    store_act(headin, headin_lo, o + 1, v.y);
+    store_act(headin, headin_lo, o + 2, v.z);
+    store_act(headin, headin_lo, o + 3, v.w);
+    *reinterpret_cast<float4*>(hlog + static_cast<size_t>(b) * d + c) = v;
   }
 }
 
@@ -93,14 +107,14 @@ __global__ void accept_kernel(const int* n_arr, int* tok, int tok_stride, const 
 // Move the accepted nodes' K/V rows from tree slot n+path[j] to slot n+j (j = 1..L)
 // in every layer.  All source rows are loaded before any store: a destination slot
 // can be the source of another path entry.
-__global__ void compact_kernel(char* pool, long long layer_stride_bytes, int H, int row_bytes,
+__global__ void compact_kernel(char* pool, long long layer_stride_bytes, int H, int planes, int row_bytes,
                                const int* n_arr, const int* path, const int* Lacc, int D1,
                                const int* page_table, int max_pages) {
   const int b = blockIdx.y;
   const int L = Lacc[b];
   if (L == 0) return;
-  const int layer = blockIdx.x / (2 * H);
-  const int kv = (blockIdx.x / H) & 1;
+  const int layer = blockIdx.x / (planes * H);
+  const int kv = (blockIdx.x / H) % planes;  // plane index
   const int h = blockIdx.x % H;
   const int n = n_arr[b];
   const int chunks = row_bytes / 16;
@@ -109,7 +123,7 @@ __global__ void compact_kernel(char* pool, long long layer_stride_bytes, int H, 
   char* base = pool + layer * layer_stride_bytes;
   auto row_ptr = [&](int slot) {
     const int page = page_table[b * max_pages + (slot >> 4)];
-    return reinterpret_cast<uint4*>(base + ((static_cast<size_t>(page) * H + h) * 2 + kv) * 16 * row_bytes +
+    return reinterpret_cast<uint4*>(base + ((static_cast<size_t>(page) * H + h) * planes + kv) * 16 * row_bytes +
                                     static_cast<size_t>(slot & 15) * row_bytes) + c;
   };
   uint4 v = make_uint4(0, 0, 0, 0);
@@ -178,23 +192,23 @@ __global__ void set_root_kernel(const int* n_arr, int* tok, int tok_stride, cons
 
 cudaError_t launch_trigram_gather(int dtype, const void* E, int d, int V, const int* n, const int* tok,
                                   int tok_stride, const int* topk, int K, int KMAX, int k, void* out,
-                                  int B, int* err, cudaStream_t s) {
+                                  int B, int* err, float* zero, cudaStream_t s) {
   if (dtype == 0)
     trigram_gather_kernel<float><<<B, 256, 0, s>>>(static_cast<const float*>(E), d, V, n, tok, tok_stride,
-                                                   topk, K, KMAX, k, static_cast<float*>(out), err);
+                                                   topk, K, KMAX, k, static_cast<float*>(out), err, zero);
   else
     trigram_gather_kernel<bf16><<<B, 256, 0, s>>>(static_cast<const bf16*>(E), d, V, n, tok, tok_stride,
-                                                  topk, K, KMAX, k, static_cast<bf16*>(out), err);
+                                                  topk, K, KMAX, k, static_cast<bf16*>(out), err, zero);
   return cudaGetLastError();
 }
 
 cudaError_t launch_hfull_store(int dtype, const float* dres, int d, void* headin, void* headin_lo, float* hlog,
-                               int B, cudaStream_t s) {
+                               float* zero, int V, int B, cudaStream_t s) {
   if (dtype == 0)
-    hfull_store_kernel<float><<<B, 256, 0, s>>>(dres, d, static_cast<float*>(headin), nullptr, hlog);
+    hfull_store_kernel<float><<<B, 256, 0, s>>>(dres, d, static_cast<float*>(headin), nullptr, hlog, zero, V);
   else
     hfull_store_kernel<bf16><<<B, 256, 0, s>>>(dres, d, static_cast<bf16*>(headin), static_cast<bf16*>(headin_lo),
-                                               hlog);
+                                               hlog, zero, V);
   return cudaGetLastError();
 }
 
@@ -213,14 +227,14 @@ cudaError_t launch_accept(const int* n, int* tok, int tok_stride, const int* nod
   return cudaGetLastError();
 }
 
-cudaError_t launch_compact(void* pool, long long layer_stride_bytes, int n_layers, int H, int row_bytes,
+cudaError_t launch_compact(void* pool, long long layer_stride_bytes, int n_layers, int H, int planes, int row_bytes,
                            const int* n, const int* path, const int* Lacc, int D1, const int* page_table,
                            int max_pages, int B, cudaStream_t s) {
   const int threads = (row_bytes / 16) * (D1 - 1);
   if (threads <= 0) return cudaSuccess;
-  dim3 grid(n_layers * 2 * H, B);
-  compact_kernel<<<grid, threads, 0, s>>>(static_cast<char*>(pool), layer_stride_bytes, H, row_bytes, n, path,
-                                          Lacc, D1, page_table, max_pages);
+  dim3 grid(n_layers * planes * H, B);
+  compact_kernel<<<grid, threads, 0, s>>>(static_cast<char*>(pool), layer_stride_bytes, H, planes, row_bytes, n,
+                                          path, Lacc, D1, page_table, max_pages);
   return cudaGetLastError();
 }
 

@@ -7,16 +7,16 @@ namespace chimera {
 
 cudaError_t launch_trigram_gather(int dtype, const void* E, int d, int V, const int* n, const int* tok,
                                   int tok_stride, const int* topk, int K, int KMAX, int k, void* out,
-                                  int B, int* err, cudaStream_t s);
+                                  int B, int* err, float* zero, cudaStream_t s);
 cudaError_t launch_hfull_store(int dtype, const float* dres, int d, void* headin, void* headin_lo, float* hlog,
-                               int B, cudaStream_t s);
+                               float* zero, int V, int B, cudaStream_t s);
 cudaError_t launch_tree_expand(const int* n, const int* tok, int tok_stride, const int* topk, int K, int KMAX,
                                const int* depth, const int* rank, int N, const int* ovr_flag, const int* ovr,
                                int* node_tok, int B, cudaStream_t s);
 cudaError_t launch_accept(const int* n, int* tok, int tok_stride, const int* node_tok, const int* amax,
                           const int* child_start, const int* child, int N, int D1, int* path, int* Lacc,
                           int* bonus, int B, cudaStream_t s);
-cudaError_t launch_compact(void* pool, long long layer_stride_bytes, int n_layers, int H, int row_bytes,
+cudaError_t launch_compact(void* pool, long long layer_stride_bytes, int n_layers, int H, int planes, int row_bytes,
                            const int* n, const int* path, const int* Lacc, int D1, const int* page_table,
                            int max_pages, int B, cudaStream_t s);
 cudaError_t launch_gather_hidden(int dtype, const float* hfin, int d, int N, const int* path, const int* Lacc,
