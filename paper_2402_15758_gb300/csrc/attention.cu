@@ -14,6 +14,7 @@
 #include <cmath>
 
 #include "common.cuh"
+#include "launch.cuh"
 #include "kernels.h"
 
 namespace chimera {
@@ -40,54 +41,88 @@ constexpr int MAX_SPLITS = 16;
 // Merge the per-split partials (unnormalised output, running max, running sum) of the
 // nq queries of one (b, h), in split order.  Run by the last CTA of the pair; every
 // thread takes part: first the per-query weights exp(m_s - M) / L into shared memory,
-// then the outputs, 4 dims per item with the splits' loads in flight together.
+// then the outputs, 4 dims per item, up to 8 items x 4 splits of loads in flight.
 template <typename T>
 __device__ void combine_splits(const AttnParams& p, const float* wsb, int nq, int hd, int b, int h, T* out,
                                T* out_lo, float* s_w /* [nq][MAX_SPLITS] */) {
-  const size_t rec = hd + 4;  // 16-byte aligned records
+  const size_t rec = hd + 4;
   for (int qi = threadIdx.x; qi < nq; qi += blockDim.x) {
+    float mv[MAX_SPLITS], lv[MAX_SPLITS];
+#pragma unroll
+    for (int sp = 0; sp < MAX_SPLITS; ++sp) {
+      mv[sp] = -INFINITY;
+      lv[sp] = 0.f;
+      if (sp < p.splits) {
+        const float* w = wsb + (static_cast<size_t>(sp) * p.nq_max + qi) * rec + hd;
+        mv[sp] = __ldcg(w);
+        lv[sp] = __ldcg(w + 1);
+      }
+    }
     float M = -INFINITY;
-    for (int sp = 0; sp < p.splits; ++sp) M = fmaxf(M, __ldcg(&wsb[(static_cast<size_t>(sp) * p.nq_max + qi) * rec + hd]));
+#pragma unroll
+    for (int sp = 0; sp < MAX_SPLITS; ++sp) M = fmaxf(M, mv[sp]);
     float L = 0.f;
-    for (int sp = 0; sp < p.splits; ++sp) {
-      const float* w = wsb + (static_cast<size_t>(sp) * p.nq_max + qi) * rec;
-      const float ms = __ldcg(&w[hd]);
-      const float e = (M == -INFINITY || ms == -INFINITY) ? 0.f : expf(ms - M);
-      s_w[qi * MAX_SPLITS + sp] = e;
-      L += e * __ldcg(&w[hd + 1]);
+#pragma unroll
+    for (int sp = 0; sp < MAX_SPLITS; ++sp) {
+      mv[sp] = (M == -INFINITY || mv[sp] == -INFINITY) ? 0.f : expf(mv[sp] - M);
+      L += mv[sp] * lv[sp];
     }
     const float inv = L > 0.f ? 1.f / L : 0.f;
-    for (int sp = 0; sp < p.splits; ++sp) s_w[qi * MAX_SPLITS + sp] *= inv;
+#pragma unroll
+    for (int sp = 0; sp < MAX_SPLITS; ++sp)
+      if (sp < p.splits) s_w[qi * MAX_SPLITS + sp] = mv[sp] * inv;
   }
   __syncthreads();
+  constexpr int J = 8;
   const int c4n = hd / 4;
   const int items = nq * c4n;
-  for (int it = threadIdx.x; it < items; it += blockDim.x) {
-    const int qi = it / c4n, c = (it % c4n) * 4;
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  const int nt = blockDim.x;
+  for (int it0 = threadIdx.x; it0 < items; it0 += J * nt) {
+    float4 acc[J];
+#pragma unroll
+    for (int j = 0; j < J; ++j) acc[j] = make_float4(0.f, 0.f, 0.f, 0.f);
     for (int sp0 = 0; sp0 < p.splits; sp0 += 4) {
-      float4 v[4];
+      float4 v[J][4];
 #pragma unroll
-      for (int j = 0; j < 4; ++j)
-        if (sp0 + j < p.splits)
-          v[j] = __ldcg(reinterpret_cast<const float4*>(wsb + (static_cast<size_t>(sp0 + j) * p.nq_max + qi) * rec + c));
+      for (int j = 0; j < J; ++j) {
+        const int it = it0 + j * nt;
+        const int qi = it / c4n, c = (it % c4n) * 4;
 #pragma unroll
-      for (int j = 0; j < 4; ++j)
-        if (sp0 + j < p.splits) {
-          const float e = s_w[qi * MAX_SPLITS + sp0 + j];
-          acc.x += e * v[j].x; acc.y += e * v[j].y; acc.z += e * v[j].z; acc.w += e * v[j].w;
-        }
+        for (int u = 0; u < 4; ++u)
+          if (it < items && sp0 + u < p.splits)
+            v[j][u] = __ldcg(reinterpret_cast<const float4*>(wsb + (static_cast<size_t>(sp0 + u) * p.nq_max + qi) * rec + c));
+      }
+#pragma unroll
+      for (int j = 0; j < J; ++j) {
+        const int it = it0 + j * nt;
+        if (it >= items) continue;
+        const int qi = it / c4n;
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          if (sp0 + u < p.splits) {
+            const float e = s_w[qi * MAX_SPLITS + sp0 + u];
+            acc[j].x += e * v[j][u].x; acc[j].y += e * v[j][u].y; acc[j].z += e * v[j][u].z; acc[j].w += e * v[j][u].w;
+          }
+      }
     }
-    const size_t o = static_cast<size_t>(b * p.q_rows + qi) * p.ldo + h * hd + c;
-    store_act(out, out_lo, o, acc.x);
-    store_act(out, out_lo, o + 1, acc.y);
-    store_act(out, out_lo, o + 2, acc.z);
-    store_act(out, out_lo, o + 3, acc.w);
+#pragma unroll
+    for (int j = 0; j < J; ++j) {
+      const int it = it0 + j * nt;
+      if (it >= items) continue;
+      const int qi = it / c4n, c = (it % c4n) * 4;
+      const size_t o = static_cast<size_t>(b * p.q_rows + qi) * p.ldo + h * hd + c;
+      store_act(out, out_lo, o, acc[j].x);
+      store_act(out, out_lo, o + 1, acc[j].y);
+      store_act(out, out_lo, o + 2, acc[j].z);
+      store_act(out, out_lo, o + 3, acc[j].w);
+    }
   }
 }
 
 template <typename TKV, typename T, int HD>
 __global__ void __launch_bounds__(WARPS * 32) attn_kernel(const AttnParams p) {
+  pdl_trigger();  // the next kernel may start its prologue
+  pdl_wait();     // inputs of this kernel are complete
   // SIMT path: fp32 models and bf16 models with head_dim 64
   constexpr int DPL = HD / 32;
   extern __shared__ float sm[];
@@ -231,10 +266,19 @@ __global__ void __launch_bounds__(WARPS * 32) attn_kernel(const AttnParams p) {
 // in shared memory as bf16 hi/lo planes (padded rows, ldmatrix-friendly); each warp
 // owns 16 queries.
 // ---------------------------------------------------------------------------
+#ifdef CHIMERA_ATTN_TRACE
+// per-CTA timestamps of the last launch (instrumented builds only)
+__device__ unsigned long long g_attn_trace[2048][8];
+#define ATRACE(i) \
+  if (threadIdx.x == 0) g_attn_trace[(blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x][i] = global_timer_ns()
+#else
+#define ATRACE(i)
+#endif
+
 constexpr int MKT = 64;              // keys per tile
 constexpr int MHD = 128;             // head dim
 constexpr int MLDS = MHD + 8;        // smem row pitch (bf16): 272 B, conflict-free ldmatrix
-constexpr int MWARPS = 4;
+constexpr int MWARPS = 8;
 
 __device__ __forceinline__ uint32_t pack_bf16(bf16 a, bf16 b) {
   return static_cast<uint32_t>(__bfloat16_as_ushort(a)) | (static_cast<uint32_t>(__bfloat16_as_ushort(b)) << 16);
@@ -275,8 +319,12 @@ __device__ __forceinline__ void cp_async_wait1() { asm volatile("cp.async.wait_g
 
 // SPLIT: the cache holds K_hi, K_lo, V_hi, V_lo planes (three-term products);
 // otherwise K, V planes (K_lo = V_lo = 0: two-term products for the split queries and P).
+// 8 warps: warp w owns queries 16*(w & 3) .. +15 and the key half (w >> 2) of every
+// 64-key tile; the two halves' online-softmax states merge at the end.
 template <bool SPLIT>
 __global__ void __launch_bounds__(MWARPS * 32) attn_mma_kernel(const AttnParams p) {
+  pdl_trigger();  // the next kernel may start its prologue
+  pdl_wait();     // inputs of this kernel are complete
   constexpr int NP = SPLIT ? 4 : 2;                  // planes per (block, head)
   constexpr int STAGE = NP * MKT * MLDS;             // bf16 elements per pipeline stage
   extern __shared__ __align__(16) uint8_t smem_raw[];
@@ -285,6 +333,8 @@ __global__ void __launch_bounds__(MWARPS * 32) attn_mma_kernel(const AttnParams 
 
   const int s = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int qg = warp & 3, kh = warp >> 2;
+  ATRACE(0);
   const int nctx = p.n_ctx[b];
   const int nloc = p.n_local_dev ? p.n_local_dev[b] : p.n_local;
   const int nq = p.nq_dev ? p.nq_dev[b] : p.nq;
@@ -295,26 +345,29 @@ __global__ void __launch_bounds__(MWARPS * 32) attn_mma_kernel(const AttnParams 
   const int t1 = min(ntiles, t0 + tps);
   const bf16* pool = static_cast<const bf16*>(p.pool) + static_cast<size_t>(p.layer) * p.pool_layer_stride;
 
-  // stage one 64-key tile of every plane into pipeline stage `st` (16-byte cp.async;
-  // keys past the end are zero-filled)
+  // staging: thread copies 16-byte chunk (tid & 15) of key row (tid >> 4) + 16u of every
+  // plane, u = 0..3 (one 16-key page each); keys past the end are zero-filled
+  const int krow = threadIdx.x >> 4, kch = threadIdx.x & 15;
   auto issue_tile = [&](int t, int st) {
     const uint32_t sbase = smem_u32(stage_base + st * STAGE);
-    for (int idx = threadIdx.x; idx < NP * MKT * 16; idx += blockDim.x) {
-      const int plane = idx / (MKT * 16), rem = idx % (MKT * 16);
-      const int key = rem >> 4, ch = rem & 15;
-      const int kg = t * MKT + key;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int kg = t * MKT + u * 16 + krow;
       const bool valid = kg < total;
       const bf16* src = pool;
       if (valid) {
-        const int page = p.page_table[b * p.max_pages + (kg >> 4)];
-        src = pool + ((static_cast<size_t>(page) * p.H + h) * NP + plane) * 16 * MHD + (kg & 15) * MHD + ch * 8;
+        const int page = p.page_table[b * p.max_pages + t * 4 + u];
+        src = pool + (static_cast<size_t>(page) * p.H + h) * NP * 16 * MHD + krow * MHD + kch * 8;
       }
-      cp_async16(sbase + static_cast<uint32_t>(((plane * MKT + key) * MLDS + ch * 8) * 2), src, valid);
+#pragma unroll
+      for (int plane = 0; plane < NP; ++plane)
+        cp_async16(sbase + static_cast<uint32_t>(((plane * MKT + u * 16 + krow) * MLDS + kch * 8) * 2),
+                   valid ? src + plane * 16 * MHD : src, valid);
     }
     cp_async_commit();
   };
 
-  const int qw = warp * 16;
+  const int qw = qg * 16;
   const bool active = qw < nq;
   const int r0 = qw + (lane >> 2), r1 = r0 + 8;
   const int cq = (lane & 3) * 2;
@@ -342,6 +395,7 @@ __global__ void __launch_bounds__(MWARPS * 32) attn_mma_kernel(const AttnParams 
 #pragma unroll
   for (int i = 0; i < 16; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
   float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.f, 0.f};
+  ATRACE(1);
 
   if (t0 < t1) issue_tile(t0, 0);
   for (int t = t0; t < t1; ++t) {
@@ -352,117 +406,146 @@ __global__ void __launch_bounds__(MWARPS * 32) attn_mma_kernel(const AttnParams 
       cp_async_commit();
     cp_async_wait1();
     __syncthreads();
-    const uint32_t kh_base = smem_u32(stage_base + st * STAGE);
-    const uint32_t kl_base = kh_base + (SPLIT ? MKT * MLDS * 2 : 0);
-    const uint32_t vh_base = kh_base + (SPLIT ? 2 : 1) * MKT * MLDS * 2;
-    const uint32_t vl_base = vh_base + (SPLIT ? MKT * MLDS * 2 : 0);
-    if (!active) {
-      __syncthreads();
-      continue;
-    }
-
-    // S = Q K^T : 16 queries x 64 keys (8 n-tiles of 8 keys); k-steps outer so the
-    // eight accumulators form independent chains
-    float sc[8][4];
+    if (t == t0) ATRACE(2);
+    if (active) {
+      const uint32_t kh_base = smem_u32(stage_base + st * STAGE);
+      const uint32_t kl_base = kh_base + (SPLIT ? MKT * MLDS * 2 : 0);
+      const uint32_t vh_base = kh_base + (SPLIT ? 2 : 1) * MKT * MLDS * 2;
+      const uint32_t vl_base = vh_base + (SPLIT ? MKT * MLDS * 2 : 0);
+      // S = Q K^T on this warp's 32 keys (4 n-tiles of 8)
+      float sc[4][4];
 #pragma unroll
-    for (int nt = 0; nt < 8; ++nt) sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.f;
+      for (int nt = 0; nt < 4; ++nt) sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.f;
 #pragma unroll
-    for (int kp = 0; kp < 4; ++kp) {  // 32 dims per ldmatrix.x4 = two k-steps
+      for (int kp = 0; kp < 4; ++kp) {  // 32 dims per ldmatrix.x4 = two k-steps
 #pragma unroll
-      for (int nt = 0; nt < 8; ++nt) {
-        // ldmatrix rows: key nt*8 + (lane & 7), dims 8*(lane >> 3) within a 32-dim group
-        const uint32_t roff = static_cast<uint32_t>(((nt * 8 + (lane & 7)) * MLDS + (lane >> 3) * 8) * 2);
-        uint32_t bh0, bh1, bh2, bh3;
-        ldsm_x4(kh_base + roff + kp * 64, bh0, bh1, bh2, bh3);
-        mma16816(sc[nt], qh[2 * kp], bh0, bh1);
-        mma16816(sc[nt], ql[2 * kp], bh0, bh1);
-        mma16816(sc[nt], qh[2 * kp + 1], bh2, bh3);
-        mma16816(sc[nt], ql[2 * kp + 1], bh2, bh3);
-        if (SPLIT) {
-          uint32_t bl0, bl1, bl2, bl3;
-          ldsm_x4(kl_base + roff + kp * 64, bl0, bl1, bl2, bl3);
-          mma16816(sc[nt], qh[2 * kp], bl0, bl1);
-          mma16816(sc[nt], qh[2 * kp + 1], bl2, bl3);
+        for (int nt = 0; nt < 4; ++nt) {
+          const uint32_t roff =
+              static_cast<uint32_t>((((kh * 4 + nt) * 8 + (lane & 7)) * MLDS + (lane >> 3) * 8) * 2);
+          uint32_t bh0, bh1, bh2, bh3;
+          ldsm_x4(kh_base + roff + kp * 64, bh0, bh1, bh2, bh3);
+          mma16816(sc[nt], qh[2 * kp], bh0, bh1);
+          mma16816(sc[nt], ql[2 * kp], bh0, bh1);
+          mma16816(sc[nt], qh[2 * kp + 1], bh2, bh3);
+          mma16816(sc[nt], ql[2 * kp + 1], bh2, bh3);
+          if (SPLIT) {
+            uint32_t bl0, bl1, bl2, bl3;
+            ldsm_x4(kl_base + roff + kp * 64, bl0, bl1, bl2, bl3);
+            mma16816(sc[nt], qh[2 * kp], bl0, bl1);
+            mma16816(sc[nt], qh[2 * kp + 1], bl2, bl3);
+          }
         }
       }
-    }
-    // mask, scale, online softmax (rows r0: elements 0,1; r1: elements 2,3)
-    float tmax[2] = {-INFINITY, -INFINITY};
+      // mask, scale, online softmax (rows r0: elements 0,1; r1: elements 2,3)
+      float tmax[2] = {-INFINITY, -INFINITY};
 #pragma unroll
-    for (int nt = 0; nt < 8; ++nt) {
+      for (int nt = 0; nt < 4; ++nt) {
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int key = t * MKT + nt * 8 + cq + (e & 1);
-        const unsigned long long m = (e < 2) ? m0 : m1;
-        const bool vis = key < nctx || (key < total && ((m >> (key - nctx)) & 1ull));
-        sc[nt][e] = vis ? sc[nt][e] * p.scale : -INFINITY;
-        tmax[e >> 1] = fmaxf(tmax[e >> 1], sc[nt][e]);
+        for (int e = 0; e < 4; ++e) {
+          const int key = t * MKT + (kh * 4 + nt) * 8 + cq + (e & 1);
+          const unsigned long long m = (e < 2) ? m0 : m1;
+          const bool vis = key < nctx || (key < total && ((m >> (key - nctx)) & 1ull));
+          sc[nt][e] = vis ? sc[nt][e] * p.scale : -INFINITY;
+          tmax[e >> 1] = fmaxf(tmax[e >> 1], sc[nt][e]);
+        }
       }
-    }
-    float corr[2];
+      float corr[2];
 #pragma unroll
-    for (int r = 0; r < 2; ++r) {
-      tmax[r] = fmaxf(tmax[r], __shfl_xor_sync(0xffffffffu, tmax[r], 1));
-      tmax[r] = fmaxf(tmax[r], __shfl_xor_sync(0xffffffffu, tmax[r], 2));
-      const float mnew = fmaxf(mrow[r], tmax[r]);
-      corr[r] = (mnew == -INFINITY) ? 1.f : expf(mrow[r] - mnew);
-      mrow[r] = mnew;
-    }
-    float rsum[2] = {0.f, 0.f};
-#pragma unroll
-    for (int nt = 0; nt < 8; ++nt) {
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const float mr = mrow[e >> 1];
-        const float pv = (sc[nt][e] == -INFINITY) ? 0.f : expf(sc[nt][e] - mr);
-        sc[nt][e] = pv;
-        rsum[e >> 1] += pv;
+      for (int r = 0; r < 2; ++r) {
+        tmax[r] = fmaxf(tmax[r], __shfl_xor_sync(0xffffffffu, tmax[r], 1));
+        tmax[r] = fmaxf(tmax[r], __shfl_xor_sync(0xffffffffu, tmax[r], 2));
+        const float mnew = fmaxf(mrow[r], tmax[r]);
+        corr[r] = (mnew == -INFINITY) ? 1.f : expf(mrow[r] - mnew);
+        mrow[r] = mnew;
       }
-    }
+      float rsum[2] = {0.f, 0.f};
 #pragma unroll
-    for (int r = 0; r < 2; ++r) {
-      rsum[r] += __shfl_xor_sync(0xffffffffu, rsum[r], 1);
-      rsum[r] += __shfl_xor_sync(0xffffffffu, rsum[r], 2);
-      lrow[r] = lrow[r] * corr[r] + rsum[r];
-    }
+      for (int nt = 0; nt < 4; ++nt) {
 #pragma unroll
-    for (int dt = 0; dt < 16; ++dt) {
-      o[dt][0] *= corr[0]; o[dt][1] *= corr[0];
-      o[dt][2] *= corr[1]; o[dt][3] *= corr[1];
-    }
-    // O += P V : four k-steps of 16 keys, 16 n-tiles of 8 dims
+        for (int e = 0; e < 4; ++e) {
+          const float pv = (sc[nt][e] == -INFINITY) ? 0.f : expf(sc[nt][e] - mrow[e >> 1]);
+          sc[nt][e] = pv;
+          rsum[e >> 1] += pv;
+        }
+      }
 #pragma unroll
-    for (int kk = 0; kk < 4; ++kk) {
-      uint32_t ph[4], pl[4];
-      split2(sc[2 * kk][0], sc[2 * kk][1], ph[0], pl[0]);
-      split2(sc[2 * kk][2], sc[2 * kk][3], ph[1], pl[1]);
-      split2(sc[2 * kk + 1][0], sc[2 * kk + 1][1], ph[2], pl[2]);
-      split2(sc[2 * kk + 1][2], sc[2 * kk + 1][3], ph[3], pl[3]);
-      // ldmatrix.trans rows: key kk*16 + (lane & 15), dims dt*8 + 8 * (lane >> 4)
-      const uint32_t roff = static_cast<uint32_t>(((kk * 16 + (lane & 15)) * MLDS + (lane >> 4) * 8) * 2);
+      for (int r = 0; r < 2; ++r) {
+        rsum[r] += __shfl_xor_sync(0xffffffffu, rsum[r], 1);
+        rsum[r] += __shfl_xor_sync(0xffffffffu, rsum[r], 2);
+        lrow[r] = lrow[r] * corr[r] + rsum[r];
+      }
 #pragma unroll
-      for (int dp = 0; dp < 8; ++dp) {  // two n-tiles per ldmatrix.x4
-        uint32_t vh0, vh1, vh2, vh3;
-        ldsm_x4_t(vh_base + roff + dp * 32, vh0, vh1, vh2, vh3);
-        mma16816(o[2 * dp], ph, vh0, vh1);
-        mma16816(o[2 * dp], pl, vh0, vh1);
-        mma16816(o[2 * dp + 1], ph, vh2, vh3);
-        mma16816(o[2 * dp + 1], pl, vh2, vh3);
-        if (SPLIT) {
-          uint32_t vl0, vl1, vl2, vl3;
-          ldsm_x4_t(vl_base + roff + dp * 32, vl0, vl1, vl2, vl3);
-          mma16816(o[2 * dp], ph, vl0, vl1);
-          mma16816(o[2 * dp + 1], ph, vl2, vl3);
+      for (int dt = 0; dt < 16; ++dt) {
+        o[dt][0] *= corr[0]; o[dt][1] *= corr[0];
+        o[dt][2] *= corr[1]; o[dt][3] *= corr[1];
+      }
+      // O += P V over this warp's 32 keys: two k-steps of 16 keys, 16 n-tiles of 8 dims
+#pragma unroll
+      for (int kk = 0; kk < 2; ++kk) {
+        uint32_t ph[4], pl[4];
+        split2(sc[2 * kk][0], sc[2 * kk][1], ph[0], pl[0]);
+        split2(sc[2 * kk][2], sc[2 * kk][3], ph[1], pl[1]);
+        split2(sc[2 * kk + 1][0], sc[2 * kk + 1][1], ph[2], pl[2]);
+        split2(sc[2 * kk + 1][2], sc[2 * kk + 1][3], ph[3], pl[3]);
+        // ldmatrix.trans rows: key kh*32 + kk*16 + (lane & 15), dims 8 * (lane >> 4)
+        const uint32_t roff =
+            static_cast<uint32_t>(((kh * 32 + kk * 16 + (lane & 15)) * MLDS + (lane >> 4) * 8) * 2);
+#pragma unroll
+        for (int dp = 0; dp < 8; ++dp) {  // two n-tiles per ldmatrix.x4
+          uint32_t vh0, vh1, vh2, vh3;
+          ldsm_x4_t(vh_base + roff + dp * 32, vh0, vh1, vh2, vh3);
+          mma16816(o[2 * dp], ph, vh0, vh1);
+          mma16816(o[2 * dp], pl, vh0, vh1);
+          mma16816(o[2 * dp + 1], ph, vh2, vh3);
+          mma16816(o[2 * dp + 1], pl, vh2, vh3);
+          if (SPLIT) {
+            uint32_t vl0, vl1, vl2, vl3;
+            ldsm_x4_t(vl_base + roff + dp * 32, vl0, vl1, vl2, vl3);
+            mma16816(o[2 * dp], ph, vl0, vl1);
+            mma16816(o[2 * dp + 1], ph, vl2, vl3);
+          }
         }
       }
     }
     __syncthreads();  // this stage may be refilled by the next iteration's copies
   }
 
+  ATRACE(3);
+  // merge the two key halves: warps 4..7 hand their state to warps 0..3 (same lane,
+  // same query rows and dims)
+  float* xch = reinterpret_cast<float*>(smem_raw);  // [4 groups][32 lanes][68]
+  if (kh == 1 && active) {
+    float* x = xch + (qg * 32 + lane) * 68;
+#pragma unroll
+    for (int dt = 0; dt < 16; ++dt)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) x[dt * 4 + e] = o[dt][e];
+    x[64] = mrow[0]; x[65] = mrow[1]; x[66] = lrow[0]; x[67] = lrow[1];
+  }
+  __syncthreads();
+  if (kh == 0 && active) {
+    const float* x = xch + (qg * 32 + lane) * 68;
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      const float mb = x[64 + r], lb = x[66 + r];
+      const float M = fmaxf(mrow[r], mb);
+      const float ca = (M == -INFINITY) ? 0.f : expf(mrow[r] - M);
+      const float cb = (M == -INFINITY) ? 0.f : expf(mb - M);
+      lrow[r] = lrow[r] * ca + lb * cb;
+      mrow[r] = M;
+#pragma unroll
+      for (int dt = 0; dt < 16; ++dt) {
+        o[dt][2 * r] = o[dt][2 * r] * ca + x[dt * 4 + 2 * r] * cb;
+        o[dt][2 * r + 1] = o[dt][2 * r + 1] * ca + x[dt * 4 + 2 * r + 1] * cb;
+      }
+    }
+  }
+  const bool writer = kh == 0 && active;
+
   bf16* out = static_cast<bf16*>(p.out);
   bf16* out_lo = static_cast<bf16*>(p.out_lo);
   if (p.splits == 1) {
-    if (!active) return;
+    if (!writer) return;
 #pragma unroll
     for (int r = 0; r < 2; ++r) {
       const int row = r ? r1 : r0;
@@ -480,7 +563,7 @@ __global__ void __launch_bounds__(MWARPS * 32) attn_mma_kernel(const AttnParams 
 
   const size_t rec = MHD + 4;
   float* wsb = p.ws + (static_cast<size_t>(b * p.H + h) * p.splits) * p.nq_max * rec;
-  if (active) {
+  if (writer) {
 #pragma unroll
     for (int r = 0; r < 2; ++r) {
       const int row = r ? r1 : r0;
@@ -504,10 +587,12 @@ __global__ void __launch_bounds__(MWARPS * 32) attn_mma_kernel(const AttnParams 
     s_last = (old == p.splits - 1) ? 1 : 0;
   }
   __syncthreads();
+  ATRACE(4);
   if (!s_last) return;
   __threadfence();
   combine_splits(p, wsb, nq, MHD, b, h, out, out_lo, reinterpret_cast<float*>(smem_raw));
   if (threadIdx.x == 0) p.counters[b * p.H + h] = 0;
+  ATRACE(5);
 }
 
 template <bool SPLIT>
@@ -519,7 +604,7 @@ cudaError_t launch_mma(const AttnParams& p, cudaStream_t s) {
     attr = true;
   }
   dim3 grid(p.splits, p.H, p.B);
-  attn_mma_kernel<SPLIT><<<grid, MWARPS * 32, smem, s>>>(p);
+  launch_pdl(attn_mma_kernel<SPLIT>, dim3(grid), dim3(MWARPS * 32), smem, s, p);
   return cudaGetLastError();
 }
 
@@ -532,11 +617,17 @@ cudaError_t launch(const AttnParams& p, cudaStream_t s) {
     attr = true;
   }
   dim3 grid(p.splits, p.H, p.B);
-  attn_kernel<TKV, T, HD><<<grid, WARPS * 32, smem, s>>>(p);
+  launch_pdl(attn_kernel<TKV, T, HD>, dim3(grid), dim3(WARPS * 32), smem, s, p);
   return cudaGetLastError();
 }
 
 }  // namespace
+
+#ifdef CHIMERA_ATTN_TRACE
+extern "C" int chimera_attn_trace(unsigned long long* host, int n) {
+  return cudaMemcpyFromSymbol(host, g_attn_trace, static_cast<size_t>(n) * 8 * 8) == cudaSuccess ? 0 : -1;
+}
+#endif
 
 size_t attn_ws_floats(int B, int H, int splits, int nq_max, int hd) {
   return static_cast<size_t>(B) * H * splits * nq_max * (hd + 4);

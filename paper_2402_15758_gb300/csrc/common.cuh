@@ -46,6 +46,12 @@ __device__ __forceinline__ void store_act(bf16* hi, bf16* lo, size_t i, float x)
   if (lo) lo[i] = __float2bfloat16_rn(x - __bfloat162float(h));
 }
 
+// Programmatic dependent launch: let the next kernel in the stream start launching, and
+// wait until the previous kernel has completed with its memory visible (both are no-ops
+// when the launch has no programmatic dependency).
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 __device__ __forceinline__ uint64_t global_timer_ns() {
   uint64_t t;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));

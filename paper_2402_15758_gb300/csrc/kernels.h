@@ -12,10 +12,12 @@ namespace chimera {
 // ----------------------------------------------------------------------------
 struct TcLinearParams {
   CUtensorMap tmA;   // W: [N][K] bf16, box 128 x 64, 128-byte swizzle
+  CUtensorMap tmA2;  // optional second weight W2 [N2][K]: output columns N .. N+N2-1
   CUtensorMap tmB;   // X: [M][K] bf16 (row pitch ldx), box BN x 64, 128-byte swizzle
   CUtensorMap tmB2;  // X_lo (same shape) when the activation is a hi + lo split
   int has_lo;        // 1: two MMAs per K slice, W.X_hi + W.X_lo into one accumulator
-  int M, N, K;
+  int ft_split;      // feature tiles taken from W (the rest from W2); = feat_tiles without W2
+  int M, N, K;       // N = total output columns (N of W plus N2 of W2)
   int BN;            // token tile = UMMA N (multiple of 16, <= 256)
   int tok_tiles, feat_tiles, kblocks;
   long long units;   // feat_tiles * tok_tiles * kblocks
@@ -30,6 +32,7 @@ struct TcLinearParams {
   int* err;          // device error word
   uint32_t tmem_cols;
   uint32_t acc_stride;  // TMEM column distance between the two accumulators
+  int trace_id;         // call-site id (used by instrumented builds only)
 };
 
 struct TcLinearPlan {
@@ -47,9 +50,11 @@ int tc_max_tiles();
 // Encode the plan for one call site.  X/W/Y are device pointers; ws/counters are
 // scratch owned by the caller (sizes from tc_ws_floats / tc_max_tiles).
 // Returns 0 on success, otherwise a negative code and a message in `msg`.
+// W2 (optional, N2 rows): a second weight matrix whose outputs follow W's in Y (one
+// launch for two projections of the same input, e.g. SwiGLU gate and up); needs N % 128 == 0.
 int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, const void* X_lo, int ldx,
                    const void* W, void* Y, void* Y_lo, int ldy, int epi, int out_f32, float* ws,
-                   int* counters, int* err, char* msg, size_t msg_len);
+                   int* counters, int* err, char* msg, size_t msg_len, const void* W2 = nullptr, int N2 = 0);
 cudaError_t tc_linear_launch(const TcLinearPlan& plan, cudaStream_t s);
 
 // ----------------------------------------------------------------------------

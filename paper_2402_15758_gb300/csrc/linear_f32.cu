@@ -2,6 +2,7 @@
 // One warp per output feature streams that weight row once (coalesced) against up to
 // MT token rows; fp32 FMA in a fixed order, then a butterfly sum over the warp.
 #include "common.cuh"
+#include "launch.cuh"
 #include "kernels.h"
 
 namespace chimera {
@@ -14,6 +15,8 @@ __global__ void __launch_bounds__(WARPS * 32) f32_linear_kernel(const float* __r
                                                              const float* __restrict__ W,
                                                              float* __restrict__ Y, int ldy, int M,
                                                              int N, int K, int epi) {
+  pdl_trigger();  // the next kernel may start its prologue
+  pdl_wait();     // inputs of this kernel are complete
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int f = blockIdx.x * WARPS + warp;
   const int m0 = blockIdx.y * MT;
@@ -52,7 +55,7 @@ __global__ void __launch_bounds__(WARPS * 32) f32_linear_kernel(const float* __r
 cudaError_t f32_linear(int M, int N, int K, const float* X, int ldx, const float* W, float* Y,
                        int ldy, int epi, cudaStream_t s) {
   dim3 grid((N + WARPS - 1) / WARPS, (M + MT - 1) / MT);
-  f32_linear_kernel<<<grid, WARPS * 32, 0, s>>>(X, ldx, W, Y, ldy, M, N, K, epi);
+  launch_pdl(f32_linear_kernel, dim3(grid), dim3(WARPS * 32), 0, s, X, ldx, W, Y, ldy, M, N, K, epi);
   return cudaGetLastError();
 }
 

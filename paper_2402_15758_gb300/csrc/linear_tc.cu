@@ -25,6 +25,7 @@
 #include <mutex>
 
 #include "common.cuh"
+#include "launch.cuh"
 #include "kernels.h"
 
 namespace chimera {
@@ -53,11 +54,17 @@ constexpr int MAX_BN = 256;
 constexpr int MAX_TILES = 8192;
 
 #ifdef CHIMERA_LIN_TRACE
-// Per-CTA timestamps of one launch (instrumented builds only).
+// Per-CTA timestamps of one launch, and per call site (trace_id) the earliest start,
+// latest first data, latest last MMA and latest end over its CTAs (instrumented builds).
 __device__ unsigned long long g_lin_trace[1024][8];
+__device__ unsigned long long g_lin_tl[4096][4];
 #define TRACE(i) g_lin_trace[blockIdx.x][i] = global_timer_ns()
+#define TL_MIN(i) atomicMin(&g_lin_tl[p.trace_id & 4095][i], global_timer_ns())
+#define TL_MAX(i) atomicMax(&g_lin_tl[p.trace_id & 4095][i], global_timer_ns())
 #else
 #define TRACE(i)
+#define TL_MIN(i)
+#define TL_MAX(i)
 #endif
 
 // Stream-K partition in 32-bit arithmetic (the host checks units * grid < 2^32).
@@ -144,8 +151,10 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const _
     *s_last = 0;
     mbar_fence_init();
   }
+  pdl_trigger();  // the next kernel may start launching (its CTAs fit once ours exit)
   if (warp == 0 && lane == 0) {
     prefetch_tensormap(&p.tmA);
+    if (p.ft_split < p.feat_tiles) prefetch_tensormap(&p.tmA2);
     prefetch_tensormap(&p.tmB);
     if (p.has_lo) prefetch_tensormap(&p.tmB2);
   }
@@ -154,7 +163,10 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const _
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  if (threadIdx.x == 0) TRACE(0);
+  if (threadIdx.x == 0) {
+    TRACE(0);
+    TL_MIN(0);
+  }
 
   const uint32_t U = static_cast<uint32_t>(p.units);
   const uint32_t G = gridDim.x;
@@ -171,29 +183,49 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const _
       int stage = 0;
       uint32_t phase = 0;
       uint32_t issued_mask = 0, issued_par = 0;
-      for (uint32_t u = u_begin; u < u_end && !*abort;) {
-        const int t = static_cast<int>(u / KB);
-        int kb = static_cast<int>(u % KB);
-        const uint32_t seg_end = min(u_end, static_cast<uint32_t>(t + 1) * KB);
-        const int ft = t / p.tok_tiles, tt = t % p.tok_tiles;
-        for (; u < seg_end; ++u, ++kb) {
-          if (!mbar_wait(&empty[stage], phase ^ 1u, abort)) break;
-          uint8_t* sa = smem + stage * stage_bytes;
-          uint8_t* sb = sa + a_atom * BKA;
-          mbar_arrive_expect_tx(&full[stage], static_cast<uint32_t>(stage_bytes));
-          if (u == u_begin) TRACE(1);
+      auto load_a = [&](uint32_t u, uint8_t* sa, uint64_t* bar) {
+        const int t = static_cast<int>(u / KB), kb = static_cast<int>(u % KB);
+        const int ft = t / p.tok_tiles;
+        const bool second = ft >= p.ft_split;
+        const CUtensorMap* map = second ? &p.tmA2 : &p.tmA;
+        const int row = (second ? ft - p.ft_split : ft) * BM;
 #pragma unroll
-          for (int a = 0; a < BKA; ++a) {
-            tma_load_2d_hint(sa + a * a_atom, &p.tmA, kb * BK + a * ATOM, ft * BM, &full[stage], pol_w);
-            tma_load_2d(sb + a * b_atom, &p.tmB, kb * BK + a * ATOM, tt * p.BN, &full[stage]);
-            if (p.has_lo) tma_load_2d(sb + b_bytes + a * b_atom, &p.tmB2, kb * BK + a * ATOM, tt * p.BN, &full[stage]);
-          }
-          issued_mask |= 1u << stage;
-          issued_par = (issued_par & ~(1u << stage)) | (phase << stage);
-          if (++stage == p.stages) {
-            stage = 0;
-            phase ^= 1u;
-          }
+        for (int a = 0; a < BKA; ++a) tma_load_2d_hint(sa + a * a_atom, map, kb * BK + a * ATOM, row, bar, pol_w);
+      };
+      auto load_b = [&](uint32_t u, uint8_t* sb, uint64_t* bar) {
+        const int t = static_cast<int>(u / KB), kb = static_cast<int>(u % KB);
+        const int tt = t % p.tok_tiles;
+#pragma unroll
+        for (int a = 0; a < BKA; ++a) {
+          tma_load_2d(sb + a * b_atom, &p.tmB, kb * BK + a * ATOM, tt * p.BN, bar);
+          if (p.has_lo) tma_load_2d(sb + b_bytes + a * b_atom, &p.tmB2, kb * BK + a * ATOM, tt * p.BN, bar);
+        }
+      };
+      // The weights do not depend on earlier kernels: request the first stages' weight
+      // tiles before waiting for the previous kernel, then their activation tiles.
+      const uint32_t npre = min(static_cast<uint32_t>(p.stages), u_end - u_begin);
+      for (uint32_t i = 0; i < npre; ++i) {
+        uint8_t* sa = smem + i * stage_bytes;
+        mbar_arrive_expect_tx(&full[i], static_cast<uint32_t>(stage_bytes));
+        if (i == 0) TRACE(1);
+        load_a(u_begin + i, sa, &full[i]);
+        issued_mask |= 1u << i;
+      }
+      pdl_wait();
+      for (uint32_t i = 0; i < npre; ++i) load_b(u_begin + i, smem + i * stage_bytes + a_atom * BKA, &full[i]);
+      stage = static_cast<int>(npre % p.stages);
+      phase = (npre == static_cast<uint32_t>(p.stages)) ? 1u : 0u;
+      for (uint32_t u = u_begin + npre; u < u_end && !*abort; ++u) {
+        if (!mbar_wait(&empty[stage], phase ^ 1u, abort)) break;
+        uint8_t* sa = smem + stage * stage_bytes;
+        mbar_arrive_expect_tx(&full[stage], static_cast<uint32_t>(stage_bytes));
+        load_a(u, sa, &full[stage]);
+        load_b(u, sa + a_atom * BKA, &full[stage]);
+        issued_mask |= 1u << stage;
+        issued_par = (issued_par & ~(1u << stage)) | (phase << stage);
+        if (++stage == p.stages) {
+          stage = 0;
+          phase ^= 1u;
         }
       }
       if (*abort) {
@@ -219,7 +251,10 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const _
         bool first = true;
         for (; u < seg_end; ++u) {
           if (!mbar_wait(&full[stage], phase, abort)) break;
-          if (u == u_begin) TRACE(2);
+          if (u == u_begin) {
+            TRACE(2);
+            TL_MAX(1);
+          }
           tc_fence_after();
           const uint32_t sa = smem_u32(smem + stage * stage_bytes);
           const uint32_t sb = sa + a_atom * BKA;
@@ -242,6 +277,7 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const _
         }
         tc_commit(&tfull[buf]);
         TRACE(3);
+        TL_MAX(2);
         buf ^= 1;
         if (buf == 0) aphase ^= 1u;
       }
@@ -253,6 +289,7 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const _
     }
   } else {
     // ---------------- epilogue (warps 2..5, TMEM lanes 32*(warp%4) ..) ----------------
+    pdl_wait();  // Y, the split workspace and the counters are shared with earlier kernels
     const int q = warp & 3;
     const int row = q * 32 + lane;
     int buf = 0;
@@ -350,7 +387,10 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const _
     tmem_dealloc(tmem_base, p.tmem_cols);
   }
   if (threadIdx.x == 0 && *abort) atomicOr(p.err, ERR_TIMEOUT);
-  if (threadIdx.x == 0) TRACE(7);
+  if (threadIdx.x == 0) {
+    TRACE(7);
+    TL_MAX(3);
+  }
 }
 
 // ----------------------------------------------------------------------------
@@ -411,6 +451,20 @@ size_t tc_ws_floats(int max_bn) {
 int tc_max_tiles() { return MAX_TILES; }
 
 #ifdef CHIMERA_LIN_TRACE
+extern "C" int chimera_lin_timeline(unsigned long long* host, int n, int reset) {
+  if (reset) {
+    static unsigned long long init[4096][4];
+    for (int i = 0; i < 4096; ++i) {
+      init[i][0] = ~0ull;
+      init[i][1] = init[i][2] = init[i][3] = 0;
+    }
+    return cudaMemcpyToSymbol(g_lin_tl, init, sizeof(init)) == cudaSuccess ? 0 : -1;
+  }
+  return cudaMemcpyFromSymbol(host, g_lin_tl, static_cast<size_t>(n) * 4 * sizeof(unsigned long long)) ==
+                 cudaSuccess
+             ? 0
+             : -1;
+}
 extern "C" int chimera_lin_trace(unsigned long long* host, int ctas) {
   return cudaMemcpyFromSymbol(host, g_lin_trace, static_cast<size_t>(ctas) * 8 * sizeof(unsigned long long)) ==
                  cudaSuccess
@@ -421,7 +475,7 @@ extern "C" int chimera_lin_trace(unsigned long long* host, int ctas) {
 
 int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, const void* X_lo, int ldx,
                    const void* W, void* Y, void* Y_lo, int ldy, int epi, int out_f32, float* ws,
-                   int* counters, int* err, char* msg, size_t msg_len) {
+                   int* counters, int* err, char* msg, size_t msg_len, const void* W2, int N2) {
   auto fail = [&](const char* m) {
     if (msg && msg_len) snprintf(msg, msg_len, "linear(M=%d,N=%d,K=%d): %s", M, N, K, m);
     return -1;
@@ -433,6 +487,11 @@ int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, const
       (reinterpret_cast<uintptr_t>(X_lo) & 15))
     return fail("X, X_lo and W must be 16-byte aligned");
   if (epi == EPI_RESID && !out_f32) return fail("accumulating epilogue needs an fp32 output");
+  if (W2 && (N % BM != 0 || N2 < 1 || (reinterpret_cast<uintptr_t>(W2) & 15)))
+    return fail("second weight needs N % 128 == 0 and a 16-byte aligned W2");
+  const int N1 = N;
+  if (W2) N += N2;
+  if (ldy < N) return fail("row pitch of Y smaller than the two outputs");
   TcLinearParams& p = plan->p;
   memset(&p, 0, sizeof(p));
   p.M = M;
@@ -441,6 +500,7 @@ int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, const
   p.BN = M <= MAX_BN ? ((M + 15) / 16) * 16 : MAX_BN;
   p.tok_tiles = (M + p.BN - 1) / p.BN;
   p.feat_tiles = (N + BM - 1) / BM;
+  p.ft_split = W2 ? N1 / BM : p.feat_tiles;
   p.kblocks = (K + BK - 1) / BK;
   if (static_cast<long long>(p.feat_tiles) * p.tok_tiles > MAX_TILES) return fail("too many tiles");
   p.units = static_cast<long long>(p.feat_tiles) * p.tok_tiles * p.kblocks;
@@ -462,7 +522,8 @@ int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, const
   p.tmem_cols = pow2ceil(2 * p.acc_stride);
   if (p.tmem_cols < 32) p.tmem_cols = 32;
   if (p.tmem_cols > 512) return fail("accumulators exceed tensor memory");
-  if (encode_2d_bf16(&p.tmA, W, K, N, K, ATOM, BM) != 0) return fail("tensor map of W");
+  if (encode_2d_bf16(&p.tmA, W, K, N1, K, ATOM, BM) != 0) return fail("tensor map of W");
+  if (W2 && encode_2d_bf16(&p.tmA2, W2, K, N2, K, ATOM, BM) != 0) return fail("tensor map of W2");
   if (encode_2d_bf16(&p.tmB, X, K, M, ldx, ATOM, p.BN) != 0) return fail("tensor map of X");
   if (X_lo && encode_2d_bf16(&p.tmB2, X_lo, K, M, ldx, ATOM, p.BN) != 0) return fail("tensor map of X_lo");
   const int sms = tc_num_sms() * CTAS_PER_SM;
@@ -477,7 +538,7 @@ cudaError_t tc_linear_launch(const TcLinearPlan& plan, cudaStream_t s) {
   std::call_once(once, [] {
     cudaFuncSetAttribute(tc_linear_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
   });
-  tc_linear_kernel<<<plan.grid, THREADS, plan.smem, s>>>(plan.p);
+  launch_pdl(tc_linear_kernel, dim3(plan.grid), dim3(THREADS), plan.smem, s, plan.p);
   return cudaGetLastError();
 }
 

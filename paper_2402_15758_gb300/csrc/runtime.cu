@@ -29,6 +29,8 @@ struct Lin {
   int M = 0, N = 0, K = 0, ldx = 0, ldy = 0, epi = 0, out_f32 = 0;
   const void* X = nullptr;
   const void* W = nullptr;
+  const void* W2 = nullptr;  // optional second weight: outputs at columns N .. N+N2-1
+  int N2 = 0;
   void* Y = nullptr;
   double bytes = 0;
 };
@@ -230,6 +232,7 @@ struct chimera_ctx {
 
   std::string err;
   std::vector<void*> allocs;
+  int lin_sites = 0;  // call-site ids of the linear plans (instrumented builds)
 };
 
 namespace {
@@ -289,14 +292,19 @@ struct Scope {
 };
 
 cudaError_t run_lin(chimera_ctx* ctx, const Lin& l) {
+  if (l.N == 0) return cudaSuccess;  // folded into the previous call site
   Scope sc(ctx, CHIMERA_KIND_LINEAR, l.bytes);
   if (l.tc) return tc_linear_launch(l.tp, ctx->stream);
-  return f32_linear(l.M, l.N, l.K, static_cast<const float*>(l.X), l.ldx, static_cast<const float*>(l.W),
-                    static_cast<float*>(l.Y), l.ldy, l.epi, ctx->stream);
+  cudaError_t e = f32_linear(l.M, l.N, l.K, static_cast<const float*>(l.X), l.ldx, static_cast<const float*>(l.W),
+                             static_cast<float*>(l.Y), l.ldy, l.epi, ctx->stream);
+  if (e != cudaSuccess || !l.W2) return e;
+  return f32_linear(l.M, l.N2, l.K, static_cast<const float*>(l.X), l.ldx, static_cast<const float*>(l.W2),
+                    static_cast<float*>(l.Y) + l.N, l.ldy, l.epi, ctx->stream);
 }
 
 bool make_lin(chimera_ctx* ctx, Lin* l, int M, int N, int K, const void* X, const void* X_lo, int ldx,
-              const void* W, void* Y, void* Y_lo, int ldy, int epi, int out_f32) {
+              const void* W, void* Y, void* Y_lo, int ldy, int epi, int out_f32, const void* W2 = nullptr,
+              int N2 = 0) {
   l->M = M;
   l->N = N;
   l->K = K;
@@ -307,15 +315,18 @@ bool make_lin(chimera_ctx* ctx, Lin* l, int M, int N, int K, const void* X, cons
   l->ldy = ldy;
   l->epi = epi;
   l->out_f32 = out_f32;
-  l->bytes = static_cast<double>(N) * K * ctx->esz;
+  l->W2 = W2;
+  l->N2 = W2 ? N2 : 0;
+  l->bytes = static_cast<double>(N + l->N2) * K * ctx->esz;
   l->tc = ctx->dtype == 1;
   if (!l->tc) return true;
   char msg[256];
   if (tc_linear_plan(&l->tp, M, N, K, X, X_lo, ldx, W, Y, Y_lo, ldy, epi, out_f32, ctx->lin_ws, ctx->lin_cnt,
-                     ctx->d_err, msg, sizeof(msg)) != 0) {
+                     ctx->d_err, msg, sizeof(msg), W2, N2) != 0) {
     ctx->err = msg;
     return false;
   }
+  l->tp.p.trace_id = ctx->lin_sites++;
   return true;
 }
 
@@ -565,8 +576,10 @@ bool build_plans(chimera_ctx* ctx, int B) {
       Lin* p = &v[5 * l];
       if (!make_lin(ctx, &p[0], M, 3 * d, d, xn, xl, d, w.wqkv, ctx->qkv, nullptr, 3 * d, ACC, f32)) return false;
       if (!make_lin(ctx, &p[1], M, d, d, ao, al, d, w.wo, ctx->x, nullptr, d, ACC, f32)) return false;
-      if (!make_lin(ctx, &p[2], M, F, d, xn, xl, d, w.w_gate, ctx->gu, nullptr, 2 * F, ACC, f32)) return false;
-      if (!make_lin(ctx, &p[3], M, F, d, xn, xl, d, w.w_up, ctx->gu + F, nullptr, 2 * F, ACC, f32)) return false;
+      // gate and up: one launch writing gu[:, 0:F] and gu[:, F:2F]
+      if (!make_lin(ctx, &p[2], M, F, d, xn, xl, d, w.w_gate, ctx->gu, nullptr, 2 * F, ACC, f32, w.w_up, F))
+        return false;
+      p[3] = Lin();  // N = 0: nothing to launch
       if (!make_lin(ctx, &p[4], M, d, F, hf, hl, F, w.w_down, ctx->x, nullptr, d, ACC, f32)) return false;
     }
     return true;
@@ -594,8 +607,9 @@ bool build_plans(chimera_ctx* ctx, int B) {
   const chimera_block_weights& w = ctx->draft;
   if (!make_lin(ctx, &ctx->dqkv, B, 3 * d, d, xn, xl, d, w.wqkv, ctx->qkv, nullptr, 3 * d, ACC, f32)) return false;
   if (!make_lin(ctx, &ctx->dwo, B, d, d, ao, al, d, w.wo, ctx->dres, nullptr, d, ACC, f32)) return false;
-  if (!make_lin(ctx, &ctx->dgate, B, F, d, xn, xl, d, w.w_gate, ctx->gu, nullptr, 2 * F, ACC, f32)) return false;
-  if (!make_lin(ctx, &ctx->dup, B, F, d, xn, xl, d, w.w_up, ctx->gu + F, nullptr, 2 * F, ACC, f32)) return false;
+  if (!make_lin(ctx, &ctx->dgate, B, F, d, xn, xl, d, w.w_gate, ctx->gu, nullptr, 2 * F, ACC, f32, w.w_up, F))
+    return false;
+  ctx->dup = Lin();
   if (!make_lin(ctx, &ctx->ddown, B, d, F, hf, hl, F, w.w_down, ctx->dres, nullptr, d, ACC, f32)) return false;
   ctx->dhead.assign(ctx->K, Lin());
   for (int k = 0; k < ctx->K; ++k)
@@ -755,7 +769,7 @@ chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
       c.max_batch > 64 || c.kv_block != 16 || c.max_seq_len < 32 || !(c.rms_eps > 0) || !(c.rope_theta > 0) ||
       (c.precision != 0 && c.precision != 1))
     return CHIMERA_EINVAL;
-  if (c.dtype == 1 && (c.d_model % 64 != 0 || c.ffn_dim % 8 != 0)) return CHIMERA_EINVAL;
+  if (c.dtype == 1 && (c.d_model % 64 != 0 || c.ffn_dim % 128 != 0)) return CHIMERA_EINVAL;
   // row kernels read 16-byte vectors; the top-k covers at most 64 slices of 2048 scores
   if ((c.d_model & 3) || (c.ffn_dim & 3) || (c.vocab & 3) || c.vocab > TOPK_MAX_BLOCKS * 2048) return CHIMERA_EINVAL;
   for (int k = 0; k < c.n_draft_heads; ++k)
@@ -981,6 +995,7 @@ chimera_status chimera_prefill(chimera_ctx* ctx, int batch, const int32_t* token
   }
   ctx->batch = batch;
   ctx->plan_keys = max_len;
+  ctx->lin_sites = 0;
   if (!build_plans(ctx, batch)) return CHIMERA_EINVAL;
   for (int b = 0; b < batch; ++b) {
     chimera_status st = ensure_blocks(ctx, b, lens[b] + need);

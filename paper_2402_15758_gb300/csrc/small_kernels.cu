@@ -3,6 +3,7 @@
 #include <cmath>
 
 #include "common.cuh"
+#include "launch.cuh"
 #include "kernels.h"
 
 namespace chimera {
@@ -62,6 +63,8 @@ __global__ void __launch_bounds__(NORM_THREADS) rmsnorm_kernel(const float* __re
                                                                T* __restrict__ Y_lo, float* __restrict__ Y32,
                                                                int ldy, int d, float eps, float* __restrict__ Z,
                                                                int ldz, int zcols) {
+  pdl_trigger();  // the next kernel may start its prologue
+  pdl_wait();     // inputs of this kernel are complete
   __shared__ float red[33];
   const float* x = X + static_cast<size_t>(blockIdx.x) * ldx;
   float4 v[NORM_VEC];
@@ -136,6 +139,8 @@ __device__ __forceinline__ float4 rot_hi(float4 x1, float4 x2, float4 c, float4 
 
 template <typename T>
 __global__ void rope_kv_kernel(const RopeKvParams p) {
+  pdl_trigger();  // the next kernel may start its prologue
+  pdl_wait();     // inputs of this kernel are complete
   const int row = blockIdx.x;
   const int b = row / p.rows_per_seq, i = row % p.rows_per_seq;
   const int n = p.n[b];
@@ -207,6 +212,8 @@ __global__ void rope_kv_kernel(const RopeKvParams p) {
 template <typename T>
 __global__ void swiglu_kernel(const float* __restrict__ gu, int ldgu, int F, T* __restrict__ h,
                               T* __restrict__ h_lo, int ldh) {
+  pdl_trigger();  // the next kernel may start its prologue
+  pdl_wait();     // inputs of this kernel are complete
   const float* g = gu + static_cast<size_t>(blockIdx.y) * ldgu;
   const size_t row = static_cast<size_t>(blockIdx.y) * ldh;
   const int f = (blockIdx.x * blockDim.x + threadIdx.x) * 4;
@@ -220,6 +227,8 @@ template <typename T>
 __global__ void embed_kernel(const T* __restrict__ E, int d, int V, float* __restrict__ x,
                              int rows_per_seq, const int* tokens, const int* tok_hist,
                              int hist_stride, const int* n, const int* valid, int* err) {
+  pdl_trigger();  // the next kernel may start its prologue
+  pdl_wait();     // inputs of this kernel are complete
   const int r = blockIdx.x;
   int tok;
   if (tokens) {
@@ -243,6 +252,8 @@ __device__ __forceinline__ bool better(float v, int i, float bv, int bi) {
 }
 
 __global__ void __launch_bounds__(512) argmax_kernel(const float* __restrict__ logits, int V, int* __restrict__ out) {
+  pdl_trigger();  // the next kernel may start its prologue
+  pdl_wait();     // inputs of this kernel are complete
   __shared__ float sv[32];
   __shared__ int si[32];
   const float* z = logits + static_cast<size_t>(blockIdx.x) * V;
@@ -385,6 +396,8 @@ __global__ void __launch_bounds__(TOPK_THREADS) topk_kernel(const float* __restr
                                                             int* __restrict__ idx, float* __restrict__ val,
                                                             int out_stride, float* __restrict__ ws_v,
                                                             int* __restrict__ ws_i, int* __restrict__ counters) {
+  pdl_trigger();  // the next kernel may start its prologue
+  pdl_wait();     // inputs of this kernel are complete
   __shared__ float s_bv[TOPK_MAX];
   __shared__ int s_bi[TOPK_MAX];
   __shared__ int s_last;
@@ -457,10 +470,10 @@ cudaError_t rmsnorm(int dtype, const float* X, int ldx, const void* g, void* Y, 
   if (Z && ((zcols & 3) || (ldz & 3) || (reinterpret_cast<uintptr_t>(Z) & 15))) return cudaErrorInvalidValue;
   if ((d & 3) || (ldx & 3) || (ldy & 3) || d > NORM_THREADS * NORM_VEC * 4) return cudaErrorInvalidValue;
   if (dtype == 0)
-    rmsnorm_kernel<float><<<rows, NORM_THREADS, 0, s>>>(X, ldx, static_cast<const float*>(g), static_cast<float*>(Y),
+    launch_pdl(rmsnorm_kernel<float>, dim3(rows), dim3(NORM_THREADS), 0, s, X, ldx, static_cast<const float*>(g), static_cast<float*>(Y),
                                                nullptr, Y32, ldy, d, eps, Z, ldz, zcols);
   else
-    rmsnorm_kernel<bf16><<<rows, NORM_THREADS, 0, s>>>(X, ldx, static_cast<const bf16*>(g), static_cast<bf16*>(Y),
+    launch_pdl(rmsnorm_kernel<bf16>, dim3(rows), dim3(NORM_THREADS), 0, s, X, ldx, static_cast<const bf16*>(g), static_cast<bf16*>(Y),
                                               static_cast<bf16*>(Y_lo), Y32, ldy, d, eps, Z, ldz, zcols);
   return cudaGetLastError();
 }
@@ -473,9 +486,9 @@ cudaError_t rope_kv(const RopeKvParams& p, int dtype, cudaStream_t s) {
     return cudaErrorInvalidValue;
   if (p.planes != 2 && !(p.planes == 4 && dtype == 1)) return cudaErrorInvalidValue;
   if (dtype == 0)
-    rope_kv_kernel<float><<<rows, 256, 0, s>>>(p);
+    launch_pdl(rope_kv_kernel<float>, dim3(rows), dim3(256), 0, s, p);
   else
-    rope_kv_kernel<bf16><<<rows, 256, 0, s>>>(p);
+    launch_pdl(rope_kv_kernel<bf16>, dim3(rows), dim3(256), 0, s, p);
   return cudaGetLastError();
 }
 
@@ -485,9 +498,9 @@ cudaError_t swiglu(int dtype, const float* gu, int ldgu, int F, void* h, void* h
   if ((F & 3) || (ldh & 3)) return cudaErrorInvalidValue;
   dim3 grid((F / 4 + 255) / 256, rows);
   if (dtype == 0)
-    swiglu_kernel<float><<<grid, 256, 0, s>>>(gu, ldgu, F, static_cast<float*>(h), nullptr, ldh);
+    launch_pdl(swiglu_kernel<float>, dim3(grid), dim3(256), 0, s, gu, ldgu, F, static_cast<float*>(h), nullptr, ldh);
   else
-    swiglu_kernel<bf16><<<grid, 256, 0, s>>>(gu, ldgu, F, static_cast<bf16*>(h), static_cast<bf16*>(h_lo), ldh);
+    launch_pdl(swiglu_kernel<bf16>, dim3(grid), dim3(256), 0, s, gu, ldgu, F, static_cast<bf16*>(h), static_cast<bf16*>(h_lo), ldh);
   return cudaGetLastError();
 }
 
@@ -496,10 +509,10 @@ cudaError_t embed(int dtype, const void* E, int d, int V, float* x, int rows, in
                   const int* valid, int* err, cudaStream_t s) {
   if (rows <= 0) return cudaSuccess;
   if (dtype == 0)
-    embed_kernel<float><<<rows, 256, 0, s>>>(static_cast<const float*>(E), d, V, x, rows_per_seq,
+    launch_pdl(embed_kernel<float>, dim3(rows), dim3(256), 0, s, static_cast<const float*>(E), d, V, x, rows_per_seq,
                                              tokens, tok_hist, hist_stride, n, valid, err);
   else
-    embed_kernel<bf16><<<rows, 256, 0, s>>>(static_cast<const bf16*>(E), d, V, x, rows_per_seq,
+    launch_pdl(embed_kernel<bf16>, dim3(rows), dim3(256), 0, s, static_cast<const bf16*>(E), d, V, x, rows_per_seq,
                                             tokens, tok_hist, hist_stride, n, valid, err);
   return cudaGetLastError();
 }
@@ -507,7 +520,7 @@ cudaError_t embed(int dtype, const void* E, int d, int V, float* x, int rows, in
 cudaError_t argmax_rows(const float* logits, int V, int rows, int* out, cudaStream_t s) {
   if (rows <= 0) return cudaSuccess;
   if (V & 3) return cudaErrorInvalidValue;  // rows are read as float4
-  argmax_kernel<<<rows, 512, 0, s>>>(logits, V, out);
+  launch_pdl(argmax_kernel, dim3(rows), dim3(512), 0, s, logits, V, out);
   return cudaGetLastError();
 }
 
@@ -518,7 +531,7 @@ cudaError_t topk_rows(const float* logits, int V, int rows, int k, int* idx, flo
   const int nblk = (V + TOPK_SLICE - 1) / TOPK_SLICE;
   if (nblk > TOPK_MAX_BLOCKS) return cudaErrorInvalidValue;
   dim3 grid(nblk, rows);
-  topk_kernel<<<grid, TOPK_THREADS, 0, s>>>(logits, V, k, idx, val, out_stride, ws_v, ws_i, counters);
+  launch_pdl(topk_kernel, dim3(grid), dim3(TOPK_THREADS), 0, s, logits, V, k, idx, val, out_stride, ws_v, ws_i, counters);
   return cudaGetLastError();
 }
 

@@ -1,6 +1,7 @@
 // Small kernels that stitch the step together: trigram gather, tree expansion,
 // greedy acceptance, KV compaction, hidden-state gathers and state update.
 #include "common.cuh"
+#include "launch.cuh"
 #include "step_kernels.h"
 
 namespace chimera {
@@ -14,6 +15,8 @@ template <typename T>
 __global__ void trigram_gather_kernel(const T* __restrict__ E, int d, int V, const int* n_arr,
                                       const int* tok, int tok_stride, const int* topk, int K,
                                       int KMAX, int k, T* __restrict__ out, int* err, float* __restrict__ zero) {
+  pdl_trigger();  // the next kernel may start its prologue
+  pdl_wait();     // inputs of this kernel are complete
   const int b = blockIdx.x;
   const int n = n_arr[b];
   for (int c = threadIdx.x * 4; c < d; c += blockDim.x * 4)
@@ -42,6 +45,8 @@ template <typename T>
 __global__ void hfull_store_kernel(const float* __restrict__ dres, int d, T* __restrict__ headin,
                                    T* __restrict__ headin_lo, float* __restrict__ hlog,
                                    float* __restrict__ zero, int V) {
+  pdl_trigger();  // the next kernel may start its prologue
+  pdl_wait();     // inputs of this kernel are complete
   const int b = blockIdx.x;
   for (int c = threadIdx.x * 4; c < V; c += blockDim.x * 4)
     *reinterpret_cast<float4*>(zero + static_cast<size_t>(b) * V + c) = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -61,6 +66,8 @@ __global__ void hfull_store_kernel(const float* __restrict__ dres, int d, T* __r
 __global__ void tree_expand_kernel(const int* n_arr, const int* tok, int tok_stride, const int* topk,
                                    int K, int KMAX, const int* depth, const int* rank, int N,
                                    const int* ovr_flag, const int* ovr, int* node_tok) {
+  pdl_trigger();  // the next kernel may start its prologue
+  pdl_wait();     // inputs of this kernel are complete
   const int b = blockIdx.x, i = threadIdx.x;
   if (i >= N) return;
   int t;
@@ -80,6 +87,8 @@ __global__ void tree_expand_kernel(const int* n_arr, const int* tok, int tok_str
 __global__ void accept_kernel(const int* n_arr, int* tok, int tok_stride, const int* node_tok,
                               const int* amax, const int* child_start, const int* child, int N,
                               int D1, int* path, int* Lacc, int* bonus) {
+  pdl_trigger();  // the next kernel may start its prologue
+  pdl_wait();     // inputs of this kernel are complete
   const int b = blockIdx.x;
   if (threadIdx.x != 0) return;
   const int n = n_arr[b];
@@ -110,6 +119,8 @@ __global__ void accept_kernel(const int* n_arr, int* tok, int tok_stride, const 
 __global__ void compact_kernel(char* pool, long long layer_stride_bytes, int H, int planes, int row_bytes,
                                const int* n_arr, const int* path, const int* Lacc, int D1,
                                const int* page_table, int max_pages) {
+  pdl_trigger();  // the next kernel may start its prologue
+  pdl_wait();     // inputs of this kernel are complete
   const int b = blockIdx.y;
   const int L = Lacc[b];
   if (L == 0) return;
@@ -139,6 +150,8 @@ template <typename T>
 __global__ void gather_hidden_kernel(const float* __restrict__ hfin, int d, int N, const int* path,
                                      const int* Lacc, int D1, float* __restrict__ hsel,
                                      T* __restrict__ headin, T* __restrict__ headin_lo) {
+  pdl_trigger();  // the next kernel may start its prologue
+  pdl_wait();     // inputs of this kernel are complete
   const int b = blockIdx.x, j = blockIdx.y;
   const int L = Lacc[b];
   const int node = path[b * D1 + (j <= L ? j : L)];
@@ -154,6 +167,8 @@ __global__ void gather_hidden_kernel(const float* __restrict__ hfin, int d, int 
 // Commit: x[n+L+1] = bonus (the next root), n += L + 1, per-step count log.
 __global__ void finalize_kernel(int* n_arr, int* tok, int tok_stride, const int* Lacc,
                                 const int* bonus, int* count_log, int log_cap, int* step, int B) {
+  pdl_trigger();  // the next kernel may start its prologue
+  pdl_wait();     // inputs of this kernel are complete
   const int b = threadIdx.x;
   const int s = *step;
   __syncthreads();
@@ -173,6 +188,8 @@ template <typename T>
 __global__ void prefill_advance_kernel(const float* __restrict__ hfin, int d, int rows_per_seq,
                                        const int* valid, const int* last, int* n_arr,
                                        T* __restrict__ headin, T* __restrict__ headin_lo) {
+  pdl_trigger();  // the next kernel may start its prologue
+  pdl_wait();     // inputs of this kernel are complete
   const int b = blockIdx.x;
   const int li = last[b];
   if (li >= 0) {
@@ -184,6 +201,8 @@ __global__ void prefill_advance_kernel(const float* __restrict__ hfin, int d, in
 }
 
 __global__ void set_root_kernel(const int* n_arr, int* tok, int tok_stride, const int* amax, int B) {
+  pdl_trigger();  // the next kernel may start its prologue
+  pdl_wait();     // inputs of this kernel are complete
   const int b = threadIdx.x;
   if (b < B) tok[static_cast<size_t>(b) * tok_stride + n_arr[b]] = amax[b];
 }
@@ -194,10 +213,10 @@ cudaError_t launch_trigram_gather(int dtype, const void* E, int d, int V, const 
                                   int tok_stride, const int* topk, int K, int KMAX, int k, void* out,
                                   int B, int* err, float* zero, cudaStream_t s) {
   if (dtype == 0)
-    trigram_gather_kernel<float><<<B, 256, 0, s>>>(static_cast<const float*>(E), d, V, n, tok, tok_stride,
+    launch_pdl(trigram_gather_kernel<float>, dim3(B), dim3(256), 0, s, static_cast<const float*>(E), d, V, n, tok, tok_stride,
                                                    topk, K, KMAX, k, static_cast<float*>(out), err, zero);
   else
-    trigram_gather_kernel<bf16><<<B, 256, 0, s>>>(static_cast<const bf16*>(E), d, V, n, tok, tok_stride,
+    launch_pdl(trigram_gather_kernel<bf16>, dim3(B), dim3(256), 0, s, static_cast<const bf16*>(E), d, V, n, tok, tok_stride,
                                                   topk, K, KMAX, k, static_cast<bf16*>(out), err, zero);
   return cudaGetLastError();
 }
@@ -205,9 +224,9 @@ cudaError_t launch_trigram_gather(int dtype, const void* E, int d, int V, const 
 cudaError_t launch_hfull_store(int dtype, const float* dres, int d, void* headin, void* headin_lo, float* hlog,
                                float* zero, int V, int B, cudaStream_t s) {
   if (dtype == 0)
-    hfull_store_kernel<float><<<B, 256, 0, s>>>(dres, d, static_cast<float*>(headin), nullptr, hlog, zero, V);
+    launch_pdl(hfull_store_kernel<float>, dim3(B), dim3(256), 0, s, dres, d, static_cast<float*>(headin), nullptr, hlog, zero, V);
   else
-    hfull_store_kernel<bf16><<<B, 256, 0, s>>>(dres, d, static_cast<bf16*>(headin), static_cast<bf16*>(headin_lo),
+    launch_pdl(hfull_store_kernel<bf16>, dim3(B), dim3(256), 0, s, dres, d, static_cast<bf16*>(headin), static_cast<bf16*>(headin_lo),
                                                hlog, zero, V);
   return cudaGetLastError();
 }
@@ -215,14 +234,14 @@ cudaError_t launch_hfull_store(int dtype, const float* dres, int d, void* headin
 cudaError_t launch_tree_expand(const int* n, const int* tok, int tok_stride, const int* topk, int K, int KMAX,
                                const int* depth, const int* rank, int N, const int* ovr_flag, const int* ovr,
                                int* node_tok, int B, cudaStream_t s) {
-  tree_expand_kernel<<<B, 64, 0, s>>>(n, tok, tok_stride, topk, K, KMAX, depth, rank, N, ovr_flag, ovr, node_tok);
+  launch_pdl(tree_expand_kernel, dim3(B), dim3(64), 0, s, n, tok, tok_stride, topk, K, KMAX, depth, rank, N, ovr_flag, ovr, node_tok);
   return cudaGetLastError();
 }
 
 cudaError_t launch_accept(const int* n, int* tok, int tok_stride, const int* node_tok, const int* amax,
                           const int* child_start, const int* child, int N, int D1, int* path, int* Lacc,
                           int* bonus, int B, cudaStream_t s) {
-  accept_kernel<<<B, 32, 0, s>>>(n, tok, tok_stride, node_tok, amax, child_start, child, N, D1, path, Lacc,
+  launch_pdl(accept_kernel, dim3(B), dim3(32), 0, s, n, tok, tok_stride, node_tok, amax, child_start, child, N, D1, path, Lacc,
                                  bonus);
   return cudaGetLastError();
 }
@@ -233,7 +252,7 @@ cudaError_t launch_compact(void* pool, long long layer_stride_bytes, int n_layer
   const int threads = (row_bytes / 16) * (D1 - 1);
   if (threads <= 0) return cudaSuccess;
   dim3 grid(n_layers * planes * H, B);
-  compact_kernel<<<grid, threads, 0, s>>>(static_cast<char*>(pool), layer_stride_bytes, H, planes, row_bytes, n,
+  launch_pdl(compact_kernel, dim3(grid), dim3(threads), 0, s, static_cast<char*>(pool), layer_stride_bytes, H, planes, row_bytes, n,
                                           path, Lacc, D1, page_table, max_pages);
   return cudaGetLastError();
 }
@@ -242,33 +261,33 @@ cudaError_t launch_gather_hidden(int dtype, const float* hfin, int d, int N, con
                                  int D1, float* hsel, void* headin, void* headin_lo, int B, cudaStream_t s) {
   dim3 grid(B, D1);
   if (dtype == 0)
-    gather_hidden_kernel<float><<<grid, 256, 0, s>>>(hfin, d, N, path, Lacc, D1, hsel, static_cast<float*>(headin),
+    launch_pdl(gather_hidden_kernel<float>, dim3(grid), dim3(256), 0, s, hfin, d, N, path, Lacc, D1, hsel, static_cast<float*>(headin),
                                                      nullptr);
   else
-    gather_hidden_kernel<bf16><<<grid, 256, 0, s>>>(hfin, d, N, path, Lacc, D1, hsel, static_cast<bf16*>(headin),
+    launch_pdl(gather_hidden_kernel<bf16>, dim3(grid), dim3(256), 0, s, hfin, d, N, path, Lacc, D1, hsel, static_cast<bf16*>(headin),
                                                     static_cast<bf16*>(headin_lo));
   return cudaGetLastError();
 }
 
 cudaError_t launch_finalize(int* n, int* tok, int tok_stride, const int* Lacc, const int* bonus, int* count_log,
                             int log_cap, int* step, int B, cudaStream_t s) {
-  finalize_kernel<<<1, ((B + 31) / 32) * 32, 0, s>>>(n, tok, tok_stride, Lacc, bonus, count_log, log_cap, step, B);
+  launch_pdl(finalize_kernel, dim3(1), dim3(((B + 31) / 32) * 32), 0, s, n, tok, tok_stride, Lacc, bonus, count_log, log_cap, step, B);
   return cudaGetLastError();
 }
 
 cudaError_t launch_prefill_advance(int dtype, const float* hfin, int d, int rows_per_seq, const int* valid,
                                    const int* last, int* n, void* headin, void* headin_lo, int B, cudaStream_t s) {
   if (dtype == 0)
-    prefill_advance_kernel<float><<<B, 256, 0, s>>>(hfin, d, rows_per_seq, valid, last, n,
+    launch_pdl(prefill_advance_kernel<float>, dim3(B), dim3(256), 0, s, hfin, d, rows_per_seq, valid, last, n,
                                                     static_cast<float*>(headin), nullptr);
   else
-    prefill_advance_kernel<bf16><<<B, 256, 0, s>>>(hfin, d, rows_per_seq, valid, last, n,
+    launch_pdl(prefill_advance_kernel<bf16>, dim3(B), dim3(256), 0, s, hfin, d, rows_per_seq, valid, last, n,
                                                    static_cast<bf16*>(headin), static_cast<bf16*>(headin_lo));
   return cudaGetLastError();
 }
 
 cudaError_t launch_set_root(const int* n, int* tok, int tok_stride, const int* amax, int B, cudaStream_t s) {
-  set_root_kernel<<<1, ((B + 31) / 32) * 32, 0, s>>>(n, tok, tok_stride, amax, B);
+  launch_pdl(set_root_kernel, dim3(1), dim3(((B + 31) / 32) * 32), 0, s, n, tok, tok_stride, amax, B);
   return cudaGetLastError();
 }
 
