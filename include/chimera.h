@@ -227,6 +227,22 @@ chimera_status chimera_op_attention(int dtype, int kv_split, int batch, int n_he
                                     int max_pages, const int32_t* n_ctx, const uint64_t* anc,
                                     void* out, void* out_lo, int ldo, int splits, void* cuda_stream);
 
+/* Same computation as chimera_op_linear with dtype 1 (bf16, tcgen05), but it allocates
+ * nothing: for callers that cannot allocate device memory when they call (code running
+ * under a fixed per-process memory budget, inside host callbacks or allocator hooks,
+ * or on memory owned by another allocator).  Its split-K scratch lives in arrays that
+ * the library defines at file scope (5.2 MB on every GPU that loads the library, held
+ * until the process exits).  The paper has no counterpart; it is a service of this
+ * library.  Limits: M <= 32, at most 4096 output tiles of 128 columns; larger sizes
+ * return CHIMERA_EINVAL with a message on stderr.  The first call on a device looks up
+ * the arrays' device addresses (make that first call outside any stream capture).
+ * Every call shares the arrays and keeps the last call's contents; the call clears
+ * what must start at zero.  Calls that overlap on the GPU race on the scratch: the
+ * caller serialises them (one stream, or explicit synchronisation). */
+chimera_status chimera_op_linear_noalloc(int epi, int out_f32, int M, int N, int K, const void* X,
+                                         const void* X_lo, int ldx, const void* W, void* Y, int ldy,
+                                         void* cuda_stream);
+
 #ifdef __cplusplus
 }
 #endif

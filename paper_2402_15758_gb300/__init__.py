@@ -74,6 +74,9 @@ _SIGS = {
     "chimera_op_linear": (ctypes.c_int, [ctypes.c_int] * 6 + [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int,
                                                               ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int,
                                                               ctypes.c_void_p]),
+    "chimera_op_linear_noalloc": (ctypes.c_int, [ctypes.c_int] * 5 + [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int,
+                                                                      ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int,
+                                                                      ctypes.c_void_p]),
     "chimera_op_attention": (ctypes.c_int, [ctypes.c_int] * 8 + [ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
                                                                  ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int,
                                                                  ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
@@ -274,6 +277,18 @@ def op_linear(X, W, Y, epi: int = 0, out_f32: bool = False, X_lo=None, stream=No
                                _ptr(Y), Y.stride(0), _stream_handle(stream))
     if st != 0:
         raise ChimeraError(st, "chimera_op_linear")
+
+
+def op_linear_noalloc(X, W, Y, epi: int = 0, out_f32: bool = False, X_lo=None, stream=None):
+    """Y (epilogue)= (X + X_lo) W^T through chimera_op_linear_noalloc (bf16 X, W; the
+    library keeps the scratch in static device arrays, so the call allocates nothing)."""
+    lib = load()
+    M, K = X.shape
+    N = W.shape[0]
+    st = lib.chimera_op_linear_noalloc(epi, int(out_f32), M, N, K, _ptr(X), _ptr(X_lo), X.stride(0), _ptr(W),
+                                       _ptr(Y), Y.stride(0), _stream_handle(stream))
+    if st != 0:
+        raise ChimeraError(st, "chimera_op_linear_noalloc")
 
 
 def op_attention(q, pool, page_table, n_ctx, anc, out, nq, q_local0, n_local, q_rows, n_heads, head_dim,
