@@ -42,17 +42,19 @@ def peaks():
     return 6800.0, "fallback"
 
 
-def step_bytes(cfg, n_ctx):
+def step_bytes(cfg, n_ctx, kv_elem_bytes=None):
     """Algorithmic HBM bytes of one step at committed length n_ctx (batch 1).
 
     Every weight matrix counts once per use (the trigram encoder and the draft block
     once per draft sub-step), embeddings only for the gathered rows, KV as the rows
-    read; activations are excluded."""
+    read; activations are excluded.  kv_elem_bytes is the stored size of one K (or V)
+    element: 4 for the fp32-equivalent hi+lo bf16 planes of precision mode 1, else the
+    weight element size."""
     d, F, V, L, K, N = (cfg["d_model"], cfg["ffn_dim"], cfg["vocab"], cfg["n_layers"],
                         cfg["n_draft_heads"], cfg["tree_nodes"])
     e = 2 if cfg["dtype"] == "bf16" else 4
     layer = (3 * d * d + d * d + 3 * d * F) * e
-    kv_row = 2 * d * e
+    kv_row = 2 * d * (kv_elem_bytes or e)
     verify = L * layer + V * d * e + N * d * e + L * (n_ctx + N) * kv_row
     draft_w = K * ((3 * d * d + d * d) * e + layer) + K * V * 2 * d * e + K * 3 * d * e
     draft_kv = sum((n_ctx + k + 1) * kv_row for k in range(K))
@@ -130,17 +132,97 @@ def cpu_sample(cfg, w_dev, n_ctx, threads):
     return dict(t_layer=t_layer, t_lm=t_lm, t_draft_sub=t_draft, step_s=est, threads=threads)
 
 
+def op_bench(args, hbm, peak_kind):
+    """One kernel through its C-ABI entry point, on the operand shapes the 7B step
+    launches, cycling through enough operand copies that every launch reads from HBM.
+    This is the small case for per-kernel ncu captures (a few GB on the device)."""
+    import paper_2402_15758_gb300 as pkg
+    from paper_2402_15758_gb300 import build as pkg_build
+    pkg_build.build()
+    pkg.load()
+    g = torch.Generator(device="cuda").manual_seed(0)
+    dev = "cuda"
+    if args.op == "linear":
+        M, N, K = (int(v) for v in args.shape.split(","))
+        wbytes = N * K * 2
+        copies = max(2, -(-400_000_000 // wbytes))
+        Ws = [(torch.randn(N, K, generator=g, device=dev) * 0.02).to(torch.bfloat16) for _ in range(copies)]
+        X32 = torch.randn(M, K, generator=g, device=dev)
+        X = X32.to(torch.bfloat16)
+        X_lo = (X32 - X.float()).to(torch.bfloat16)
+        Y = torch.empty(M, N, dtype=torch.bfloat16, device=dev)
+        nbytes = wbytes + 2 * M * K * 2 + M * N * 2
+
+        def launch(i):
+            pkg.op_linear(X, Ws[i % copies], Y, epi=0, X_lo=X_lo, stream=stream)
+        desc = (f"chimera_op_linear bf16 split operand (X_hi + X_lo), M={M} N={N} K={K}, "
+                f"{copies} weight copies ({copies * wbytes / 1e9:.2f} GB) cycled")
+    else:
+        H, hd, nq, n_ctx = 32, 128, 64, args.ctx
+        n_keys = n_ctx + nq
+        pages = (n_keys + 15) // 16
+        lay = pages * H * 4 * 16 * hd * 2
+        copies = max(2, -(-400_000_000 // lay))
+        pools = [torch.randn(pages, H, 4, 16, hd, generator=g, device=dev).to(torch.bfloat16)
+                 for _ in range(copies)]
+        pt = torch.arange(pages, dtype=torch.int32, device=dev).reshape(1, pages)
+        nctx = torch.tensor([n_ctx], dtype=torch.int32, device=dev)
+        anc_l = []
+        for i in range(nq):  # a 4-ary tree over the 64 rows: node i's parent is (i - 1) // 4
+            m, j = 0, i
+            while j >= 0:
+                m |= 1 << j
+                j = (j - 1) // 4 if j > 0 else -1
+            anc_l.append(m - (1 << 64) if m >= 1 << 63 else m)
+        anc = torch.tensor(anc_l, dtype=torch.int64, device=dev)
+        q = torch.randn(nq, H * hd, generator=g, device=dev)
+        out = torch.empty(nq, H * hd, dtype=torch.bfloat16, device=dev)
+        out_lo = torch.empty_like(out)
+        splits = max(1, min(16, -(-2 * torch.cuda.get_device_properties(0).multi_processor_count // H),
+                            (n_keys + 191) // 192))
+        nbytes = n_keys * H * hd * 4 * 2 + nq * H * hd * 4 + 2 * nq * H * hd * 2
+
+        def launch(i):
+            pkg.op_attention(q, pools[i % copies], pt, nctx, anc, out, nq=nq, q_local0=0, n_local=nq,
+                             q_rows=nq, n_heads=H, head_dim=hd, splits=splits, out_lo=out_lo, stream=stream)
+        desc = (f"chimera_op_attention 7B verify layer: 32 heads x 128, 64 tree rows, {n_ctx} context rows, "
+                f"4 bf16 KV planes, {splits} KV splits, {copies} KV pools cycled")
+    stream = torch.cuda.Stream()
+    with torch.cuda.stream(stream):
+        for i in range(args.warmup):
+            launch(i)
+        stream.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(args.steps):
+            launch(i)
+        e1.record(stream)
+        stream.synchronize()
+    ms = e0.elapsed_time(e1) / args.steps
+    gbs = nbytes / (ms * 1e-3) / 1e9
+    print(json.dumps({"op": args.op, "workload": desc, "us_per_launch": ms * 1e3, "bytes_per_launch": nbytes,
+                      "achieved_gbs": gbs, "peak_gbs": hbm, "peak_kind": peak_kind, "frac": gbs / hbm,
+                      "launches": args.steps, "note": "back-to-back launches with host calls between them"}))
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=30)
-    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="chimera", choices=["chimera", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--profile-steps", type=int, default=3)
+    ap.add_argument("--op", choices=["linear", "attention"], default=None,
+                    help="time one kernel entry point instead of the step")
+    ap.add_argument("--shape", default="64,22016,4096", help="--op linear: M,N,K")
+    ap.add_argument("--ctx", type=int, default=1024, help="--op attention: committed context rows")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
+    if args.op:
+        op_bench(args, *peaks())
+        return
 
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -200,9 +282,11 @@ def main():
         torch.distributed.barrier()
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.nvtx.range_push("timed_steps")
     e0.record(stream)
     ctx.step_async(args.steps)
     e1.record(stream)
+    torch.cuda.nvtx.range_pop()
     ctx.sync()
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1) / args.steps
@@ -249,7 +333,7 @@ def main():
     d2h = B * 4 + 4 + int(round(4 * emitted / args.steps))
 
     hbm, peak_kind = peaks()
-    nb = step_bytes(cfg, (n0 + n1) // 2)
+    nb = step_bytes(cfg, (n0 + n1) // 2, kv_elem_bytes=4 if ctx.kv_f32 else None)
     value = world * B * N / (ms * 1e-3)
     if lin_ms <= 0:
         raise RuntimeError("per-kernel profile returned no linear time")
