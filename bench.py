@@ -179,8 +179,8 @@ def op_bench(args, hbm, peak_kind):
         q = torch.randn(nq, H * hd, generator=g, device=dev)
         out = torch.empty(nq, H * hd, dtype=torch.bfloat16, device=dev)
         out_lo = torch.empty_like(out)
-        splits = max(1, min(16, -(-2 * torch.cuda.get_device_properties(0).multi_processor_count // H),
-                            (n_keys + 191) // 192))
+        # as the step: one cluster of <= 8 CTAs per head, all heads resident at once
+        splits = max(1, min(8, torch.cuda.get_device_properties(0).multi_processor_count // H, -(-n_keys // 64)))
         nbytes = n_keys * H * hd * 4 * 2 + nq * H * hd * 4 + 2 * nq * H * hd * 2
 
         def launch(i):

@@ -220,7 +220,9 @@ chimera_status chimera_op_linear(int dtype, int epi, int out_f32, int M, int N, 
  * slots n_ctx..; query i sees local row j iff bit j of anc[q_local0+i] (device
  * uint64); page_table device int32 [batch][max_pages]; out [batch*q_rows][ldo] in the
  * model dtype, out_lo (optional, bf16 only) its lo half.  nq <= 64, n_local <= 64,
- * hd in {64, 128}. */
+ * hd in {64, 128}.  `splits` cuts each sequence's keys into that many contiguous
+ * ranges: at most 16, and at most 8 for dtype 1 with hd 128 (the ranges of one
+ * (sequence, head) run as one thread-block cluster); EINVAL beyond. */
 chimera_status chimera_op_attention(int dtype, int kv_split, int batch, int n_heads, int head_dim,
                                     int nq, int q_local0, int n_local, const float* q, int ldq,
                                     int q_rows, const void* pool, const int32_t* page_table,

@@ -46,6 +46,75 @@ __device__ __forceinline__ void store_act(bf16* hi, bf16* lo, size_t i, float x)
   if (lo) lo[i] = __float2bfloat16_rn(x - __bfloat162float(h));
 }
 
+
+// Four consecutive values into the KV cache (T = cache element type), as one vector
+// store; store4_split writes the two-term split x = hi + lo into a hi and a lo plane.
+template <typename T>
+__device__ __forceinline__ void store4(T* dst, float4 v);
+template <>
+__device__ __forceinline__ void store4<float>(float* dst, float4 v) { *reinterpret_cast<float4*>(dst) = v; }
+template <>
+__device__ __forceinline__ void store4<bf16>(bf16* dst, float4 v) {
+  __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y), b = __floats2bfloat162_rn(v.z, v.w);
+  uint2 u;
+  u.x = *reinterpret_cast<uint32_t*>(&a);
+  u.y = *reinterpret_cast<uint32_t*>(&b);
+  *reinterpret_cast<uint2*>(dst) = u;
+}
+
+template <typename T>
+__device__ __forceinline__ void store4_split(T* hi, T* lo, float4 v) {
+  store4<T>(hi, v);
+}
+template <>
+__device__ __forceinline__ void store4_split<bf16>(bf16* hi, bf16* lo, float4 v) {
+  __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y), b = __floats2bfloat162_rn(v.z, v.w);
+  const float2 fa = __bfloat1622float2(a), fb = __bfloat1622float2(b);
+  __nv_bfloat162 la = __floats2bfloat162_rn(v.x - fa.x, v.y - fa.y), lb = __floats2bfloat162_rn(v.z - fb.x, v.w - fb.y);
+  uint2 u, w;
+  u.x = *reinterpret_cast<uint32_t*>(&a);
+  u.y = *reinterpret_cast<uint32_t*>(&b);
+  w.x = *reinterpret_cast<uint32_t*>(&la);
+  w.y = *reinterpret_cast<uint32_t*>(&lb);
+  *reinterpret_cast<uint2*>(hi) = u;
+  *reinterpret_cast<uint2*>(lo) = w;
+}
+
+// Rotate-half RoPE of four pairs (x1[i], x2[i]) = (x[j+i], x[j+i+hd/2]) with
+// c = cos, s = sin of their angles: the first and the second half of the result.
+__device__ __forceinline__ float4 rot_lo(float4 x1, float4 x2, float4 c, float4 s) {
+  return make_float4(x1.x * c.x - x2.x * s.x, x1.y * c.y - x2.y * s.y, x1.z * c.z - x2.z * s.z, x1.w * c.w - x2.w * s.w);
+}
+__device__ __forceinline__ float4 rot_hi(float4 x1, float4 x2, float4 c, float4 s) {
+  return make_float4(x2.x * c.x + x1.x * s.x, x2.y * c.y + x1.y * s.y, x2.z * c.z + x1.z * s.z, x2.w * c.w + x1.w * s.w);
+}
+
+// ---------------------------------------------------------------------------
+// Thread-block clusters: rank, cluster-wide barrier, distributed shared memory
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// Address of the same shared-memory location in the CTA of cluster rank `rank`.
+__device__ __forceinline__ uint32_t dsmem_addr(uint32_t smem_addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_addr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ float ld_dsmem(uint32_t addr) {
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr) : "memory");
+  return v;
+}
+__device__ __forceinline__ float4 ld_dsmem4(uint32_t addr) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(addr)
+               : "memory");
+  return v;
+}
+
 // Programmatic dependent launch: let the next kernel in the stream start launching, and
 // wait until the previous kernel has completed with its memory visible (both are no-ops
 // when the launch has no programmatic dependency).

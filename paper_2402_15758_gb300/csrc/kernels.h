@@ -91,10 +91,33 @@ struct AttnParams {
   float* ws;              // [B][H][splits][nq_max][hd + 4] (output, max, sum, pad)
   int* counters;          // [B][H], zero between launches
   int nq_max;
+  // Fused RoPE + KV write (bf16 models, head_dim 128).  With qkv set, the queries and
+  // the nq fresh local rows come from the fp32 projections: row (b * q_rows + i) holds
+  // q at column h*hd, k at H*hd + h*hd, v at 2*H*hd + h*hd.  Query / fresh row i sits at
+  // position n_ctx + pos_base + (pos_off ? pos_off[i] : i) and at local row q_local0 + i
+  // (slot n_ctx + q_local0 + i); the kernel rotates q and k and writes k and v of its
+  // key range into the pool before reading it.
+  const float* qkv;
+  int ldqkv;
+  const float2* rope;     // [max_pos][hd / 2] (cos, sin)
+  int max_pos;
+  int pos_base;
+  const int* pos_off;
+  // 1: the preceding kernel in the stream lets its dependents launch only after its
+  // own griddepcontrol.wait, so every kernel before it is complete and committed KV
+  // rows (slots < n_ctx) may be read before this kernel's own wait
+  int prewait_kv;
+  int* err;
 };
 // dtype: 0 fp32 model (fp32 KV), 1 bf16 model (bf16 KV planes).
 cudaError_t attention(const AttnParams& p, int dtype, cudaStream_t s);
 size_t attn_ws_floats(int B, int H, int splits, int nq_max, int hd);
+// Splits per (b, h) for the tensor-core tree attention (bf16, head_dim 128): at most
+// `want` and 8 (one thread-block cluster per (b, h)), reduced until all B * H clusters
+// are resident at once.  Other paths return `want` unchanged.
+int attn_pick_splits(int dtype, int hd, int planes, int B, int H, int want);
+// True when attention() fuses RoPE and the KV write (qkv given) for this model.
+bool attn_fuses_rope(int dtype, int hd);
 
 // ----------------------------------------------------------------------------
 // row-wise / small kernels

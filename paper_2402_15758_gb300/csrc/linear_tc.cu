@@ -151,7 +151,9 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const _
     *s_last = 0;
     mbar_fence_init();
   }
-  pdl_trigger();  // the next kernel may start launching (its CTAs fit once ours exit)
+  // Programmatic dependent launch: every thread calls pdl_trigger() only after its own
+  // pdl_wait(), so a dependent that starts early knows that every kernel before this
+  // one is complete (it may read their outputs before its own wait).
   if (warp == 0 && lane == 0) {
     prefetch_tensormap(&p.tmA);
     if (p.ft_split < p.feat_tiles) prefetch_tensormap(&p.tmA2);
@@ -212,6 +214,7 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const _
         issued_mask |= 1u << i;
       }
       pdl_wait();
+      pdl_trigger();
       for (uint32_t i = 0; i < npre; ++i) load_b(u_begin + i, smem + i * stage_bytes + a_atom * BKA, &full[i]);
       stage = static_cast<int>(npre % p.stages);
       phase = (npre == static_cast<uint32_t>(p.stages)) ? 1u : 0u;
@@ -233,8 +236,13 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const _
         for (int s = 0; s < p.stages; ++s)
           if (issued_mask >> s & 1u) mbar_wait_plain(&full[s], issued_par >> s & 1u, 200000000ull);
       }
+    } else {
+      pdl_wait();
+      pdl_trigger();
     }
   } else if (warp == 1) {
+    pdl_wait();
+    pdl_trigger();
     if (lane == 0) {
       // ---------------- MMA issuer ----------------
       const uint32_t idesc = idesc_bf16_m128(p.BN);
@@ -290,6 +298,7 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const _
   } else {
     // ---------------- epilogue (warps 2..5, TMEM lanes 32*(warp%4) ..) ----------------
     pdl_wait();  // Y, the split workspace and the counters are shared with earlier kernels
+    pdl_trigger();
     const int q = warp & 3;
     const int row = q * 32 + lane;
     int buf = 0;

@@ -334,17 +334,36 @@ bool make_lin(chimera_ctx* ctx, Lin* l, int M, int N, int K, const void* X, cons
 // attention (the draft), and about three 64-key tiles per split for tree queries so
 // the per-split partials stay few (their merge is latency-bound).
 int att_splits(const chimera_ctx* ctx, int B, int nq, int n_keys) {
+  if (attn_fuses_rope(ctx->dtype, ctx->hd)) {
+    // tensor-core tree attention: one cluster of S CTAs per (b, h), all resident at once
+    const int want = std::max(1, std::min(ctx->num_sms / (B * ctx->H), (n_keys + 63) / 64));
+    return attn_pick_splits(ctx->dtype, ctx->hd, ctx->kv_planes, B, ctx->H, want);
+  }
   const int target = 2 * ctx->num_sms;
   int s = (target + B * ctx->H - 1) / (B * ctx->H);
   if (nq > 1) s = std::min(s, (n_keys + 191) / 192);
   return std::max(1, std::min(16, s));
 }
 
+// With qkv (models where attn_fuses_rope holds) the kernel also rotates q and the nq
+// fresh rows' k (positions n + pos_base + pos_off[i]) and writes their k, v to the pool;
+// its predecessor is always the QKV linear, which triggers only after its own wait.
 cudaError_t run_attention(chimera_ctx* ctx, bool draft_pool, int layer, int nq, const int* nq_dev, int q_local0,
                           int n_local, const int* n_local_dev, const unsigned long long* anc, int q_rows, int splits,
-                          int nq_max, double bytes) {
+                          int nq_max, double bytes, const float* qkv = nullptr, int pos_base = 0,
+                          const int* pos_off = nullptr) {
   Scope sc(ctx, CHIMERA_KIND_ATTENTION, bytes);
   AttnParams p{};
+  if (qkv) {
+    p.qkv = qkv;
+    p.ldqkv = 3 * ctx->d;
+    p.rope = ctx->d_rope;
+    p.max_pos = ctx->max_pos;
+    p.pos_base = pos_base;
+    p.pos_off = pos_off;
+    p.prewait_kv = 1;
+  }
+  p.err = ctx->d_err;
   p.q = ctx->qr;
   p.ldq = ctx->d;
   p.q_rows = q_rows;
@@ -443,9 +462,14 @@ cudaError_t enqueue_layer(chimera_ctx* ctx, int l, const Lin* lin, int rows, int
   const int d = ctx->d;
   RUN(run_norm(ctx, ctx->x, w.attn_norm, rows, ctx->qkv, 3 * d));
   RUN(run_lin(ctx, lin[0]));
-  RUN(run_rope(ctx, false, l, ctx->qkv, 3 * d, 0, d, 2 * d, rows_per_seq, valid, 0, 0, 0, pos_off));
-  RUN(run_attention(ctx, false, l, rows_per_seq, valid, 0, rows_per_seq, valid, anc, rows_per_seq, splits,
-                    rows_per_seq, kv_bytes));
+  if (attn_fuses_rope(ctx->dtype, ctx->hd)) {
+    RUN(run_attention(ctx, false, l, rows_per_seq, valid, 0, rows_per_seq, valid, anc, rows_per_seq, splits,
+                      rows_per_seq, kv_bytes, ctx->qkv, 0, pos_off));
+  } else {
+    RUN(run_rope(ctx, false, l, ctx->qkv, 3 * d, 0, d, 2 * d, rows_per_seq, valid, 0, 0, 0, pos_off));
+    RUN(run_attention(ctx, false, l, rows_per_seq, valid, 0, rows_per_seq, valid, anc, rows_per_seq, splits,
+                      rows_per_seq, kv_bytes));
+  }
   RUN(run_lin(ctx, lin[1]));
   RUN(run_norm(ctx, ctx->x, w.ffn_norm, rows, ctx->gu, 2 * ctx->F));
   RUN(run_lin(ctx, lin[2]));
@@ -483,9 +507,14 @@ cudaError_t enqueue_step(chimera_ctx* ctx) {
     RUN(run_lin(ctx, ctx->tri2));
     RUN(run_norm(ctx, ctx->dres, ctx->draft.attn_norm, B, ctx->qkv, 3 * d));
     RUN(run_lin(ctx, ctx->dqkv));
-    RUN(run_rope(ctx, true, 0, ctx->qkv, 3 * d, 0, d, 2 * d, 1, nullptr, 0, k, k, nullptr));
-    RUN(run_attention(ctx, true, 0, 1, nullptr, k, k + 1, nullptr, ctx->d_chain, 1, ctx->att_splits_draft, 1,
-                      kv_read_bytes(ctx, k + 1, true)));
+    if (attn_fuses_rope(ctx->dtype, ctx->hd)) {
+      RUN(run_attention(ctx, true, 0, 1, nullptr, k, k + 1, nullptr, ctx->d_chain, 1, ctx->att_splits_draft, 1,
+                        kv_read_bytes(ctx, k + 1, true), ctx->qkv, k, nullptr));
+    } else {
+      RUN(run_rope(ctx, true, 0, ctx->qkv, 3 * d, 0, d, 2 * d, 1, nullptr, 0, k, k, nullptr));
+      RUN(run_attention(ctx, true, 0, 1, nullptr, k, k + 1, nullptr, ctx->d_chain, 1, ctx->att_splits_draft, 1,
+                        kv_read_bytes(ctx, k + 1, true)));
+    }
     RUN(run_lin(ctx, ctx->dwo));
     RUN(run_norm(ctx, ctx->dres, ctx->draft.ffn_norm, B, ctx->gu, 2 * ctx->F));
     RUN(run_lin(ctx, ctx->dgate));
@@ -1324,7 +1353,7 @@ chimera_status chimera_op_attention(int dtype, int kv_split, int batch, int n_he
                                     void* out, void* out_lo, int ldo, int splits, void* cuda_stream) {
   if ((dtype != 0 && dtype != 1) || batch < 1 || n_heads < 1 || (head_dim != 64 && head_dim != 128) || nq < 1 ||
       nq > 64 || n_local < 0 || n_local > 64 || q_local0 < 0 || !q || !pool || !page_table || !n_ctx || !anc || !out ||
-      splits < 1 || splits > 64 || batch * n_heads > 64 * 256)
+      splits < 1 || splits > 16 || (dtype == 1 && head_dim == 128 && splits > 8) || batch * n_heads > 64 * 256)
     return CHIMERA_EINVAL;
   std::lock_guard<std::mutex> lk(g_op_mu);
   if (!op_scratch()) return CHIMERA_ENOMEM;

@@ -98,44 +98,6 @@ __global__ void __launch_bounds__(NORM_THREADS) rmsnorm_kernel(const float* __re
 // Rotate-half RoPE of q and k, plus the write of k and v into the paged cache
 // (T = element type of the cache).  One block per row; an item is 4 consecutive
 // pair indices j..j+3 of one head (pairs (j, j + hd/2)).
-template <typename T>
-__device__ __forceinline__ void store4(T* dst, float4 v);
-template <>
-__device__ __forceinline__ void store4<float>(float* dst, float4 v) { *reinterpret_cast<float4*>(dst) = v; }
-template <>
-__device__ __forceinline__ void store4<bf16>(bf16* dst, float4 v) {
-  __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y), b = __floats2bfloat162_rn(v.z, v.w);
-  uint2 u;
-  u.x = *reinterpret_cast<uint32_t*>(&a);
-  u.y = *reinterpret_cast<uint32_t*>(&b);
-  *reinterpret_cast<uint2*>(dst) = u;
-}
-
-// Two-term bf16 split of 4 values into a hi plane and a lo plane.
-template <typename T>
-__device__ __forceinline__ void store4_split(T* hi, T* lo, float4 v) {
-  store4<T>(hi, v);
-}
-template <>
-__device__ __forceinline__ void store4_split<bf16>(bf16* hi, bf16* lo, float4 v) {
-  __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y), b = __floats2bfloat162_rn(v.z, v.w);
-  const float2 fa = __bfloat1622float2(a), fb = __bfloat1622float2(b);
-  __nv_bfloat162 la = __floats2bfloat162_rn(v.x - fa.x, v.y - fa.y), lb = __floats2bfloat162_rn(v.z - fb.x, v.w - fb.y);
-  uint2 u, w;
-  u.x = *reinterpret_cast<uint32_t*>(&a);
-  u.y = *reinterpret_cast<uint32_t*>(&b);
-  w.x = *reinterpret_cast<uint32_t*>(&la);
-  w.y = *reinterpret_cast<uint32_t*>(&lb);
-  *reinterpret_cast<uint2*>(hi) = u;
-  *reinterpret_cast<uint2*>(lo) = w;
-}
-
-__device__ __forceinline__ float4 rot_lo(float4 x1, float4 x2, float4 c, float4 s) {
-  return make_float4(x1.x * c.x - x2.x * s.x, x1.y * c.y - x2.y * s.y, x1.z * c.z - x2.z * s.z, x1.w * c.w - x2.w * s.w);
-}
-__device__ __forceinline__ float4 rot_hi(float4 x1, float4 x2, float4 c, float4 s) {
-  return make_float4(x2.x * c.x + x1.x * s.x, x2.y * c.y + x1.y * s.y, x2.z * c.z + x1.z * s.z, x2.w * c.w + x1.w * s.w);
-}
 
 template <typename T>
 __global__ void rope_kv_kernel(const RopeKvParams p) {

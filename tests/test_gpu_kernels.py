@@ -119,7 +119,8 @@ ATT_CASES = [
     (1, 4, 64, [77], 16, 16, 0, 5),
     (2, 3, 128, [0, 300], 64, 64, 0, 7),
     (3, 2, 128, [16, 1, 129], 5, 1, 4, 3),     # draft-style: one query, local rows 0..4
-    (1, 2, 128, [1000], 64, 64, 0, 16),
+    (1, 2, 128, [1000], 64, 64, 0, 8),
+    (2, 3, 128, [700, 3], 64, 64, 0, 4),     # a split whose key range is empty for b=1
 ]
 
 
