@@ -322,6 +322,10 @@ __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commi
 __device__ __forceinline__ void cp_async_wait1() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
 
 __device__ __forceinline__ void cp_async_wait0() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait2() { asm volatile("cp.async.wait_group 2;" ::: "memory"); }
+
+constexpr int TREE_STAGES = 3;         // KV tiles in the ring
+constexpr int TREE_PAGE_CACHE = 1024;  // page indices cached per CTA (256 tiles)
 
 // SPLIT: the cache holds K_hi, K_lo, V_hi, V_lo planes (three-term products);
 // otherwise K, V planes (K_lo = V_lo = 0: two-term products for the split queries and P).
@@ -331,14 +335,17 @@ __device__ __forceinline__ void cp_async_wait0() { asm volatile("cp.async.wait_g
 // 16*(w & 3) .. +15 and the key half (w >> 2) of every tile, the two halves merge in
 // shared memory, and the S partial states (unnormalised output, running max, running
 // sum) merge across the cluster through distributed shared memory: CTA r finishes the
-// query rows [r * ceil(nq / S), ...).  KV tiles stream through a two-stage cp.async
-// ring; committed-context tiles may be requested before the kernel's dependency wait.
+// query rows [r * ceil(nq / S), ...).  KV tiles stream through a three-stage cp.async
+// ring (two tiles in flight while one is consumed); the CTA's page indices are cached
+// in shared memory, and committed-context tiles may be requested before the kernel's
+// dependency wait.
 template <bool SPLIT>
 __global__ void __launch_bounds__(MWARPS * 32, 1) attn_tree_kernel(const AttnParams p) {
   constexpr int NP = SPLIT ? 4 : 2;                  // planes per (block, head)
   constexpr int STAGE = NP * MKT * MLDS;             // bf16 elements per pipeline stage
   constexpr int PREC = MHD + 4;                      // partial record: o[128], m, l, pad
   extern __shared__ __align__(16) uint8_t smem_raw[];
+  __shared__ int s_pages[TREE_PAGE_CACHE];
   bf16* stage_base = reinterpret_cast<bf16*>(smem_raw);
   float* xch = reinterpret_cast<float*>(smem_raw);                  // [4][32][68] key-half merge
   float* part = reinterpret_cast<float*>(smem_raw) + 4 * 32 * 68;   // [64][PREC] cluster merge
@@ -358,6 +365,13 @@ __global__ void __launch_bounds__(MWARPS * 32, 1) attn_tree_kernel(const AttnPar
   const int tps = (ntiles + S - 1) / S;
   const int t0 = min(ntiles, s * tps);
   const int t1 = min(ntiles, t0 + tps);
+  // page indices of the CTA's pages (the table is not written during a step)
+  const bool cached = (t1 - t0) * 4 <= TREE_PAGE_CACHE;
+  if (cached) {
+    const int np = min((t1 - t0) * 4, p.max_pages - t0 * 4);
+    for (int i = threadIdx.x; i < np; i += blockDim.x) s_pages[i] = p.page_table[b * p.max_pages + t0 * 4 + i];
+  }
+  __syncthreads();
 
   // staging: thread copies 16-byte chunk (tid & 15) of key row (tid >> 4) + 16u of every
   // plane, u = 0..3 (one 16-key page each); keys at or past kend are zero-filled
@@ -370,7 +384,7 @@ __global__ void __launch_bounds__(MWARPS * 32, 1) attn_tree_kernel(const AttnPar
       const bool valid = kg < kend;
       const bf16* src = pool;
       if (valid) {
-        const int page = p.page_table[b * p.max_pages + t * 4 + u];
+        const int page = cached ? s_pages[(t - t0) * 4 + u] : p.page_table[b * p.max_pages + t * 4 + u];
         src = pool + (static_cast<size_t>(page) * p.H + h) * NP * 16 * MHD + krow * MHD + kch * 8;
       }
 #pragma unroll
@@ -384,7 +398,7 @@ __global__ void __launch_bounds__(MWARPS * 32, 1) attn_tree_kernel(const AttnPar
   // committed-context tiles do not depend on the preceding kernels of this step
   int issued = t0;
   if (p.prewait_kv) {
-    while (issued < t1 && issued < t0 + 2 && (issued + 1) * MKT <= nctx) {
+    while (issued < t1 && issued < t0 + TREE_STAGES && (issued + 1) * MKT <= nctx) {
       issue_tile(issued, issued - t0, nctx);
       ++issued;
     }
@@ -444,7 +458,7 @@ __global__ void __launch_bounds__(MWARPS * 32, 1) attn_tree_kernel(const AttnPar
     __threadfence_block();
     __syncthreads();
   }
-  while (issued < t1 && issued < t0 + 2) {
+  while (issued < t1 && issued < t0 + TREE_STAGES) {
     issue_tile(issued, issued - t0, total);
     ++issued;
   }
@@ -513,8 +527,11 @@ __global__ void __launch_bounds__(MWARPS * 32, 1) attn_tree_kernel(const AttnPar
   ATRACE(1);
 
   for (int t = t0; t < t1; ++t) {
-    const int st = (t - t0) & 1;
-    if (t + 1 < issued)
+    const int st = (t - t0) % TREE_STAGES;
+    // tiles t .. issued-1 are in flight: let the newer ones stay pending
+    if (issued - t >= 3)
+      cp_async_wait2();
+    else if (issued - t == 2)
       cp_async_wait1();
     else
       cp_async_wait0();
@@ -627,7 +644,7 @@ __global__ void __launch_bounds__(MWARPS * 32, 1) attn_tree_kernel(const AttnPar
     }
     __syncthreads();  // this stage may be refilled now
     if (issued < t1) {
-      issue_tile(issued, (issued - t0) & 1, total);
+      issue_tile(issued, (issued - t0) % TREE_STAGES, total);
       ++issued;
     }
   }
@@ -747,7 +764,7 @@ __global__ void __launch_bounds__(MWARPS * 32, 1) attn_tree_kernel(const AttnPar
 
 template <bool SPLIT>
 size_t tree_smem() {
-  return 2 * static_cast<size_t>(SPLIT ? 4 : 2) * MKT * MLDS * sizeof(bf16);  // two pipeline stages
+  return TREE_STAGES * static_cast<size_t>(SPLIT ? 4 : 2) * MKT * MLDS * sizeof(bf16);
 }
 
 template <bool SPLIT>

@@ -22,6 +22,7 @@ struct TcLinearParams {
   int tok_tiles, feat_tiles, kblocks;
   long long units;   // feat_tiles * tok_tiles * kblocks
   int stages;        // smem pipeline depth
+  int vec_red;       // EPI_RESID through float4 reductions
   int epi;           // EPI_*
   int out_f32;       // Y is fp32 (else bf16) for EPI_STORE / EPI_SILU
   void* Y;

@@ -39,7 +39,7 @@ namespace {
 #define CHIMERA_LIN_PIPE_KB 200
 #endif
 #ifndef CHIMERA_LIN_BK_ATOMS
-#define CHIMERA_LIN_BK_ATOMS 1
+#define CHIMERA_LIN_BK_ATOMS 2
 #endif
 constexpr int BM = 128;   // weight rows per tile (UMMA M)
 constexpr int ATOM = 64;  // one 128-byte swizzle atom of bf16 along K
@@ -96,6 +96,28 @@ __device__ __forceinline__ void epi_store16(const TcLinearParams& p, int m0, int
   }
 }
 
+// EPI_RESID with float4 reductions: the warp's 32 feature rows x 16 token columns go
+// through shared memory (sw: [16][33] floats) so that each lane adds runs of four
+// consecutive features of one token (one vector red.global.add instead of four).
+__device__ __forceinline__ void epi_red16(const TcLinearParams& p, int m0, int f0, int lane, const float (&v)[16],
+                                          float* sw) {
+#pragma unroll
+  for (int j = 0; j < 16; ++j) sw[j * 33 + lane] = v[j];
+  __syncwarp();
+  float* y = static_cast<float*>(p.Y);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int idx = i * 32 + lane;
+    const int c = idx >> 3, k = (idx & 7) * 4;  // token c, features f0 + k .. f0 + k + 3
+    if (m0 + c < p.M && f0 + k < p.N) {
+      const float* s = sw + c * 33 + k;
+      atomicAdd(reinterpret_cast<float4*>(y + static_cast<size_t>(m0 + c) * p.ldy + f0 + k),
+                make_float4(s[0], s[1], s[2], s[3]));
+    }
+  }
+  __syncwarp();
+}
+
 __device__ __forceinline__ bool bar_any(int id, int nthreads, bool pred) {
   uint32_t r;
   asm volatile(
@@ -133,6 +155,7 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const _
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   int* s_abort = reinterpret_cast<int*>(tmem_slot + 1);
   int* s_last = s_abort + 1;
+  float* s_red = reinterpret_cast<float*>(smem + p.stages * stage_bytes + 1024);  // [4 warps][16][33]
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -323,7 +346,10 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const _
         for (int c0 = 0; c0 < p.BN; c0 += 16) {
           float v[16];
           tmem_ld_16(tbase + c0, v);
-          epi_store16(p, m0 + c0, f, v);
+          if (p.vec_red)
+            epi_red16(p, m0 + c0, ft * BM + q * 32, lane, v, s_red + q * 16 * 33);
+          else
+            epi_store16(p, m0 + c0, f, v);
         }
         tc_fence_before();
         mbar_arrive(&tempty[buf]);
@@ -537,7 +563,9 @@ int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, const
   if (X_lo && encode_2d_bf16(&p.tmB2, X_lo, K, M, ldx, ATOM, p.BN) != 0) return fail("tensor map of X_lo");
   const int sms = tc_num_sms() * CTAS_PER_SM;
   plan->grid = static_cast<int>(p.units < sms ? p.units : sms);
-  plan->smem = 1024 + static_cast<size_t>(p.stages) * stage_bytes + 2 * MAX_STAGES * 8 + 5 * 8 + 64;
+  // float4 reductions need 16-byte aligned rows of Y and whole float4 runs of features
+  p.vec_red = (epi == EPI_RESID && (reinterpret_cast<uintptr_t>(Y) & 15) == 0 && ldy % 4 == 0 && N % 4 == 0) ? 1 : 0;
+  plan->smem = 1024 + static_cast<size_t>(p.stages) * stage_bytes + 1024 + 4 * 16 * 33 * sizeof(float);
   plan->weight_bytes = 2.0 * N * K;
   return 0;
 }
