@@ -532,7 +532,11 @@ int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, const
   p.M = M;
   p.N = N;
   p.K = K;
+  p.has_lo = X_lo ? 1 : 0;
+  // token tile: all rows when the ring still holds at least two stages, else halves
   p.BN = M <= MAX_BN ? ((M + 15) / 16) * 16 : MAX_BN;
+  while (p.BN > 16 && PIPE_SMEM / (BM * BK * 2 + (p.has_lo ? 2 : 1) * p.BN * BK * 2) < 2)
+    p.BN = ((p.BN / 2 + 15) / 16) * 16;
   p.tok_tiles = (M + p.BN - 1) / p.BN;
   p.feat_tiles = (N + BM - 1) / BM;
   p.ft_split = W2 ? N1 / BM : p.feat_tiles;
