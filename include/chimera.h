@@ -214,7 +214,8 @@ chimera_status chimera_op_linear(int dtype, int epi, int out_f32, int M, int N, 
 
 /* Tree-masked attention over a paged KV pool [blocks][H][planes][16][hd] (device):
  * dtype 0: fp32 planes K, V; dtype 1: bf16 planes K, V, or with kv_split the two-term
- * split K_hi, K_lo, V_hi, V_lo.  q fp32 [batch*q_rows][ldq] rotated queries,
+ * split K_hi, K_lo, V_hi, V_lo; n_blocks = blocks in the pool (every page-table entry
+ * of a visible key must be below it).  q fp32 [batch*q_rows][ldq] rotated queries,
  * query i of sequence b at row b*q_rows+i;
  * n_ctx (device int32 [batch]) committed rows visible to all; n_local rows follow at
  * slots n_ctx..; query i sees local row j iff bit j of anc[q_local0+i] (device
@@ -225,7 +226,7 @@ chimera_status chimera_op_linear(int dtype, int epi, int out_f32, int M, int N, 
  * (sequence, head) run as one thread-block cluster); EINVAL beyond. */
 chimera_status chimera_op_attention(int dtype, int kv_split, int batch, int n_heads, int head_dim,
                                     int nq, int q_local0, int n_local, const float* q, int ldq,
-                                    int q_rows, const void* pool, const int32_t* page_table,
+                                    int q_rows, const void* pool, int n_blocks, const int32_t* page_table,
                                     int max_pages, const int32_t* n_ctx, const uint64_t* anc,
                                     void* out, void* out_lo, int ldo, int splits, void* cuda_stream);
 

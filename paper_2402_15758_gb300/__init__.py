@@ -78,7 +78,8 @@ _SIGS = {
                                                                       ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int,
                                                                       ctypes.c_void_p]),
     "chimera_op_attention": (ctypes.c_int, [ctypes.c_int] * 8 + [ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
-                                                                 ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int,
+                                                                 ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p,
+                                                                 ctypes.c_int,
                                                                  ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
                                                                  ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
                                                                  ctypes.c_void_p]),
@@ -301,7 +302,8 @@ def op_attention(q, pool, page_table, n_ctx, anc, out, nq, q_local0, n_local, q_
     dtype = 0 if out.element_size() == 4 else 1
     kv_split = int(pool.shape[2] == 4)
     st = lib.chimera_op_attention(dtype, kv_split, n_ctx.shape[0], n_heads, head_dim, nq, q_local0, n_local,
-                                  _ptr(q), q.stride(0), q_rows, _ptr(pool), _ptr(page_table), page_table.shape[1],
+                                  _ptr(q), q.stride(0), q_rows, _ptr(pool), pool.shape[0], _ptr(page_table),
+                                  page_table.shape[1],
                                   _ptr(n_ctx), _ptr(anc), _ptr(out), _ptr(out_lo), out.stride(0), splits,
                                   _stream_handle(stream))
     if st != 0:

@@ -1,0 +1,767 @@
+// Tree-masked attention on the 5th-generation tensor cores (bf16 models, head_dim 128).
+//
+// One CTA per (KV split s, head h, sequence b); the S splits of a (b, h) form one
+// thread-block cluster and merge their partial states through distributed shared
+// memory.  Per 64-key tile of the CTA's key range:
+//
+//   S  = Q K^T    tcgen05.mma, M = 64 queries, N = 64 keys, K = 128 dims, fp32 in TMEM
+//   P  = exp(S - m) on the softmax warps (tcgen05.ld of S, mask, online max/sum)
+//   O += P V      tcgen05.mma, M = 64 queries, N = 128 dims, K = 64 keys, fp32 in TMEM
+//
+// Every bf16 operand is a two-term split x = hi + lo of an fp32 value (queries, keys,
+// values, probabilities); each product takes hi*hi + lo*hi + hi*lo, so the result
+// matches fp32 arithmetic to ~2^-16.  Q, K and V tiles sit in shared memory in the
+// K-major 128-byte-swizzled layout (V is read MN-major by the PV product); P is written
+// by the softmax warps in the same layout.  Two S accumulators in tensor memory let the
+// QK product of tile t+1 overlap the softmax of tile t.  The running max is only raised
+// (and O rescaled) when a row's maximum grows by more than a factor ~e^8 (keeping P, l
+// and O finite in fp32); the final normalisation uses the same max, so the result is
+// exact.  Scores and maxima are kept in base-2 units (scaled by log2 e).
+//
+// Warps: 0..3 softmax + epilogue (tensor-memory lanes 32w.., rows 16w..16w+15),
+// 4 loads the KV tiles (one thread issues TMA copies of 16-row page boxes into
+// two-stage rings for K and for V, 128-byte swizzle applied by the copy engine), 5
+// issues the MMAs and owns the tensor-memory allocation.
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace chimera {
+namespace {
+
+constexpr int HD = 128;
+constexpr int KT = 64;                      // keys per tile
+constexpr int NQ = 64;                      // query rows (UMMA M)
+constexpr int SOFT_WARPS = 4, LOAD_WARPS = 1;
+constexpr int THREADS = (SOFT_WARPS + LOAD_WARPS + 1) * 32;
+constexpr int MMA_WARP = SOFT_WARPS + LOAD_WARPS;
+constexpr int ATOM_ROWS64 = 64 * 128;       // bytes of one 64-row x 128-byte swizzle atom column
+constexpr int TILE64 = 2 * ATOM_ROWS64;     // 64 rows x 128 bf16 (two atoms): 16 KB
+constexpr int STAGES = 2;
+constexpr int L2_AHEAD = 3;                 // tiles requested into L2 beyond the newest ring load
+constexpr int PAGE_CACHE = 1024;
+constexpr float RESCALE_LOG2 = 11.5f;        // raise the running max when it grows by > 2^11.5 (~e^8)
+constexpr uint32_t TMEM_COLS = 256;          // S[2] (64 cols each) + O (128 cols)
+constexpr int PREC = HD + 4;                 // partial record (o[128], m, l, pad)
+
+// Byte offset of 16-byte chunk c (0..7) of row r inside a 128-byte-swizzled atom column.
+__device__ __forceinline__ uint32_t swz(int r, int c) {
+  return static_cast<uint32_t>((r >> 3) * 1024 + (r & 7) * 128 + ((c ^ (r & 7)) << 4));
+}
+
+// K-major (or, for the PV B operand, MN-major) 128-byte-swizzled smem descriptor.
+__device__ __forceinline__ uint64_t desc_sw128(uint32_t addr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((addr & 0x3FFFFu) >> 4);
+  d |= static_cast<uint64_t>((lbo >> 4) & 0x3FFFu) << 16;
+  d |= static_cast<uint64_t>((sbo >> 4) & 0x3FFFu) << 32;
+  d |= static_cast<uint64_t>(1) << 46;
+  d |= static_cast<uint64_t>(2) << 61;
+  return d;
+}
+
+// kind::f16 instruction descriptor: D fp32, A and B bf16, A K-major, B K-major or
+// MN-major (b_mn), shape M x N.
+__device__ __forceinline__ uint32_t idesc_f16(int m, int n, bool b_mn) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | (b_mn ? (1u << 16) : 0u) | (static_cast<uint32_t>(n >> 3) << 17) |
+         (static_cast<uint32_t>(m >> 4) << 24);
+}
+
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* r) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+      "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]),
+      "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+      : "memory");
+}
+__device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+__device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+__device__ __forceinline__ void fence_async_global() { asm volatile("fence.proxy.async.global;" ::: "memory"); }
+
+// Kernel arguments: the tensor map of the pool viewed as [pool_rows][hd] bf16 (box
+// 64 dims x 16 rows) and the attention parameters.
+struct TcArgs {
+  CUtensorMap kv_map;
+  AttnParams p;
+};
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
+  const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<const uint32_t*>(&v);
+}
+// (a, b) -> hi pair, lo pair (lo = rounding residual of hi)
+__device__ __forceinline__ void split_pair(float a, float b, uint32_t& hi, uint32_t& lo) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+  const float2 hf = __bfloat1622float2(h);
+  hi = *reinterpret_cast<const uint32_t*>(&h);
+  lo = pack_bf16x2(a - hf.x, b - hf.y);
+}
+
+// Tensor-memory row of query r under the M = 64 data-path layout: 16 rows per 32-lane
+// sub-partition, in its lanes 0..15.
+__device__ __forceinline__ int row_of(int warp, int lane) { return lane < 16 ? warp * 16 + lane : -1; }
+
+#ifdef CHIMERA_ATTN_TRACE
+// per-CTA timestamps of the last launch (instrumented builds only)
+__device__ unsigned long long g_atc_trace[2048][32];
+#define TTRACE(i) g_atc_trace[(blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x][i] = global_timer_ns()
+#else
+#define TTRACE(i)
+#endif
+
+template <bool SPLIT>
+__global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_constant__ TcArgs args) {
+  const AttnParams& p = args.p;
+  constexpr int NP = SPLIT ? 4 : 2;
+  constexpr int KP = NP / 2;                 // planes of K (and of V): hi (, lo)
+  constexpr int HALF_BYTES = KP * TILE64;   // one stage of K or of V
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint8_t* q_hi = smem;                     // 64 x 128 (two atoms)
+  uint8_t* q_lo = q_hi + TILE64;
+  uint8_t* p_buf = q_lo + TILE64;           // [2 buffers][hi, lo] 64 x 64 (one atom each, 8 KB)
+  uint8_t* kbuf = p_buf + 4 * (NQ * 128);   // [STAGES][KP planes] 64 keys x 128 dims
+  uint8_t* vbuf = kbuf + STAGES * HALF_BYTES;
+  float* part = reinterpret_cast<float*>(kbuf);  // [64][PREC], reuses the KV stages after the loop
+  uint64_t* bars = reinterpret_cast<uint64_t*>(vbuf + STAGES * HALF_BYTES);
+  uint64_t* k_full = bars;           // [2] count 1 + transaction bytes (TMA)
+  uint64_t* v_full = bars + 2;       // [2] count 1 + transaction bytes (TMA)
+  uint64_t* k_empty = bars + 4;      // [2] tcgen05.commit after QK
+  uint64_t* v_empty = bars + 6;      // [2] tcgen05.commit after PV
+  uint64_t* s_full = bars + 8;       // [2] tcgen05.commit
+  uint64_t* s_free = bars + 10;      // [2] count 4 (softmax warps)
+  uint64_t* p_full = bars + 12;      // [2] count 4
+  uint64_t* pv_done = bars + 14;     // [2] tcgen05.commit
+  uint64_t* o_done = bars + 16;      // tcgen05.commit
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 17);
+  int* s_abort = reinterpret_cast<int*>(tmem_slot + 1);
+  int* s_pages = s_abort + 2;        // [PAGE_CACHE]
+  float* s_stat = reinterpret_cast<float*>(s_pages + PAGE_CACHE);  // [64][2] final (m, l)
+  volatile int* abort = s_abort;
+
+  const int s = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int S = gridDim.x;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  bf16* pool = static_cast<bf16*>(const_cast<void*>(p.pool)) + static_cast<size_t>(p.layer) * p.pool_layer_stride;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&k_full[i], 1);
+      mbar_init(&v_full[i], 1);
+      mbar_init(&k_empty[i], 1);
+      mbar_init(&v_empty[i], 1);
+      mbar_init(&s_full[i], 1);
+      mbar_init(&s_free[i], SOFT_WARPS);
+      mbar_init(&p_full[i], SOFT_WARPS);
+      mbar_init(&pv_done[i], 1);
+    }
+    mbar_init(o_done, 1);
+    *s_abort = 0;
+    mbar_fence_init();
+  }
+  if (warp == MMA_WARP) tmem_alloc(tmem_slot, TMEM_COLS);
+
+  if (threadIdx.x == 0) TTRACE(0);
+  if (!p.prewait_kv) pdl_wait();
+  const int nctx = p.n_ctx[b];
+  const int ntiles = (nctx + p.n_local + KT - 1) / KT;
+  const int tps = (ntiles + S - 1) / S;
+  const int t0 = min(ntiles, s * tps);
+  const int t1 = min(ntiles, t0 + tps);
+  const int nt = t1 - t0;
+  const bool cached = nt * 4 <= PAGE_CACHE;
+  if (cached) {
+    const int np = min(nt * 4, p.max_pages - t0 * 4);
+    for (int i = threadIdx.x; i < np; i += blockDim.x) s_pages[i] = p.page_table[b * p.max_pages + t0 * 4 + i];
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  // ---- KV staging (one thread of the loader warp): K or V of tile t into stage st as
+  // 4 pages x KP planes x 2 swizzle atoms of 16 rows; pages at or past kend are
+  // requested out of bounds (zero fill) ----
+  const bool loader = warp == SOFT_WARPS && lane == 0;
+  const long long rows_per_layer = p.pool_layer_stride / HD;
+  auto issue_half = [&](int t, int st, int kend, bool is_v) {
+    uint64_t* bar = is_v ? &v_full[st] : &k_full[st];
+    mbar_arrive_expect_tx(bar, static_cast<uint32_t>(HALF_BYTES));
+    uint8_t* base = (is_v ? vbuf : kbuf) + st * HALF_BYTES;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int kg = t * KT + u * 16;
+      long long y0 = p.pool_rows;  // out of bounds
+      if (kg < kend) {
+        const int page = cached ? s_pages[(t - t0) * 4 + u] : p.page_table[b * p.max_pages + t * 4 + u];
+        y0 = static_cast<long long>(p.layer) * rows_per_layer + ((static_cast<long long>(page) * p.H + h) * NP +
+                                                                  (is_v ? KP : 0)) * 16;
+      }
+#pragma unroll
+      for (int plane = 0; plane < KP; ++plane) {
+        const long long y = y0 < p.pool_rows ? y0 + plane * 16 : p.pool_rows;
+#pragma unroll
+        for (int a = 0; a < 2; ++a)
+          tma_load_2d(base + plane * TILE64 + a * ATOM_ROWS64 + u * 16 * 128, &args.kv_map, a * 64,
+                      static_cast<int>(y), bar);
+      }
+    }
+  };
+
+  // L2 prefetch of tile t's page-planes (4 KB each, contiguous), ahead of the ring
+  auto prefetch_tile = [&](int t, int kend) {
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      if (t * KT + u * 16 >= kend) break;
+      const int page = cached ? s_pages[(t - t0) * 4 + u] : p.page_table[b * p.max_pages + t * 4 + u];
+      const bf16* src = pool + (static_cast<size_t>(page) * p.H + h) * NP * 16 * HD;
+      prefetch_l2_bulk(src, NP * 16 * HD * 2);
+    }
+  };
+  int pf = 0;  // tiles [0, pf) of the range were requested into L2
+
+  int pre = 0;  // leading tiles (K and V) requested before the dependency wait
+  if (p.prewait_kv) {
+    if (loader) {
+      prefetch_tensormap(&args.kv_map);
+      while (pre < nt && pre < STAGES && (t0 + pre + 1) * KT <= nctx) {
+        issue_half(t0 + pre, pre, nctx, false);
+        issue_half(t0 + pre, pre, nctx, true);
+        ++pre;
+      }
+      for (; pf < nt && pf < STAGES + L2_AHEAD && (t0 + pf + 1) * KT <= nctx; ++pf)
+        if (pf >= pre) prefetch_tile(t0 + pf, nctx);
+    }
+    pdl_wait();
+  }
+  pdl_trigger();
+  if (threadIdx.x == 0) TTRACE(1);
+
+  const int nloc = min(p.n_local_dev ? p.n_local_dev[b] : p.n_local, p.n_local);
+  const int nq = p.nq_dev ? p.nq_dev[b] : p.nq;
+  const int total = nctx + nloc;
+  const int dm = p.H * HD;
+
+  // ---- queries: rotate (fused mode), split, write the swizzled Q tiles ----
+  for (int it = threadIdx.x; it < NQ * 8; it += blockDim.x) {
+    const int r = it >> 3, j = it & 7;  // row, 8-dim chunk j of the first half (dims 8j.., 64 + 8j..)
+    float lo_half[8], hi_half[8];
+    if (r < nq) {
+      const float* src = p.qkv ? p.qkv + static_cast<size_t>(b * p.q_rows + r) * p.ldqkv + h * HD + 8 * j
+                               : p.q + static_cast<size_t>(b * p.q_rows + r) * p.ldq + h * HD + 8 * j;
+      const float4 a0 = *reinterpret_cast<const float4*>(src), a1 = *reinterpret_cast<const float4*>(src + 4);
+      const float4 b0 = *reinterpret_cast<const float4*>(src + HD / 2),
+                   b1 = *reinterpret_cast<const float4*>(src + HD / 2 + 4);
+      const float x1[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+      const float x2[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+      if (p.qkv) {
+        const int pos = min(max(nctx + p.pos_base + (p.pos_off ? p.pos_off[r] : r), 0), p.max_pos - 1);
+        const float2* tab = p.rope + static_cast<size_t>(pos) * (HD / 2) + 8 * j;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float2 cs = tab[e];
+          lo_half[e] = x1[e] * cs.x - x2[e] * cs.y;
+          hi_half[e] = x2[e] * cs.x + x1[e] * cs.y;
+        }
+      } else {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          lo_half[e] = x1[e];
+          hi_half[e] = x2[e];
+        }
+      }
+    } else {
+#pragma unroll
+      for (int e = 0; e < 8; ++e) lo_half[e] = hi_half[e] = 0.f;
+    }
+    uint4 h0, l0, h1, l1;
+    split_pair(lo_half[0], lo_half[1], h0.x, l0.x);
+    split_pair(lo_half[2], lo_half[3], h0.y, l0.y);
+    split_pair(lo_half[4], lo_half[5], h0.z, l0.z);
+    split_pair(lo_half[6], lo_half[7], h0.w, l0.w);
+    split_pair(hi_half[0], hi_half[1], h1.x, l1.x);
+    split_pair(hi_half[2], hi_half[3], h1.y, l1.y);
+    split_pair(hi_half[4], hi_half[5], h1.z, l1.z);
+    split_pair(hi_half[6], hi_half[7], h1.w, l1.w);
+    *reinterpret_cast<uint4*>(q_hi + swz(r, j)) = h0;
+    *reinterpret_cast<uint4*>(q_lo + swz(r, j)) = l0;
+    *reinterpret_cast<uint4*>(q_hi + ATOM_ROWS64 + swz(r, j)) = h1;
+    *reinterpret_cast<uint4*>(q_lo + ATOM_ROWS64 + swz(r, j)) = l1;
+  }
+  // the P tiles' rows are all rewritten every tile; nothing else to clear
+
+  // ---- fresh local rows of this CTA's key range: rotate k, write k and v to the pool ----
+  if (p.qkv) {
+    const int fresh0 = nctx + p.q_local0;
+    const int f0 = max(0, t0 * KT - fresh0), f1 = min(nq, t1 * KT - fresh0);
+    for (int it = threadIdx.x; it < (f1 - f0) * 16; it += blockDim.x) {
+      const int i = f0 + (it >> 4), j = (it & 15) * 4;
+      const int slot = fresh0 + i;
+      const int pos = nctx + p.pos_base + (p.pos_off ? p.pos_off[i] : i);
+      if (pos < 0 || pos >= p.max_pos || (slot >> 4) >= p.max_pages) {
+        if (p.err) atomicOr(p.err, ERR_CAPACITY);
+        continue;
+      }
+      const int page = p.page_table[b * p.max_pages + (slot >> 4)];
+      const float* src = p.qkv + static_cast<size_t>(b * p.q_rows + i) * p.ldqkv + h * HD + j;
+      const float4 k1 = *reinterpret_cast<const float4*>(src + dm);
+      const float4 k2 = *reinterpret_cast<const float4*>(src + dm + HD / 2);
+      const float4 v1 = *reinterpret_cast<const float4*>(src + 2 * dm);
+      const float4 v2 = *reinterpret_cast<const float4*>(src + 2 * dm + HD / 2);
+      const float2* tab = p.rope + static_cast<size_t>(pos) * (HD / 2) + j;
+      const float4 cs01 = *reinterpret_cast<const float4*>(tab);
+      const float4 cs23 = *reinterpret_cast<const float4*>(tab + 2);
+      const float4 c = make_float4(cs01.x, cs01.z, cs23.x, cs23.z);
+      const float4 sn = make_float4(cs01.y, cs01.w, cs23.y, cs23.w);
+      const float4 ka = rot_lo(k1, k2, c, sn), kb = rot_hi(k1, k2, c, sn);
+      bf16* base = pool + (static_cast<size_t>(page) * p.H + h) * NP * 16 * HD + (slot & 15) * HD + j;
+      constexpr size_t plane = 16 * HD;
+      if (SPLIT) {
+        store4_split(base, base + plane, ka);
+        store4_split(base + HD / 2, base + plane + HD / 2, kb);
+        store4_split(base + 2 * plane, base + 3 * plane, v1);
+        store4_split(base + 2 * plane + HD / 2, base + 3 * plane + HD / 2, v2);
+      } else {
+        store4<bf16>(base, ka);
+        store4<bf16>(base + HD / 2, kb);
+        store4<bf16>(base + plane, v1);
+        store4<bf16>(base + plane + HD / 2, v2);
+      }
+    }
+    fence_async_global();  // the rows are read back by TMA (async proxy)
+  }
+  fence_async_smem();  // the Q tiles are read by the tensor cores (async proxy)
+  __threadfence_block();
+  __syncthreads();
+  if (threadIdx.x == 0) TTRACE(2);
+
+  if (warp == SOFT_WARPS) {
+    // ---------------- KV loader (lane 0; the other lanes idle) ----------------
+   if (loader) {
+    if (!p.prewait_kv) prefetch_tensormap(&args.kv_map);
+    // K of tile j needs the QK product of tile j - 2 done, V of tile j the PV product
+    // of tile j - 2; both are polled so that neither waits behind the other
+    int nk = pre, nv = pre;
+    uint64_t last_progress = global_timer_ns();
+    while ((nk < nt || nv < nt) && !*abort) {
+      bool moved = false;
+      if (nk < nt && (nk < STAGES || mbar_try_wait(&k_empty[nk & 1], ((nk - STAGES) >> 1) & 1))) {
+        issue_half(t0 + nk, nk & 1, total, false);
+        for (pf = max(pf, nk + 1); pf < nt && pf <= nk + L2_AHEAD; ++pf) prefetch_tile(t0 + pf, total);
+        ++nk;
+        moved = true;
+      }
+      if (nv < nk && (nv < STAGES || mbar_try_wait(&v_empty[nv & 1], ((nv - STAGES) >> 1) & 1))) {
+        issue_half(t0 + nv, nv & 1, total, true);
+        ++nv;
+        moved = true;
+      }
+      if (moved) {
+        last_progress = global_timer_ns();
+      } else if (global_timer_ns() - last_progress > 2000000000ull) {
+        *abort = 1;
+      }
+    }
+    // copies still in flight when the CTA gives up: let them land before it exits
+    if (*abort) {
+      for (int j = nk - 1; j >= 0 && j >= nk - STAGES; --j) mbar_wait_plain(&k_full[j & 1], (j >> 1) & 1, 200000000ull);
+      for (int j = nv - 1; j >= 0 && j >= nv - STAGES; --j) mbar_wait_plain(&v_full[j & 1], (j >> 1) & 1, 200000000ull);
+    }
+   }
+  } else if (warp == MMA_WARP) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0 && nt > 0) {
+      const uint32_t id_qk = idesc_f16(NQ, KT, false);
+      const uint32_t id_pv = idesc_f16(NQ, HD, true);
+      const uint32_t qh = smem_u32(q_hi), ql = smem_u32(q_lo);
+      auto pv = [&](int i) {  // O += P_i V_i
+        const int st = i & 1;
+        const uint32_t ph = smem_u32(p_buf + (2 * (i & 1)) * (NQ * 128));
+        const uint32_t pl = ph + NQ * 128;
+        const uint32_t vh = smem_u32(vbuf + st * HALF_BYTES);
+        const uint32_t vl = vh + TILE64;
+        const uint32_t o_t = tmem + 128;
+#pragma unroll
+        for (int ks = 0; ks < KT / 16; ++ks) {
+          const uint64_t a_h = desc_sw128(ph + ks * 32, 16, 1024), a_l = desc_sw128(pl + ks * 32, 16, 1024);
+          // V as MN-major B: 64-dim atoms 8 KB apart (leading), 8-key groups 1 KB apart
+          const uint64_t b_h = desc_sw128(vh + ks * 2048, ATOM_ROWS64, 1024);
+          tc_mma_bf16(o_t, a_h, b_h, id_pv, (i > 0 || ks > 0) ? 1u : 0u);
+          tc_mma_bf16(o_t, a_l, b_h, id_pv, 1u);
+          if (SPLIT) tc_mma_bf16(o_t, a_h, desc_sw128(vl + ks * 2048, ATOM_ROWS64, 1024), id_pv, 1u);
+        }
+        tc_commit(&pv_done[i & 1]);
+        tc_commit(&v_empty[st]);
+      };
+      auto qk = [&](int i) {  // S_i = Q K_i^T into S buffer i & 1
+        const int st = i & 1;
+        const uint32_t kh = smem_u32(kbuf + st * HALF_BYTES);
+        const uint32_t kl = kh + TILE64;
+        const uint32_t s_t = tmem + st * 64;
+#pragma unroll
+        for (int ks = 0; ks < HD / 16; ++ks) {
+          const uint32_t off = (ks >> 2) * ATOM_ROWS64 + (ks & 3) * 32;
+          const uint64_t a_h = desc_sw128(qh + off, 16, 1024), a_l = desc_sw128(ql + off, 16, 1024);
+          const uint64_t b_h = desc_sw128(kh + off, 16, 1024);
+          tc_mma_bf16(s_t, a_h, b_h, id_qk, ks > 0 ? 1u : 0u);
+          tc_mma_bf16(s_t, a_l, b_h, id_qk, 1u);
+          if (SPLIT) tc_mma_bf16(s_t, a_h, desc_sw128(kl + off, 16, 1024), id_qk, 1u);
+        }
+        tc_commit(&s_full[st]);
+        tc_commit(&k_empty[st]);
+      };
+      // issue whichever product is ready: PV(np) when P and V of tile np are in, QK(nq)
+      // when K is in, its S buffer is free and it runs at most one tile ahead of the PV
+      // products (so no barrier is ever two phases ahead of its waiter)
+      int nqk = 0, npv = 0;
+      uint64_t last_progress = global_timer_ns();
+      while (npv < nt && !*abort) {
+        bool moved = false;
+        if (npv < nqk && mbar_try_wait(&p_full[npv & 1], (npv >> 1) & 1) &&
+            mbar_try_wait(&v_full[npv & 1], (npv >> 1) & 1)) {
+          tc_fence_after();
+          if (npv == 10) TTRACE(22);
+          pv(npv);
+          ++npv;
+          moved = true;
+        }
+        if (nqk < nt && nqk <= npv + 1 && mbar_try_wait(&k_full[nqk & 1], (nqk >> 1) & 1) &&
+            (nqk < 2 || mbar_try_wait(&s_free[nqk & 1], ((nqk - 2) >> 1) & 1))) {
+          tc_fence_after();
+          if (nqk == 0) TTRACE(5);
+          if (nqk == 10) TTRACE(19);
+          qk(nqk);
+          ++nqk;
+          moved = true;
+        }
+        if (moved) {
+          last_progress = global_timer_ns();
+        } else if (global_timer_ns() - last_progress > 2000000000ull) {
+          *abort = 1;
+        }
+      }
+      tc_commit(o_done);  // all MMAs issued by this thread, including any after an abort
+      // tensor memory and the KV stages are released only after every MMA completed
+      mbar_wait_plain(o_done, 0, 200000000ull);
+    }
+  } else {
+    // ---------------- softmax (warps 0..3) ----------------
+    const int r = row_of(warp, lane);
+    const bool live = r >= 0 && r < nq;
+    const unsigned long long anc = live ? p.anc[p.q_local0 + r] : 0ull;
+    const float scale2 = p.scale * 1.4426950408889634f;  // softmax in base 2: exp(x) = 2^(x log2 e)
+    float m_used = -INFINITY, l = 0.f;
+    for (int t = t0; t < t1; ++t) {
+      const int i = t - t0, sb = i & 1;
+      bool ok = mbar_wait(&s_full[sb], (i >> 1) & 1, abort);
+      if (!__all_sync(0xffffffffu, ok)) break;
+      tc_fence_after();
+      if (warp == 0 && lane == 0 && i == 0) TTRACE(6);
+      if (warp == 0 && lane == 0 && i == 1) TTRACE(13);
+      if (warp == 0 && lane == 0 && i == 10) TTRACE(20);
+      float sv[KT];
+      {
+        uint32_t rr[64];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) tmem_ld16_issue(tmem + (static_cast<uint32_t>(warp * 32) << 16) + sb * 64 + 16 * j, rr + 16 * j);
+        tmem_wait_ld64(rr);
+#pragma unroll
+        for (int j = 0; j < KT; ++j) sv[j] = __uint_as_float(rr[j]);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s_free[sb]);
+      if (warp == 0 && lane == 0 && i == 0) TTRACE(8);
+      // visibility of the tile's keys for this row (bit j: key 64t + j): committed keys,
+      // then local keys whose ancestor bit is set, cut at the sequence's end
+      unsigned long long vmask = 0ull;
+      if (live) {
+        const int base = t * KT;
+        const int nc = nctx - base, nv = total - base, off = base - nctx;
+        const unsigned long long cm = nc >= 64 ? ~0ull : (nc <= 0 ? 0ull : ((1ull << nc) - 1ull));
+        const unsigned long long lm = off >= 0 ? (off < 64 ? (anc >> off) : 0ull) : (-off < 64 ? (anc << -off) : 0ull);
+        const unsigned long long vm = nv >= 64 ? ~0ull : (nv <= 0 ? 0ull : ((1ull << nv) - 1ull));
+        vmask = (cm | lm) & vm;
+      }
+      // scores in log2 units, tile maximum
+      float tmax = -INFINITY;
+#pragma unroll
+      for (int j = 0; j < KT; ++j) {
+        sv[j] = ((vmask >> j) & 1ull) ? sv[j] * scale2 : -INFINITY;
+        tmax = fmaxf(tmax, sv[j]);
+      }
+      // this tile's P buffer was read by the PV product of tile i - 2
+      if (i >= 2) {
+        ok = mbar_wait(&pv_done[i & 1], ((i - 2) >> 1) & 1, abort);
+        if (!__all_sync(0xffffffffu, ok)) break;
+        tc_fence_after();
+      }
+      if (warp == 0 && lane == 0 && i == 10) TTRACE(23);
+      const bool raise = tmax > m_used + RESCALE_LOG2 || (m_used == -INFINITY && tmax > -INFINITY);
+      float corr = 1.f;
+      if (raise) {
+        corr = (m_used == -INFINITY) ? 0.f : exp2f(m_used - tmax);
+        m_used = tmax;
+      }
+      if (__any_sync(0xffffffffu, raise && corr != 0.f && l > 0.f) && i > 0) {
+        // O holds the products up to tile i - 1: wait for the last one before rescaling
+        ok = mbar_wait(&pv_done[(i - 1) & 1], ((i - 1) >> 1) & 1, abort);
+        if (!__all_sync(0xffffffffu, ok)) break;
+        tc_fence_after();
+        // rescale this warp's O rows in tensor memory (factor 1 for rows that kept m)
+        const float f = (raise && l > 0.f) ? corr : 1.f;
+#pragma unroll
+        for (int c0 = 0; c0 < HD; c0 += 64) {
+          uint32_t rr[64];
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            tmem_ld16_issue(tmem + (static_cast<uint32_t>(warp * 32) << 16) + 128 + c0 + 16 * j, rr + 16 * j);
+          tmem_wait_ld64(rr);
+#pragma unroll
+          for (int j = 0; j < 64; ++j) rr[j] = __float_as_uint(__uint_as_float(rr[j]) * f);
+#pragma unroll
+          for (int j = 0; j < 4; ++j) tmem_st16(tmem + (static_cast<uint32_t>(warp * 32) << 16) + 128 + c0 + 16 * j, rr + 16 * j);
+        }
+        tmem_wait_st();
+      }
+      l *= corr;
+      // P = exp(S - m), two-term split into the swizzled P tile of this tile
+      uint8_t* ph = p_buf + (2 * sb) * (NQ * 128);
+      uint8_t* pl = ph + NQ * 128;
+      float rsum = 0.f;
+#pragma unroll
+      for (int c = 0; c < 8; ++c) {
+        float pv8[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float x = sv[8 * c + e];
+          pv8[e] = (x == -INFINITY) ? 0.f : exp2f(x - m_used);
+          rsum += pv8[e];
+        }
+        uint4 hh, ll;
+        split_pair(pv8[0], pv8[1], hh.x, ll.x);
+        split_pair(pv8[2], pv8[3], hh.y, ll.y);
+        split_pair(pv8[4], pv8[5], hh.z, ll.z);
+        split_pair(pv8[6], pv8[7], hh.w, ll.w);
+        if (r >= 0) {
+          *reinterpret_cast<uint4*>(ph + swz(r, c)) = hh;
+          *reinterpret_cast<uint4*>(pl + swz(r, c)) = ll;
+        }
+      }
+      l += rsum;
+      if (warp == 0 && lane == 0 && i == 0) TTRACE(15);
+      if (warp == 0 && lane == 0 && i == 10) TTRACE(21);
+      fence_async_smem();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&p_full[sb]);
+      if (warp == 0 && lane == 0 && i == 0) TTRACE(7);
+      if (warp == 0 && lane == 0 && i == nt - 1) TTRACE(14);
+    }
+    if (r >= 0) {
+      s_stat[2 * r] = m_used;
+      s_stat[2 * r + 1] = l;
+    }
+  }
+
+  // ---- epilogue: wait for the last PV product, publish the partial rows ----
+  if (warp < SOFT_WARPS) {
+    bool ok = true;
+    if (nt > 0) {
+      ok = mbar_wait(o_done, 0, abort);
+      tc_fence_after();
+    }
+    if (warp == 0 && lane == 0) TTRACE(9);
+    __syncwarp();
+  }
+  __syncthreads();  // KV stages are free: every load landed and every MMA completed
+  if (warp < SOFT_WARPS) {
+    const int r = row_of(warp, lane);
+    const bool have = nt > 0 && !*abort;
+#pragma unroll
+    for (int c0 = 0; c0 < HD; c0 += 64) {
+      uint32_t rr[64];
+      if (have) {
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          tmem_ld16_issue(tmem + (static_cast<uint32_t>(warp * 32) << 16) + 128 + c0 + 16 * j, rr + 16 * j);
+        tmem_wait_ld64(rr);
+      }
+      if (r >= 0 && r < nq) {
+        float* w = part + r * PREC + c0;
+        const float ll = s_stat[2 * r + 1];
+#pragma unroll
+        for (int j = 0; j < 64; j += 4) {
+          float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+          if (have && ll > 0.f)
+            v = make_float4(__uint_as_float(rr[j]), __uint_as_float(rr[j + 1]), __uint_as_float(rr[j + 2]),
+                            __uint_as_float(rr[j + 3]));
+          *reinterpret_cast<float4*>(w + j) = v;
+        }
+      }
+    }
+    if (r >= 0 && r < nq) {
+      part[r * PREC + HD] = (nt > 0) ? s_stat[2 * r] : -INFINITY;
+      part[r * PREC + HD + 1] = (nt > 0) ? s_stat[2 * r + 1] : 0.f;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  __syncwarp();
+  if (warp == MMA_WARP) {
+    tc_fence_after();
+    tmem_dealloc(tmem, TMEM_COLS);
+  }
+  if (threadIdx.x == 0 && *abort && p.err) atomicOr(p.err, ERR_TIMEOUT);
+
+  bf16* out = static_cast<bf16*>(p.out);
+  bf16* out_lo = static_cast<bf16*>(p.out_lo);
+  __syncwarp();
+  if (S > 1) cluster_sync();
+  {
+    const int rpc = (nq + S - 1) / S;
+    const int q0 = s * rpc, q1 = min(nq, q0 + rpc);
+    const uint32_t part_u32 = smem_u32(part);
+    for (int it = threadIdx.x; it < (q1 - q0) * (HD / 4); it += blockDim.x) {
+      const int qi = q0 + it / (HD / 4), c = (it % (HD / 4)) * 4;
+      float L = 0.f;
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (S == 1) {
+        L = part[qi * PREC + HD + 1];
+        acc = *reinterpret_cast<const float4*>(part + qi * PREC + c);
+      } else {
+        float mv[8], lv[8];
+        float M = -INFINITY;
+#pragma unroll
+        for (int rk = 0; rk < 8; ++rk) {
+          mv[rk] = -INFINITY;
+          lv[rk] = 0.f;
+          if (rk < S) {
+            const uint32_t a = dsmem_addr(part_u32 + static_cast<uint32_t>((qi * PREC + HD) * 4), rk);
+            mv[rk] = ld_dsmem(a);
+            lv[rk] = ld_dsmem(a + 4);
+            M = fmaxf(M, mv[rk]);
+          }
+        }
+#pragma unroll
+        for (int rk = 0; rk < 8; ++rk) {
+          if (rk < S) {
+            const float w = (M == -INFINITY || mv[rk] == -INFINITY) ? 0.f : exp2f(mv[rk] - M);
+            L += w * lv[rk];
+            const float4 v = ld_dsmem4(dsmem_addr(part_u32 + static_cast<uint32_t>((qi * PREC + c) * 4), rk));
+            acc.x += w * v.x; acc.y += w * v.y; acc.z += w * v.z; acc.w += w * v.w;
+          }
+        }
+      }
+      const float inv = L > 0.f ? 1.f / L : 0.f;
+      const size_t o_idx = static_cast<size_t>(b * p.q_rows + qi) * p.ldo + h * HD + c;
+      store_act(out, out_lo, o_idx, acc.x * inv);
+      store_act(out, out_lo, o_idx + 1, acc.y * inv);
+      store_act(out, out_lo, o_idx + 2, acc.z * inv);
+      store_act(out, out_lo, o_idx + 3, acc.w * inv);
+    }
+  }
+  __syncwarp();
+  if (S > 1) cluster_sync();  // peers may read this CTA's partials until here
+  if (threadIdx.x == 0) TTRACE(10);
+}
+
+template <bool SPLIT>
+size_t tc_smem() {
+  const size_t np = SPLIT ? 4 : 2;
+  return 1024 + 2 * TILE64 + 4 * NQ * 128 + STAGES * np * TILE64 + 18 * 8 + 16 + PAGE_CACHE * 4 + 2 * NQ * 4;
+}
+
+template <bool SPLIT>
+void tc_attr() {
+  static bool done = false;
+  if (!done) {
+    cudaFuncSetAttribute(attn_tc_kernel<SPLIT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         static_cast<int>(tc_smem<SPLIT>()));
+    done = true;
+  }
+}
+
+template <bool SPLIT>
+cudaError_t launch_tc(const AttnParams& p, cudaStream_t s) {
+  tc_attr<SPLIT>();
+  TcArgs args;
+  memset(&args, 0, sizeof(args));
+  args.p = p;
+  if (encode_2d_bf16(&args.kv_map, p.pool, HD, static_cast<uint64_t>(p.pool_rows), HD, 64, 16) != 0)
+    return cudaErrorInvalidValue;
+  cudaLaunchAttribute at[2];
+  int na = 0;
+  at[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[na].val.programmaticStreamSerializationAllowed = 1;
+  ++na;
+  if (p.splits > 1) {
+    at[na].id = cudaLaunchAttributeClusterDimension;
+    at[na].val.clusterDim.x = p.splits;
+    at[na].val.clusterDim.y = 1;
+    at[na].val.clusterDim.z = 1;
+    ++na;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.splits, p.H, p.B);
+  cfg.blockDim = dim3(THREADS);
+  cfg.dynamicSmemBytes = tc_smem<SPLIT>();
+  cfg.stream = s;
+  cfg.attrs = at;
+  cfg.numAttrs = na;
+  cudaLaunchKernelEx(&cfg, attn_tc_kernel<SPLIT>, args);
+  return cudaGetLastError();
+}
+
+template <bool SPLIT>
+int tc_splits(int BH, int want) {
+  tc_attr<SPLIT>();
+  int S = std::max(1, std::min(8, want));
+  for (; S > 1; --S) {
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = S;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(S, BH, 1);
+    cfg.blockDim = dim3(THREADS);
+    cfg.dynamicSmemBytes = tc_smem<SPLIT>();
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, attn_tc_kernel<SPLIT>, &cfg) == cudaSuccess && n >= BH) break;
+    cudaGetLastError();
+  }
+  return S;
+}
+
+}  // namespace
+
+#ifdef CHIMERA_ATTN_TRACE
+extern "C" int chimera_atc_trace(unsigned long long* host, int n) {
+  return cudaMemcpyFromSymbol(host, g_atc_trace, static_cast<size_t>(n) * 32 * 8) == cudaSuccess ? 0 : -1;
+}
+#endif
+
+cudaError_t attention_tc(const AttnParams& p, cudaStream_t s) {
+  if (p.hd != HD || p.nq_max > NQ || p.n_local > 64 || p.splits < 1 || p.splits > 8) return cudaErrorInvalidValue;
+  // the TMA row coordinate is a 32-bit integer; the pool base must be 16-byte aligned
+  if (p.pool_rows < 16 || p.pool_rows >= (1ll << 31) || (reinterpret_cast<uintptr_t>(p.pool) & 15))
+    return cudaErrorInvalidValue;
+  if (p.planes != 2 && p.planes != 4) return cudaErrorInvalidValue;
+  if (p.qkv && (!p.rope || !p.err || p.max_pos < 1 || (p.ldqkv & 3))) return cudaErrorInvalidValue;
+  if (!p.qkv && (p.ldq & 3)) return cudaErrorInvalidValue;
+  return p.planes == 4 ? launch_tc<true>(p, s) : launch_tc<false>(p, s);
+}
+
+int attention_tc_splits(int planes, int BH, int want) {
+  return planes == 4 ? tc_splits<true>(BH, want) : tc_splits<false>(BH, want);
+}
+
+}  // namespace chimera

@@ -77,6 +77,7 @@ struct AttnParams {
   const int* n_local_dev; // optional per-sequence local count
   const unsigned long long* anc;  // [q_local0 + nq] ancestor-or-self masks over local rows
   const void* pool;       // [blocks][H][planes][16][hd], element type of the model
+  long long pool_rows;    // 16-row page rows in the whole allocation (layers x blocks x H x planes x 16)
   int planes;             // 2: K, V;  4: K_hi, K_lo, V_hi, V_lo (bf16 two-term split)
   long long pool_layer_stride;  // elements between layers (0 for the draft pool)
   int layer;
@@ -117,6 +118,13 @@ size_t attn_ws_floats(int B, int H, int splits, int nq_max, int hd);
 // `want` and 8 (one thread-block cluster per (b, h)), reduced until all B * H clusters
 // are resident at once.  Other paths return `want` unchanged.
 int attn_pick_splits(int dtype, int hd, int planes, int B, int H, int want);
+// 2D bf16 tensor map (128-byte swizzle, zero fill out of bounds) of a row-major matrix
+// [outer][pitch_elems] with an inner extent of `inner` elements; 0 on success.
+int encode_2d_bf16(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer, uint64_t pitch_elems,
+                   uint32_t box_inner, uint32_t box_outer);
+// Tensor-core tree attention (bf16 planes, head_dim 128; splits <= 8 form one cluster).
+cudaError_t attention_tc(const AttnParams& p, cudaStream_t s);
+int attention_tc_splits(int planes, int BH, int want);
 // True when attention() fuses RoPE and the KV write (qkv given) for this model.
 bool attn_fuses_rope(int dtype, int hd);
 

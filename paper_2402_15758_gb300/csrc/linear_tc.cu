@@ -131,13 +131,6 @@ __device__ __forceinline__ bool bar_any(int id, int nthreads, bool pred) {
   return r != 0;
 }
 
-__device__ __forceinline__ bool mbar_wait_plain(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
-  const uint64_t t0 = global_timer_ns();
-  while (!mbar_try_wait(bar, parity)) {
-    if (global_timer_ns() - t0 > limit_ns) return false;
-  }
-  return true;
-}
 
 __global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const __grid_constant__ TcLinearParams p) {
   extern __shared__ uint8_t smem_raw[];
@@ -450,6 +443,8 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
+}  // namespace
+
 int encode_2d_bf16(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
                    uint64_t pitch_elems, uint32_t box_inner, uint32_t box_outer) {
   EncodeTiledFn fn = encode_fn();
@@ -463,6 +458,8 @@ int encode_2d_bf16(CUtensorMap* map, const void* base, uint64_t inner, uint64_t 
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS ? 0 : -2;
 }
+
+namespace {
 
 uint32_t pow2ceil(uint32_t v) {
   uint32_t r = 1;

@@ -376,6 +376,7 @@ cudaError_t run_attention(chimera_ctx* ctx, bool draft_pool, int layer, int nq, 
   p.pool = draft_pool ? ctx->dkv : ctx->kv;
   p.planes = ctx->kv_planes;
   p.pool_layer_stride = draft_pool ? 0 : ctx->kv_layer_stride;
+  p.pool_rows = static_cast<long long>(draft_pool ? 1 : ctx->L) * ctx->NB * ctx->H * ctx->kv_planes * 16;
   p.layer = draft_pool ? 0 : layer;
   p.page_table = ctx->d_pt;
   p.max_pages = ctx->max_pages;
@@ -1348,12 +1349,13 @@ chimera_status chimera_op_linear(int dtype, int epi, int out_f32, int M, int N, 
 }
 
 chimera_status chimera_op_attention(int dtype, int kv_split, int batch, int n_heads, int head_dim, int nq, int q_local0,
-                                    int n_local, const float* q, int ldq, int q_rows, const void* pool,
+                                    int n_local, const float* q, int ldq, int q_rows, const void* pool, int n_blocks,
                                     const int32_t* page_table, int max_pages, const int32_t* n_ctx, const uint64_t* anc,
                                     void* out, void* out_lo, int ldo, int splits, void* cuda_stream) {
   if ((dtype != 0 && dtype != 1) || batch < 1 || n_heads < 1 || (head_dim != 64 && head_dim != 128) || nq < 1 ||
       nq > 64 || n_local < 0 || n_local > 64 || q_local0 < 0 || !q || !pool || !page_table || !n_ctx || !anc || !out ||
-      splits < 1 || splits > 16 || (dtype == 1 && head_dim == 128 && splits > 8) || batch * n_heads > 64 * 256)
+      splits < 1 || splits > 16 || (dtype == 1 && head_dim == 128 && splits > 8) || batch * n_heads > 64 * 256 ||
+      n_blocks < 1)
     return CHIMERA_EINVAL;
   std::lock_guard<std::mutex> lk(g_op_mu);
   if (!op_scratch()) return CHIMERA_ENOMEM;
@@ -1367,6 +1369,7 @@ chimera_status chimera_op_attention(int dtype, int kv_split, int batch, int n_he
   p.anc = reinterpret_cast<const unsigned long long*>(anc);
   p.pool = pool;
   p.planes = (dtype == 1 && kv_split) ? 4 : 2;
+  p.pool_rows = static_cast<long long>(n_blocks) * n_heads * p.planes * 16;
   p.page_table = page_table;
   p.max_pages = max_pages;
   p.n_ctx = n_ctx;
