@@ -569,45 +569,64 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
     }
   }
 
-  // ---- epilogue: wait for the last PV product, publish the partial rows ----
+  // ---- epilogue: every CTA pushes its partial rows (O, m, l) to the cluster CTA that
+  // finishes them (rows [r * ceil(nq / S), ...) belong to rank r); the receive buffer
+  // reuses the KV rings, so the pushes start once every CTA of the cluster is past its
+  // main loop (split cluster barrier) ----
   if (warp < SOFT_WARPS) {
-    bool ok = true;
     if (nt > 0) {
-      ok = mbar_wait(o_done, 0, abort);
+      mbar_wait(o_done, 0, abort);
       tc_fence_after();
     }
-    if (warp == 0 && lane == 0) TTRACE(9);
     __syncwarp();
   }
-  __syncthreads();  // KV stages are free: every load landed and every MMA completed
-  if (warp < SOFT_WARPS) {
+  __syncthreads();  // this CTA's rings are idle: every load landed and every MMA completed
+  __syncwarp();
+  if (S > 1) cluster_arrive();
+  const int rpc = (nq + S - 1) / S;
+  float* recv = part;                     // [S][rpc][PREC], S * rpc <= NQ + 7 rows (37.5 KB)
+  float* s_w = part + (NQ + 8) * PREC;    // [rpc][8] merge weights, past the receive slots
+  {
     const int r = row_of(warp, lane);
-    const bool have = nt > 0 && !*abort;
+    const bool soft = warp < SOFT_WARPS;
+    const bool have = soft && nt > 0 && !*abort;
+    const bool mine = soft && r >= 0 && r < nq;
+    uint32_t rr[64];
+    if (have) {  // first 64 columns of the O row while the peers finish
 #pragma unroll
-    for (int c0 = 0; c0 < HD; c0 += 64) {
-      uint32_t rr[64];
-      if (have) {
+      for (int j = 0; j < 4; ++j) tmem_ld16_issue(tmem + (static_cast<uint32_t>(warp * 32) << 16) + 128 + 16 * j, rr + 16 * j);
+      tmem_wait_ld64(rr);
+    }
+    __syncwarp();
+    if (S > 1) cluster_wait();
+    if (soft) {
+      const int owner = mine ? r / rpc : 0;
+      const uint32_t slot = smem_u32(recv + (s * rpc + (mine ? r - owner * rpc : 0)) * PREC);
+      const uint32_t dst = S > 1 ? dsmem_addr(slot, owner) : slot;
+      const float lr = mine ? s_stat[2 * r + 1] : 0.f;
+      const bool keep = have && lr > 0.f;
 #pragma unroll
-        for (int j = 0; j < 4; ++j)
-          tmem_ld16_issue(tmem + (static_cast<uint32_t>(warp * 32) << 16) + 128 + c0 + 16 * j, rr + 16 * j);
-        tmem_wait_ld64(rr);
-      }
-      if (r >= 0 && r < nq) {
-        float* w = part + r * PREC + c0;
-        const float ll = s_stat[2 * r + 1];
+      for (int half = 0; half < 2; ++half) {
+        if (half == 1 && have) {
 #pragma unroll
-        for (int j = 0; j < 64; j += 4) {
-          float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-          if (have && ll > 0.f)
-            v = make_float4(__uint_as_float(rr[j]), __uint_as_float(rr[j + 1]), __uint_as_float(rr[j + 2]),
-                            __uint_as_float(rr[j + 3]));
-          *reinterpret_cast<float4*>(w + j) = v;
+          for (int j = 0; j < 4; ++j)
+            tmem_ld16_issue(tmem + (static_cast<uint32_t>(warp * 32) << 16) + 128 + 64 + 16 * j, rr + 16 * j);
+          tmem_wait_ld64(rr);
+        }
+        if (mine) {
+#pragma unroll
+          for (int j = 0; j < 64; j += 4) {
+            const float4 v = keep ? make_float4(__uint_as_float(rr[j]), __uint_as_float(rr[j + 1]),
+                                                __uint_as_float(rr[j + 2]), __uint_as_float(rr[j + 3]))
+                                  : make_float4(0.f, 0.f, 0.f, 0.f);
+            st_dsmem4(dst + static_cast<uint32_t>((half * 64 + j) * 4), v);
+          }
         }
       }
-    }
-    if (r >= 0 && r < nq) {
-      part[r * PREC + HD] = (nt > 0) ? s_stat[2 * r] : -INFINITY;
-      part[r * PREC + HD + 1] = (nt > 0) ? s_stat[2 * r + 1] : 0.f;
+      if (mine) {
+        st_dsmem(dst + HD * 4, nt > 0 ? s_stat[2 * r] : -INFINITY);
+        st_dsmem(dst + (HD + 1) * 4, nt > 0 ? lr : 0.f);
+      }
     }
   }
   tc_fence_before();
@@ -618,56 +637,49 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
     tmem_dealloc(tmem, TMEM_COLS);
   }
   if (threadIdx.x == 0 && *abort && p.err) atomicOr(p.err, ERR_TIMEOUT);
+  __syncwarp();
+  if (S > 1) cluster_sync();  // every push into this CTA is complete and visible
 
+  // ---- merge the S partials of this CTA's rows (local shared memory) ----
   bf16* out = static_cast<bf16*>(p.out);
   bf16* out_lo = static_cast<bf16*>(p.out_lo);
-  __syncwarp();
-  if (S > 1) cluster_sync();
-  {
-    const int rpc = (nq + S - 1) / S;
-    const int q0 = s * rpc, q1 = min(nq, q0 + rpc);
-    const uint32_t part_u32 = smem_u32(part);
-    for (int it = threadIdx.x; it < (q1 - q0) * (HD / 4); it += blockDim.x) {
-      const int qi = q0 + it / (HD / 4), c = (it % (HD / 4)) * 4;
-      float L = 0.f;
-      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (S == 1) {
-        L = part[qi * PREC + HD + 1];
-        acc = *reinterpret_cast<const float4*>(part + qi * PREC + c);
-      } else {
-        float mv[8], lv[8];
-        float M = -INFINITY;
+  const int q0 = s * rpc, nrows = max(0, min(nq, q0 + rpc) - q0);
+  for (int rl = threadIdx.x; rl < nrows; rl += blockDim.x) {
+    float mv[8], M = -INFINITY;
 #pragma unroll
-        for (int rk = 0; rk < 8; ++rk) {
-          mv[rk] = -INFINITY;
-          lv[rk] = 0.f;
-          if (rk < S) {
-            const uint32_t a = dsmem_addr(part_u32 + static_cast<uint32_t>((qi * PREC + HD) * 4), rk);
-            mv[rk] = ld_dsmem(a);
-            lv[rk] = ld_dsmem(a + 4);
-            M = fmaxf(M, mv[rk]);
-          }
-        }
-#pragma unroll
-        for (int rk = 0; rk < 8; ++rk) {
-          if (rk < S) {
-            const float w = (M == -INFINITY || mv[rk] == -INFINITY) ? 0.f : exp2f(mv[rk] - M);
-            L += w * lv[rk];
-            const float4 v = ld_dsmem4(dsmem_addr(part_u32 + static_cast<uint32_t>((qi * PREC + c) * 4), rk));
-            acc.x += w * v.x; acc.y += w * v.y; acc.z += w * v.z; acc.w += w * v.w;
-          }
-        }
-      }
-      const float inv = L > 0.f ? 1.f / L : 0.f;
-      const size_t o_idx = static_cast<size_t>(b * p.q_rows + qi) * p.ldo + h * HD + c;
-      store_act(out, out_lo, o_idx, acc.x * inv);
-      store_act(out, out_lo, o_idx + 1, acc.y * inv);
-      store_act(out, out_lo, o_idx + 2, acc.z * inv);
-      store_act(out, out_lo, o_idx + 3, acc.w * inv);
+    for (int k = 0; k < 8; ++k) {
+      mv[k] = k < S ? recv[(k * rpc + rl) * PREC + HD] : -INFINITY;
+      M = fmaxf(M, mv[k]);
     }
+    float L = 0.f;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      mv[k] = (k < S && M != -INFINITY && mv[k] != -INFINITY) ? exp2f(mv[k] - M) : 0.f;
+      if (k < S) L += mv[k] * recv[(k * rpc + rl) * PREC + HD + 1];
+    }
+    const float inv = L > 0.f ? 1.f / L : 0.f;
+#pragma unroll
+    for (int k = 0; k < 8; ++k)
+      if (k < S) s_w[rl * 8 + k] = mv[k] * inv;
   }
-  __syncwarp();
-  if (S > 1) cluster_sync();  // peers may read this CTA's partials until here
+  __syncthreads();
+  for (int it = threadIdx.x; it < nrows * (HD / 4); it += blockDim.x) {
+    const int rl = it / (HD / 4), c = (it % (HD / 4)) * 4;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      if (k < S) {
+        const float w = s_w[rl * 8 + k];
+        const float4 v = *reinterpret_cast<const float4*>(recv + (k * rpc + rl) * PREC + c);
+        acc.x += w * v.x; acc.y += w * v.y; acc.z += w * v.z; acc.w += w * v.w;
+      }
+    }
+    const size_t o_idx = static_cast<size_t>(b * p.q_rows + q0 + rl) * p.ldo + h * HD + c;
+    store_act(out, out_lo, o_idx, acc.x);
+    store_act(out, out_lo, o_idx + 1, acc.y);
+    store_act(out, out_lo, o_idx + 2, acc.z);
+    store_act(out, out_lo, o_idx + 3, acc.w);
+  }
   if (threadIdx.x == 0) TTRACE(10);
 }
 
