@@ -105,7 +105,17 @@ def _run_sampled(name, n_steps, forced, sample, cap, prompt_len=None):
             roots[b] = st.tokens[st.n]
         ctx.set_root(roots)
     rng = np.random.default_rng(7)
+    diverged = False
     for step in range(n_steps):
+        if diverged:  # a near-tie made the GPU commit other tokens: restart from the oracle's
+            gt, gn = ctx.read("tokens"), ctx.read("n")
+            ctx.prefill([states[b].tokens[: states[b].n] if b in states else gt[b, : gn[b]].tolist()
+                         for b in range(B)])
+            roots = [int(t) for t in ctx.read("tokens")[np.arange(B), ctx.read("n").astype(np.int64)]]
+            for b, st in states.items():
+                roots[b] = st.tokens[st.n]
+            ctx.set_root(roots)
+            diverged = False
         toks_all, drafts = [], {}
         for b in range(B):
             if b in states:
@@ -156,6 +166,7 @@ def _run_sampled(name, n_steps, forced, sample, cap, prompt_len=None):
                     assert rel_rows(v_g, ver["v"][layer][path]) <= tol
             else:
                 assert f > 0, "accepted path differs without a near-tie"
+                diverged = True
             co.commit(W, cfg, st, toks_all[b], ver, path, bonus)
         roots = [int(t) for t in ctx.read("tokens")[np.arange(B), ctx.read("n").astype(np.int64)]]
         if states:
