@@ -34,6 +34,10 @@ struct TcLinearParams {
   uint32_t tmem_cols;
   uint32_t acc_stride;  // TMEM column distance between the two accumulators
   int trace_id;         // call-site id (used by instrumented builds only)
+  // optional: [zero, zero + zero_floats) cleared by the epilogue warps after the
+  // dependency wait, spread over the CTAs (a later linear's fp32 accumulator)
+  float* zero;
+  long long zero_floats;
 };
 
 struct TcLinearPlan {
@@ -55,7 +59,8 @@ int tc_max_tiles();
 // launch for two projections of the same input, e.g. SwiGLU gate and up); needs N % 128 == 0.
 int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, const void* X_lo, int ldx,
                    const void* W, void* Y, void* Y_lo, int ldy, int epi, int out_f32, float* ws,
-                   int* counters, int* err, char* msg, size_t msg_len, const void* W2 = nullptr, int N2 = 0);
+                   int* counters, int* err, char* msg, size_t msg_len, const void* W2 = nullptr, int N2 = 0,
+                   float* zero = nullptr, long long zero_floats = 0);
 cudaError_t tc_linear_launch(const TcLinearPlan& plan, cudaStream_t s);
 
 // ----------------------------------------------------------------------------

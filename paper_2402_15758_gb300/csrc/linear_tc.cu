@@ -315,6 +315,12 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const _
     // ---------------- epilogue (warps 2..5, TMEM lanes 32*(warp%4) ..) ----------------
     pdl_wait();  // Y, the split workspace and the counters are shared with earlier kernels
     pdl_trigger();
+    if (p.zero) {  // this CTA's share (float4s) of a later linear's accumulator
+      const long long n4 = p.zero_floats / 4, per = (n4 + G - 1) / G;
+      float4* z = reinterpret_cast<float4*>(p.zero);
+      for (long long i = cta * per + (threadIdx.x - 64); i < min(n4, (cta + 1) * per); i += 128)
+        z[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
     const int q = warp & 3;
     const int row = q * 32 + lane;
     int buf = 0;
@@ -507,7 +513,8 @@ extern "C" int chimera_lin_trace(unsigned long long* host, int ctas) {
 
 int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, const void* X_lo, int ldx,
                    const void* W, void* Y, void* Y_lo, int ldy, int epi, int out_f32, float* ws,
-                   int* counters, int* err, char* msg, size_t msg_len, const void* W2, int N2) {
+                   int* counters, int* err, char* msg, size_t msg_len, const void* W2, int N2,
+                   float* zero, long long zero_floats) {
   auto fail = [&](const char* m) {
     if (msg && msg_len) snprintf(msg, msg_len, "linear(M=%d,N=%d,K=%d): %s", M, N, K, m);
     return -1;
@@ -519,6 +526,8 @@ int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, const
       (reinterpret_cast<uintptr_t>(X_lo) & 15))
     return fail("X, X_lo and W must be 16-byte aligned");
   if (epi == EPI_RESID && !out_f32) return fail("accumulating epilogue needs an fp32 output");
+  if (zero && ((zero_floats & 3) || (reinterpret_cast<uintptr_t>(zero) & 15)))
+    return fail("the buffer to clear must be 16-byte aligned and a multiple of 4 floats");
   if (W2 && (N % BM != 0 || N2 < 1 || (reinterpret_cast<uintptr_t>(W2) & 15)))
     return fail("second weight needs N % 128 == 0 and a 16-byte aligned W2");
   const int N1 = N;
@@ -551,6 +560,8 @@ int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, const
   p.Y = Y;
   p.Y2 = out_f32 ? nullptr : Y_lo;
   p.ldy = ldy;
+  p.zero = zero;
+  p.zero_floats = zero ? zero_floats : 0;
   p.ws = ws;
   p.counters = counters;
   p.err = err;

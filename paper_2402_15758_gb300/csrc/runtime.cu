@@ -196,6 +196,7 @@ struct chimera_ctx {
   void *tbuf = nullptr, *ubuf = nullptr, *ubuf_lo = nullptr, *headin = nullptr, *headin_lo = nullptr;
   float *hfull_log = nullptr, *hsel = nullptr, *kvtmp = nullptr;
   float *dres = nullptr, *hlog = nullptr;
+  bool tc_zero = false;  // tensor-core linears clear the next accumulators (see enqueue_layer)
 
   // scratch of the split kernels
   float* lin_ws = nullptr;
@@ -304,7 +305,7 @@ cudaError_t run_lin(chimera_ctx* ctx, const Lin& l) {
 
 bool make_lin(chimera_ctx* ctx, Lin* l, int M, int N, int K, const void* X, const void* X_lo, int ldx,
               const void* W, void* Y, void* Y_lo, int ldy, int epi, int out_f32, const void* W2 = nullptr,
-              int N2 = 0) {
+              int N2 = 0, float* zero = nullptr, long long zero_floats = 0) {
   l->M = M;
   l->N = N;
   l->K = K;
@@ -322,7 +323,7 @@ bool make_lin(chimera_ctx* ctx, Lin* l, int M, int N, int K, const void* X, cons
   if (!l->tc) return true;
   char msg[256];
   if (tc_linear_plan(&l->tp, M, N, K, X, X_lo, ldx, W, Y, Y_lo, ldy, epi, out_f32, ctx->lin_ws, ctx->lin_cnt,
-                     ctx->d_err, msg, sizeof(msg), W2, N2) != 0) {
+                     ctx->d_err, msg, sizeof(msg), W2, N2, zero, zero_floats) != 0) {
     ctx->err = msg;
     return false;
   }
@@ -461,7 +462,10 @@ cudaError_t enqueue_layer(chimera_ctx* ctx, int l, const Lin* lin, int rows, int
                           const int* pos_off, const unsigned long long* anc, int splits, double kv_bytes) {
   const chimera_block_weights& w = ctx->layers[l];
   const int d = ctx->d;
-  RUN(run_norm(ctx, ctx->x, w.attn_norm, rows, ctx->qkv, 3 * d));
+  // the accumulators of the QKV and gate|up linears are cleared by the norms, or (tensor-
+  // core linears) by the previous layer's down linear and this layer's O linear
+  const bool z = !ctx->tc_zero;
+  RUN(run_norm(ctx, ctx->x, w.attn_norm, rows, (z || l == 0) ? ctx->qkv : nullptr, 3 * d));
   RUN(run_lin(ctx, lin[0]));
   if (attn_fuses_rope(ctx->dtype, ctx->hd)) {
     RUN(run_attention(ctx, false, l, rows_per_seq, valid, 0, rows_per_seq, valid, anc, rows_per_seq, splits,
@@ -472,7 +476,7 @@ cudaError_t enqueue_layer(chimera_ctx* ctx, int l, const Lin* lin, int rows, int
                       rows_per_seq, kv_bytes));
   }
   RUN(run_lin(ctx, lin[1]));
-  RUN(run_norm(ctx, ctx->x, w.ffn_norm, rows, ctx->gu, 2 * ctx->F));
+  RUN(run_norm(ctx, ctx->x, w.ffn_norm, rows, z ? ctx->gu : nullptr, 2 * ctx->F));
   RUN(run_lin(ctx, lin[2]));
   RUN(run_lin(ctx, lin[3]));
   {
@@ -605,12 +609,18 @@ bool build_plans(chimera_ctx* ctx, int B) {
       const chimera_block_weights& w = ctx->layers[l];
       Lin* p = &v[5 * l];
       if (!make_lin(ctx, &p[0], M, 3 * d, d, xn, xl, d, w.wqkv, ctx->qkv, nullptr, 3 * d, ACC, f32)) return false;
-      if (!make_lin(ctx, &p[1], M, d, d, ao, al, d, w.wo, ctx->x, nullptr, d, ACC, f32)) return false;
+      // the O linear clears the gate|up accumulator of this layer, the down linear the
+      // QKV accumulator of the next one (their epilogue warps, off the critical path)
+      if (!make_lin(ctx, &p[1], M, d, d, ao, al, d, w.wo, ctx->x, nullptr, d, ACC, f32, nullptr, 0,
+                    ctx->tc_zero ? ctx->gu : nullptr, static_cast<long long>(M) * 2 * F))
+        return false;
       // gate and up: one launch writing gu[:, 0:F] and gu[:, F:2F]
       if (!make_lin(ctx, &p[2], M, F, d, xn, xl, d, w.w_gate, ctx->gu, nullptr, 2 * F, ACC, f32, w.w_up, F))
         return false;
       p[3] = Lin();  // N = 0: nothing to launch
-      if (!make_lin(ctx, &p[4], M, d, F, hf, hl, F, w.w_down, ctx->x, nullptr, d, ACC, f32)) return false;
+      if (!make_lin(ctx, &p[4], M, d, F, hf, hl, F, w.w_down, ctx->x, nullptr, d, ACC, f32, nullptr, 0,
+                    ctx->tc_zero ? ctx->qkv : nullptr, static_cast<long long>(M) * 3 * d))
+        return false;
     }
     return true;
   };
@@ -877,6 +887,7 @@ chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
   ok = ok && dalloc_bytes(ctx, &ctx->xn, Rx * d * ctx->esz);
   if (sp) ok = ok && dalloc_bytes(ctx, &ctx->xn_lo, Rx * d * ctx->esz);
   ok = ok && dalloc(ctx, &ctx->qkv, static_cast<size_t>(ctx->R) * 3 * d);
+  ctx->tc_zero = ctx->dtype == 1;
   ok = ok && dalloc(ctx, &ctx->qr, static_cast<size_t>(ctx->R) * d);
   ok = ok && dalloc_bytes(ctx, &ctx->ao, static_cast<size_t>(ctx->R) * d * ctx->esz);
   if (sp) ok = ok && dalloc_bytes(ctx, &ctx->ao_lo, static_cast<size_t>(ctx->R) * d * ctx->esz);
