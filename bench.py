@@ -32,6 +32,11 @@ import torch  # noqa: E402
 import synth  # noqa: E402
 
 WORKLOAD = "7b"
+# dram__bytes_read.sum + dram__bytes_write.sum of the 158 linear launches of one step of
+# this workload (ncu, one pass, see profiles/step_7b_bs1_launch_list.md); against the
+# 17.53 GB of weights they stream, 4 % more (the fp32 outputs read by the reductions).
+# Must be re-measured (or set to None) whenever the linear kernel changes.
+LINEAR_DRAM_BYTES_PER_STEP = 18.23e9
 
 
 def peaks():
@@ -357,7 +362,8 @@ def main():
         "config": {"workload": "7B-shaped bs1 draft-and-verify step (N=64, topk 5,5,5,5, 512-token prompt)",
                    "batch": B, "tree_nodes": N, "prompt_len": len(prompt), "n_ctx": [n0, n1],
                    "parallelism": "replicas" if world > 1 else "single",
-                   "precision": "bf16 weights; split hi+lo bf16 GEMM operands, fp32 accumulation, fp32 KV cache",
+                   "precision": "bf16 weights; split hi+lo bf16 GEMM operands, fp32 accumulation, "
+                                "KV cache as hi+lo bf16 planes (fp32-equivalent)",
                    "l2": "inputs larger than L2: 17.8 GB of weights streamed per step"},
         "breakdown": {
             "verify_ms_eager": phase_ms["verify"], "draft_ms_eager": phase_ms["draft"],
@@ -372,8 +378,9 @@ def main():
         },
         "roofline": {"bound": "hbm", "kernel": "linear_tc (tcgen05 weight-streaming linear)",
                      "achieved": lin_gbs, "peak": hbm, "peak_kind": peak_kind, "unit": "GB/s",
-                     "frac": lin_gbs / hbm, "traffic": None, "launches_per_step": lin_n,
-                     "bytes_per_step": lin_bytes, "ms_per_step": lin_ms},
+                     "frac": lin_gbs / hbm, "traffic": LINEAR_DRAM_BYTES_PER_STEP,
+                     "traffic_basis": "DRAM bytes read + written by all linear launches of one step (ncu)",
+                     "launches_per_step": lin_n, "bytes_per_step": lin_bytes, "ms_per_step": lin_ms},
         "cpu_baseline": cpu,
         "e2e": {"value": world * B * N / t_e2e, "unit": "tree tokens/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": d2h, "ms_per_step": t_e2e * 1e3},
