@@ -18,9 +18,9 @@
 // and O finite in fp32); the final normalisation uses the same max, so the result is
 // exact.  Scores and maxima are kept in base-2 units (scaled by log2 e).
 //
-// Warps: 0..3 softmax + epilogue (tensor-memory lanes 32w.., rows 16w..16w+15),
-// 4 loads the KV tiles (one thread issues TMA copies of 16-row page boxes into
-// two-stage rings for K and for V, 128-byte swizzle applied by the copy engine), 5
+// Warps: 0..7 softmax + epilogue (warp w: tensor-memory lanes 32 (w % 4).., rows
+// 16 (w % 4) .. + 15, keys / output columns of half w / 4), 8 loads the KV tiles (one thread issues TMA copies of 16-row page boxes into
+// two-stage rings for K and for V, 128-byte swizzle applied by the copy engine), 9
 // issues the MMAs and owns the tensor-memory allocation.
 #include <algorithm>
 #include <cmath>
@@ -35,7 +35,7 @@ namespace {
 constexpr int HD = 128;
 constexpr int KT = 64;                      // keys per tile
 constexpr int NQ = 64;                      // query rows (UMMA M)
-constexpr int SOFT_WARPS = 4, LOAD_WARPS = 1;
+constexpr int SOFT_WARPS = 8, LOAD_WARPS = 1;  // softmax: warps w and w + 4 share rows, split keys
 constexpr int THREADS = (SOFT_WARPS + LOAD_WARPS + 1) * 32;
 constexpr int MMA_WARP = SOFT_WARPS + LOAD_WARPS;
 constexpr int ATOM_ROWS64 = 64 * 128;       // bytes of one 64-row x 128-byte swizzle atom column
@@ -103,8 +103,8 @@ __device__ __forceinline__ void split_pair(float a, float b, uint32_t& hi, uint3
 }
 
 // Tensor-memory row of query r under the M = 64 data-path layout: 16 rows per 32-lane
-// sub-partition, in its lanes 0..15.
-__device__ __forceinline__ int row_of(int warp, int lane) { return lane < 16 ? warp * 16 + lane : -1; }
+// sub-partition, in its lanes 0..15 (warp w reaches sub-partition w % 4).
+__device__ __forceinline__ int row_of(int warp, int lane) { return lane < 16 ? (warp & 3) * 16 + lane : -1; }
 
 #ifdef CHIMERA_ATTN_TRACE
 // per-CTA timestamps of the last launch (instrumented builds only)
@@ -142,6 +142,8 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
   int* s_abort = reinterpret_cast<int*>(tmem_slot + 1);
   int* s_pages = s_abort + 2;        // [PAGE_CACHE]
   float* s_stat = reinterpret_cast<float*>(s_pages + PAGE_CACHE);  // [64][2] final (m, l)
+  float* s_xm = s_stat + 2 * NQ;     // [2 tiles][2 halves][64] tile maxima of the key halves
+  float* s_lh = s_xm + 4 * NQ;       // [2 halves][64] partial row sums
   volatile int* abort = s_abort;
 
   const int s = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
@@ -350,13 +352,15 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
     uint64_t last_progress = global_timer_ns();
     while ((nk < nt || nv < nt) && !*abort) {
       bool moved = false;
-      if (nk < nt && (nk < STAGES || mbar_try_wait(&k_empty[nk & 1], ((nk - STAGES) >> 1) & 1))) {
+      if (nk < nt && (nk < STAGES || mbar_test(&k_empty[nk & 1], ((nk - STAGES) >> 1) & 1))) {
+        if (nk == 10) TTRACE(16);
         issue_half(t0 + nk, nk & 1, total, false);
         for (pf = max(pf, nk + 1); pf < nt && pf <= nk + L2_AHEAD; ++pf) prefetch_tile(t0 + pf, total);
         ++nk;
         moved = true;
       }
-      if (nv < nk && (nv < STAGES || mbar_try_wait(&v_empty[nv & 1], ((nv - STAGES) >> 1) & 1))) {
+      if (nv < nk && (nv < STAGES || mbar_test(&v_empty[nv & 1], ((nv - STAGES) >> 1) & 1))) {
+        if (nv == 10) TTRACE(17);
         issue_half(t0 + nv, nv & 1, total, true);
         ++nv;
         moved = true;
@@ -379,38 +383,44 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
       const uint32_t id_qk = idesc_f16(NQ, KT, false);
       const uint32_t id_pv = idesc_f16(NQ, HD, true);
       const uint32_t qh = smem_u32(q_hi), ql = smem_u32(q_lo);
+      // descriptors are precomputed once; advancing a K-major operand by b bytes adds
+      // b >> 4 to its start-address field (all operands lie below 256 KB of shared memory)
+      const uint64_t dq_h = desc_sw128(qh, 16, 1024), dq_l = desc_sw128(ql, 16, 1024);
+      uint64_t dk_h[STAGES], dv_h[STAGES], dp_h[2];
+#pragma unroll
+      for (int st = 0; st < STAGES; ++st) {
+        dk_h[st] = desc_sw128(smem_u32(kbuf + st * HALF_BYTES), 16, 1024);
+        // V as MN-major B: 64-dim atoms 8 KB apart (leading), 8-key groups 1 KB apart
+        dv_h[st] = desc_sw128(smem_u32(vbuf + st * HALF_BYTES), ATOM_ROWS64, 1024);
+      }
+#pragma unroll
+      for (int pb = 0; pb < 2; ++pb) dp_h[pb] = desc_sw128(smem_u32(p_buf + (2 * pb) * (NQ * 128)), 16, 1024);
+      constexpr uint64_t LO_OFS = TILE64 >> 4;        // hi plane -> lo plane (16 KB)
+      constexpr uint64_t P_LO_OFS = (NQ * 128) >> 4;  // P hi -> P lo (8 KB)
       auto pv = [&](int i) {  // O += P_i V_i
         const int st = i & 1;
-        const uint32_t ph = smem_u32(p_buf + (2 * (i & 1)) * (NQ * 128));
-        const uint32_t pl = ph + NQ * 128;
-        const uint32_t vh = smem_u32(vbuf + st * HALF_BYTES);
-        const uint32_t vl = vh + TILE64;
         const uint32_t o_t = tmem + 128;
 #pragma unroll
         for (int ks = 0; ks < KT / 16; ++ks) {
-          const uint64_t a_h = desc_sw128(ph + ks * 32, 16, 1024), a_l = desc_sw128(pl + ks * 32, 16, 1024);
-          // V as MN-major B: 64-dim atoms 8 KB apart (leading), 8-key groups 1 KB apart
-          const uint64_t b_h = desc_sw128(vh + ks * 2048, ATOM_ROWS64, 1024);
+          const uint64_t a_h = dp_h[st] + static_cast<uint64_t>(ks * 2);  // 32 bytes per K step
+          const uint64_t b_h = dv_h[st] + static_cast<uint64_t>(ks * 128);  // 16 keys = 2 KB
           tc_mma_bf16(o_t, a_h, b_h, id_pv, (i > 0 || ks > 0) ? 1u : 0u);
-          tc_mma_bf16(o_t, a_l, b_h, id_pv, 1u);
-          if (SPLIT) tc_mma_bf16(o_t, a_h, desc_sw128(vl + ks * 2048, ATOM_ROWS64, 1024), id_pv, 1u);
+          tc_mma_bf16(o_t, a_h + P_LO_OFS, b_h, id_pv, 1u);
+          if (SPLIT) tc_mma_bf16(o_t, a_h, b_h + LO_OFS, id_pv, 1u);
         }
         tc_commit(&pv_done[i & 1]);
         tc_commit(&v_empty[st]);
       };
       auto qk = [&](int i) {  // S_i = Q K_i^T into S buffer i & 1
         const int st = i & 1;
-        const uint32_t kh = smem_u32(kbuf + st * HALF_BYTES);
-        const uint32_t kl = kh + TILE64;
         const uint32_t s_t = tmem + st * 64;
 #pragma unroll
         for (int ks = 0; ks < HD / 16; ++ks) {
-          const uint32_t off = (ks >> 2) * ATOM_ROWS64 + (ks & 3) * 32;
-          const uint64_t a_h = desc_sw128(qh + off, 16, 1024), a_l = desc_sw128(ql + off, 16, 1024);
-          const uint64_t b_h = desc_sw128(kh + off, 16, 1024);
-          tc_mma_bf16(s_t, a_h, b_h, id_qk, ks > 0 ? 1u : 0u);
-          tc_mma_bf16(s_t, a_l, b_h, id_qk, 1u);
-          if (SPLIT) tc_mma_bf16(s_t, a_h, desc_sw128(kl + off, 16, 1024), id_qk, 1u);
+          const uint64_t off = static_cast<uint64_t>(((ks >> 2) * ATOM_ROWS64 + (ks & 3) * 32) >> 4);
+          const uint64_t b_h = dk_h[st] + off;
+          tc_mma_bf16(s_t, dq_h + off, b_h, id_qk, ks > 0 ? 1u : 0u);
+          tc_mma_bf16(s_t, dq_l + off, b_h, id_qk, 1u);
+          if (SPLIT) tc_mma_bf16(s_t, dq_h + off, b_h + LO_OFS, id_qk, 1u);
         }
         tc_commit(&s_full[st]);
         tc_commit(&k_empty[st]);
@@ -422,19 +432,21 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
       uint64_t last_progress = global_timer_ns();
       while (npv < nt && !*abort) {
         bool moved = false;
-        if (npv < nqk && mbar_try_wait(&p_full[npv & 1], (npv >> 1) & 1) &&
-            mbar_try_wait(&v_full[npv & 1], (npv >> 1) & 1)) {
+        if (npv < nqk && mbar_test(&p_full[npv & 1], (npv >> 1) & 1) &&
+            mbar_test(&v_full[npv & 1], (npv >> 1) & 1)) {
           tc_fence_after();
           if (npv == 10) TTRACE(22);
+          if (npv == 9) TTRACE(25);
           pv(npv);
           ++npv;
           moved = true;
         }
-        if (nqk < nt && nqk <= npv + 1 && mbar_try_wait(&k_full[nqk & 1], (nqk >> 1) & 1) &&
-            (nqk < 2 || mbar_try_wait(&s_free[nqk & 1], ((nqk - 2) >> 1) & 1))) {
+        if (nqk < nt && nqk <= npv + 1 && mbar_test(&k_full[nqk & 1], (nqk >> 1) & 1) &&
+            (nqk < 2 || mbar_test(&s_free[nqk & 1], ((nqk - 2) >> 1) & 1))) {
           tc_fence_after();
           if (nqk == 0) TTRACE(5);
           if (nqk == 10) TTRACE(19);
+          if (nqk == 12) TTRACE(24);
           qk(nqk);
           ++nqk;
           moved = true;
@@ -450,35 +462,38 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
       mbar_wait_plain(o_done, 0, 200000000ull);
     }
   } else {
-    // ---------------- softmax (warps 0..3) ----------------
+    // ---------------- softmax (warps 0..7) ----------------
+    // warps w and w + 4 own the same 16 rows and the key halves 0 / 1 of every tile;
+    // the pair shares its tile maxima through shared memory (named barrier 1 + w % 4).
+    // After a timeout the loop keeps running (without work) so both warps of a pair
+    // still meet at every barrier.
     const int r = row_of(warp, lane);
+    const int half = warp >> 2, quad = warp & 3;
     const bool live = r >= 0 && r < nq;
     const unsigned long long anc = live ? p.anc[p.q_local0 + r] : 0ull;
     const float scale2 = p.scale * 1.4426950408889634f;  // softmax in base 2: exp(x) = 2^(x log2 e)
+    const uint32_t tlane = static_cast<uint32_t>(quad * 32) << 16;
     float m_used = -INFINITY, l = 0.f;
+    bool dead = false;
     for (int t = t0; t < t1; ++t) {
       const int i = t - t0, sb = i & 1;
-      bool ok = mbar_wait(&s_full[sb], (i >> 1) & 1, abort);
-      if (!__all_sync(0xffffffffu, ok)) break;
+      bool ok = !dead && mbar_wait(&s_full[sb], (i >> 1) & 1, abort);
+      dead = !__all_sync(0xffffffffu, ok);
       tc_fence_after();
-      if (warp == 0 && lane == 0 && i == 0) TTRACE(6);
-      if (warp == 0 && lane == 0 && i == 1) TTRACE(13);
       if (warp == 0 && lane == 0 && i == 10) TTRACE(20);
-      float sv[KT];
-      {
+      float sv[32];
+      if (!dead) {
         uint32_t rr[64];
 #pragma unroll
-        for (int j = 0; j < 4; ++j) tmem_ld16_issue(tmem + (static_cast<uint32_t>(warp * 32) << 16) + sb * 64 + 16 * j, rr + 16 * j);
+        for (int j = 0; j < 2; ++j) tmem_ld16_issue(tmem + tlane + sb * 64 + half * 32 + 16 * j, rr + 16 * j);
         tmem_wait_ld64(rr);
 #pragma unroll
-        for (int j = 0; j < KT; ++j) sv[j] = __uint_as_float(rr[j]);
+        for (int j = 0; j < 32; ++j) sv[j] = __uint_as_float(rr[j]);
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&s_free[sb]);
-      if (warp == 0 && lane == 0 && i == 0) TTRACE(8);
-      // visibility of the tile's keys for this row (bit j: key 64t + j): committed keys,
-      // then local keys whose ancestor bit is set, cut at the sequence's end
+      if (lane == 0 && !dead) mbar_arrive(&s_free[sb]);
+      // visibility of the half's keys for this row (bit j: key 64t + 32 half + j)
       unsigned long long vmask = 0ull;
       if (live) {
         const int base = t * KT;
@@ -486,56 +501,56 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
         const unsigned long long cm = nc >= 64 ? ~0ull : (nc <= 0 ? 0ull : ((1ull << nc) - 1ull));
         const unsigned long long lm = off >= 0 ? (off < 64 ? (anc >> off) : 0ull) : (-off < 64 ? (anc << -off) : 0ull);
         const unsigned long long vm = nv >= 64 ? ~0ull : (nv <= 0 ? 0ull : ((1ull << nv) - 1ull));
-        vmask = (cm | lm) & vm;
+        vmask = ((cm | lm) & vm) >> (32 * half);
       }
-      // scores in log2 units, tile maximum
       float tmax = -INFINITY;
 #pragma unroll
-      for (int j = 0; j < KT; ++j) {
-        sv[j] = ((vmask >> j) & 1ull) ? sv[j] * scale2 : -INFINITY;
+      for (int j = 0; j < 32; ++j) {
+        sv[j] = (!dead && ((vmask >> j) & 1ull)) ? sv[j] * scale2 : -INFINITY;
         tmax = fmaxf(tmax, sv[j]);
       }
+      // the row's maximum over both key halves
+      if (r >= 0) s_xm[(sb * 2 + half) * NQ + r] = tmax;
+      named_bar(1 + quad, 64);
+      if (r >= 0) tmax = fmaxf(tmax, s_xm[(sb * 2 + (half ^ 1)) * NQ + r]);
       // this tile's P buffer was read by the PV product of tile i - 2
       if (i >= 2) {
-        ok = mbar_wait(&pv_done[i & 1], ((i - 2) >> 1) & 1, abort);
-        if (!__all_sync(0xffffffffu, ok)) break;
+        ok = !dead && mbar_wait(&pv_done[i & 1], ((i - 2) >> 1) & 1, abort);
+        dead = !__all_sync(0xffffffffu, ok);
         tc_fence_after();
       }
-      if (warp == 0 && lane == 0 && i == 10) TTRACE(23);
       const bool raise = tmax > m_used + RESCALE_LOG2 || (m_used == -INFINITY && tmax > -INFINITY);
       float corr = 1.f;
       if (raise) {
         corr = (m_used == -INFINITY) ? 0.f : exp2f(m_used - tmax);
         m_used = tmax;
       }
-      if (__any_sync(0xffffffffu, raise && corr != 0.f && l > 0.f) && i > 0) {
+      if (!dead && __any_sync(0xffffffffu, raise && corr != 0.f && l > 0.f) && i > 0) {
         // O holds the products up to tile i - 1: wait for the last one before rescaling
         ok = mbar_wait(&pv_done[(i - 1) & 1], ((i - 1) >> 1) & 1, abort);
-        if (!__all_sync(0xffffffffu, ok)) break;
+        dead = !__all_sync(0xffffffffu, ok);
         tc_fence_after();
-        // rescale this warp's O rows in tensor memory (factor 1 for rows that kept m)
-        const float f = (raise && l > 0.f) ? corr : 1.f;
-#pragma unroll
-        for (int c0 = 0; c0 < HD; c0 += 64) {
+        if (!dead) {
+          // rescale this warp's half of its O rows (factor 1 for rows that kept m)
+          const float f = (raise && l > 0.f) ? corr : 1.f;
           uint32_t rr[64];
 #pragma unroll
-          for (int j = 0; j < 4; ++j)
-            tmem_ld16_issue(tmem + (static_cast<uint32_t>(warp * 32) << 16) + 128 + c0 + 16 * j, rr + 16 * j);
+          for (int j = 0; j < 4; ++j) tmem_ld16_issue(tmem + tlane + 128 + half * 64 + 16 * j, rr + 16 * j);
           tmem_wait_ld64(rr);
 #pragma unroll
           for (int j = 0; j < 64; ++j) rr[j] = __float_as_uint(__uint_as_float(rr[j]) * f);
 #pragma unroll
-          for (int j = 0; j < 4; ++j) tmem_st16(tmem + (static_cast<uint32_t>(warp * 32) << 16) + 128 + c0 + 16 * j, rr + 16 * j);
+          for (int j = 0; j < 4; ++j) tmem_st16(tmem + tlane + 128 + half * 64 + 16 * j, rr + 16 * j);
+          tmem_wait_st();
         }
-        tmem_wait_st();
       }
       l *= corr;
-      // P = exp(S - m), two-term split into the swizzled P tile of this tile
+      // P = exp(S - m), two-term split into the swizzled P tile (this half's 4 chunks)
       uint8_t* ph = p_buf + (2 * sb) * (NQ * 128);
       uint8_t* pl = ph + NQ * 128;
       float rsum = 0.f;
 #pragma unroll
-      for (int c = 0; c < 8; ++c) {
+      for (int c = 0; c < 4; ++c) {
         float pv8[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
@@ -548,24 +563,21 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
         split_pair(pv8[2], pv8[3], hh.y, ll.y);
         split_pair(pv8[4], pv8[5], hh.z, ll.z);
         split_pair(pv8[6], pv8[7], hh.w, ll.w);
-        if (r >= 0) {
-          *reinterpret_cast<uint4*>(ph + swz(r, c)) = hh;
-          *reinterpret_cast<uint4*>(pl + swz(r, c)) = ll;
+        if (r >= 0 && !dead) {
+          *reinterpret_cast<uint4*>(ph + swz(r, half * 4 + c)) = hh;
+          *reinterpret_cast<uint4*>(pl + swz(r, half * 4 + c)) = ll;
         }
       }
       l += rsum;
-      if (warp == 0 && lane == 0 && i == 0) TTRACE(15);
       if (warp == 0 && lane == 0 && i == 10) TTRACE(21);
       fence_async_smem();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&p_full[sb]);
-      if (warp == 0 && lane == 0 && i == 0) TTRACE(7);
-      if (warp == 0 && lane == 0 && i == nt - 1) TTRACE(14);
+      if (lane == 0 && !dead) mbar_arrive(&p_full[sb]);
     }
     if (r >= 0) {
-      s_stat[2 * r] = m_used;
-      s_stat[2 * r + 1] = l;
+      if (half == 0) s_stat[2 * r] = m_used;
+      s_lh[half * NQ + r] = l;
     }
   }
 
@@ -591,10 +603,12 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
     const bool soft = warp < SOFT_WARPS;
     const bool have = soft && nt > 0 && !*abort;
     const bool mine = soft && r >= 0 && r < nq;
+    const int half = (warp >> 2) & 1;
     uint32_t rr[64];
-    if (have) {  // first 64 columns of the O row while the peers finish
+    if (have) {  // this warp's 64 columns of the O row, while the peers finish
 #pragma unroll
-      for (int j = 0; j < 4; ++j) tmem_ld16_issue(tmem + (static_cast<uint32_t>(warp * 32) << 16) + 128 + 16 * j, rr + 16 * j);
+      for (int j = 0; j < 4; ++j)
+        tmem_ld16_issue(tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16) + 128 + half * 64 + 16 * j, rr + 16 * j);
       tmem_wait_ld64(rr);
     }
     __syncwarp();
@@ -603,29 +617,20 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
       const int owner = mine ? r / rpc : 0;
       const uint32_t slot = smem_u32(recv + (s * rpc + (mine ? r - owner * rpc : 0)) * PREC);
       const uint32_t dst = S > 1 ? dsmem_addr(slot, owner) : slot;
-      const float lr = mine ? s_stat[2 * r + 1] : 0.f;
+      const float lr = mine ? s_lh[r] + s_lh[NQ + r] : 0.f;
       const bool keep = have && lr > 0.f;
-#pragma unroll
-      for (int half = 0; half < 2; ++half) {
-        if (half == 1 && have) {
-#pragma unroll
-          for (int j = 0; j < 4; ++j)
-            tmem_ld16_issue(tmem + (static_cast<uint32_t>(warp * 32) << 16) + 128 + 64 + 16 * j, rr + 16 * j);
-          tmem_wait_ld64(rr);
-        }
-        if (mine) {
-#pragma unroll
-          for (int j = 0; j < 64; j += 4) {
-            const float4 v = keep ? make_float4(__uint_as_float(rr[j]), __uint_as_float(rr[j + 1]),
-                                                __uint_as_float(rr[j + 2]), __uint_as_float(rr[j + 3]))
-                                  : make_float4(0.f, 0.f, 0.f, 0.f);
-            st_dsmem4(dst + static_cast<uint32_t>((half * 64 + j) * 4), v);
-          }
-        }
-      }
       if (mine) {
-        st_dsmem(dst + HD * 4, nt > 0 ? s_stat[2 * r] : -INFINITY);
-        st_dsmem(dst + (HD + 1) * 4, nt > 0 ? lr : 0.f);
+#pragma unroll
+        for (int j = 0; j < 64; j += 4) {
+          const float4 v = keep ? make_float4(__uint_as_float(rr[j]), __uint_as_float(rr[j + 1]),
+                                              __uint_as_float(rr[j + 2]), __uint_as_float(rr[j + 3]))
+                                : make_float4(0.f, 0.f, 0.f, 0.f);
+          st_dsmem4(dst + static_cast<uint32_t>((half * 64 + j) * 4), v);
+        }
+        if (half == 0) {
+          st_dsmem(dst + HD * 4, nt > 0 ? s_stat[2 * r] : -INFINITY);
+          st_dsmem(dst + (HD + 1) * 4, nt > 0 ? lr : 0.f);
+        }
       }
     }
   }
@@ -686,7 +691,7 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
 template <bool SPLIT>
 size_t tc_smem() {
   const size_t np = SPLIT ? 4 : 2;
-  return 1024 + 2 * TILE64 + 4 * NQ * 128 + STAGES * np * TILE64 + 18 * 8 + 16 + PAGE_CACHE * 4 + 2 * NQ * 4;
+  return 1024 + 2 * TILE64 + 4 * NQ * 128 + STAGES * np * TILE64 + 18 * 8 + 16 + PAGE_CACHE * 4 + 8 * NQ * 4;
 }
 
 template <bool SPLIT>
