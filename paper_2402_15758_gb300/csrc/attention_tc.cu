@@ -481,6 +481,7 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
       dead = !__all_sync(0xffffffffu, ok);
       tc_fence_after();
       if (warp == 0 && lane == 0 && i == 10) TTRACE(20);
+      if (warp == 0 && lane == 0 && i == 0) TTRACE(6);
       float sv[32];
       if (!dead) {
         uint32_t rr[64];
@@ -570,6 +571,7 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
       }
       l += rsum;
       if (warp == 0 && lane == 0 && i == 10) TTRACE(21);
+      if (warp == 0 && lane == 0 && i == 0) TTRACE(7);
       fence_async_smem();
       tc_fence_before();
       __syncwarp();
@@ -587,8 +589,10 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
   // main loop (split cluster barrier) ----
   if (warp < SOFT_WARPS) {
     if (nt > 0) {
+      if (warp == 0 && lane == 0) TTRACE(14);
       mbar_wait(o_done, 0, abort);
       tc_fence_after();
+      if (warp == 0 && lane == 0) TTRACE(9);
     }
     __syncwarp();
   }
@@ -613,6 +617,7 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
     }
     __syncwarp();
     if (S > 1) cluster_wait();
+    if (threadIdx.x == 0) TTRACE(11);
     if (soft) {
       const int owner = mine ? r / rpc : 0;
       const uint32_t slot = smem_u32(recv + (s * rpc + (mine ? r - owner * rpc : 0)) * PREC);
@@ -643,7 +648,9 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
   }
   if (threadIdx.x == 0 && *abort && p.err) atomicOr(p.err, ERR_TIMEOUT);
   __syncwarp();
+  if (threadIdx.x == 0) TTRACE(12);
   if (S > 1) cluster_sync();  // every push into this CTA is complete and visible
+  if (threadIdx.x == 0) TTRACE(13);
 
   // ---- merge the S partials of this CTA's rows (local shared memory) ----
   bf16* out = static_cast<bf16*>(p.out);
