@@ -70,13 +70,43 @@ __device__ __forceinline__ uint32_t idesc_f16(int m, int n, bool b_mn) {
          (static_cast<uint32_t>(m >> 4) << 24);
 }
 
-__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* r) {
+// 16x32bx2 access shape: lanes 0..15 of the warp read (write) TMEM lanes 0..15 of the
+// warp's sub-partition at the addressed column, lanes 16..31 the same TMEM lanes at the
+// column plus OFS; each of the 16 registers is the next column.
+template <int OFS>
+__device__ __forceinline__ void tmem_ld16x2(uint32_t taddr, uint32_t* r) {
   asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
-      "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};" ::"r"(taddr),
-      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]),
-      "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+      "tcgen05.ld.sync.aligned.16x32bx2.x16.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16], %17;"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr), "n"(OFS));
+}
+template <int OFS>
+__device__ __forceinline__ void tmem_st16x2(uint32_t taddr, const uint32_t* r) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.16x32bx2.x16.b32 [%0], %1, "
+      "{%2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17};" ::"r"(taddr), "n"(OFS), "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
       : "memory");
+}
+// Wait for the issued TMEM loads; the registers are operands so that no use of them is
+// scheduled before the wait.
+__device__ __forceinline__ void tmem_wait_ld16(uint32_t (&r)[16]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15])
+               :
+               : "memory");
+}
+__device__ __forceinline__ void tmem_wait_ld32(uint32_t (&r)[32]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]), "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]), "+r"(r[29]), "+r"(r[30]), "+r"(r[31])
+               :
+               : "memory");
+}
+// 2^x on the special-function unit (inputs here are <= 0; results below 2^-126 flush to 0)
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
 }
 __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
@@ -102,9 +132,8 @@ __device__ __forceinline__ void split_pair(float a, float b, uint32_t& hi, uint3
   lo = pack_bf16x2(a - hf.x, b - hf.y);
 }
 
-// Tensor-memory row of query r under the M = 64 data-path layout: 16 rows per 32-lane
-// sub-partition, in its lanes 0..15 (warp w reaches sub-partition w % 4).
-__device__ __forceinline__ int row_of(int warp, int lane) { return lane < 16 ? (warp & 3) * 16 + lane : -1; }
+// Under the M = 64 data-path layout, query rows 16q .. 16q + 15 sit in TMEM lanes 0..15 of
+// sub-partition q (warp w reaches sub-partition w % 4).
 
 #ifdef CHIMERA_ATTN_TRACE
 // per-CTA timestamps of the last launch (instrumented builds only)
@@ -463,13 +492,16 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
     }
   } else {
     // ---------------- softmax (warps 0..7) ----------------
-    // warps w and w + 4 own the same 16 rows and the key halves 0 / 1 of every tile;
-    // the pair shares its tile maxima through shared memory (named barrier 1 + w % 4).
-    // After a timeout the loop keeps running (without work) so both warps of a pair
-    // still meet at every barrier.
-    const int r = row_of(warp, lane);
-    const int half = warp >> 2, quad = warp & 3;
-    const bool live = r >= 0 && r < nq;
+    // Warps w and w + 4 own the 16 rows of TMEM sub-partition w % 4 and the key halves
+    // 0 / 1 of every tile; within a warp, lanes l and l + 16 share row l % 16 and take
+    // 16 keys each (the 16x32bx2 access shape), so every lane works. The two lanes of a
+    // row combine by a shuffle, the warp pair through shared memory (named barrier
+    // 1 + w % 4). After a timeout the loop keeps running (without work) so both warps of
+    // a pair still meet at every barrier.
+    const int half = warp >> 2, quad = warp & 3, sub = lane >> 4;
+    const int r = quad * 16 + (lane & 15);
+    const bool live = r < nq;
+    const int kofs = 32 * half + 16 * sub;  // this lane's first key within a tile
     const unsigned long long anc = live ? p.anc[p.q_local0 + r] : 0ull;
     const float scale2 = p.scale * 1.4426950408889634f;  // softmax in base 2: exp(x) = 2^(x log2 e)
     const uint32_t tlane = static_cast<uint32_t>(quad * 32) << 16;
@@ -482,102 +514,120 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
       tc_fence_after();
       if (warp == 0 && lane == 0 && i == 10) TTRACE(20);
       if (warp == 0 && lane == 0 && i == 0) TTRACE(6);
-      float sv[32];
+      float sv[16];
       if (!dead) {
-        uint32_t rr[64];
+        uint32_t rr[16];
+        tmem_ld16x2<16>(tmem + tlane + sb * 64 + half * 32, rr);
+        tmem_wait_ld16(rr);
 #pragma unroll
-        for (int j = 0; j < 2; ++j) tmem_ld16_issue(tmem + tlane + sb * 64 + half * 32 + 16 * j, rr + 16 * j);
-        tmem_wait_ld64(rr);
-#pragma unroll
-        for (int j = 0; j < 32; ++j) sv[j] = __uint_as_float(rr[j]);
+        for (int j = 0; j < 16; ++j) sv[j] = __uint_as_float(rr[j]);
       }
+      if (warp == 0 && lane == 0 && i == 10) TTRACE(26);
       tc_fence_before();
       __syncwarp();
       if (lane == 0 && !dead) mbar_arrive(&s_free[sb]);
-      // visibility of the half's keys for this row (bit j: key 64t + 32 half + j)
-      unsigned long long vmask = 0ull;
+      // visibility of this lane's 16 keys (bit j: key 64t + kofs + j)
+      uint32_t vbits = 0u;
       if (live) {
         const int base = t * KT;
         const int nc = nctx - base, nv = total - base, off = base - nctx;
         const unsigned long long cm = nc >= 64 ? ~0ull : (nc <= 0 ? 0ull : ((1ull << nc) - 1ull));
         const unsigned long long lm = off >= 0 ? (off < 64 ? (anc >> off) : 0ull) : (-off < 64 ? (anc << -off) : 0ull);
         const unsigned long long vm = nv >= 64 ? ~0ull : (nv <= 0 ? 0ull : ((1ull << nv) - 1ull));
-        vmask = ((cm | lm) & vm) >> (32 * half);
+        vbits = static_cast<uint32_t>(((cm | lm) & vm) >> kofs) & 0xFFFFu;
       }
-      float tmax = -INFINITY;
+      float ta = -INFINITY, tb = -INFINITY;  // two chains of maxima
 #pragma unroll
-      for (int j = 0; j < 32; ++j) {
-        sv[j] = (!dead && ((vmask >> j) & 1ull)) ? sv[j] * scale2 : -INFINITY;
-        tmax = fmaxf(tmax, sv[j]);
+      for (int j = 0; j < 16; ++j) {
+        sv[j] = (!dead && ((vbits >> j) & 1u)) ? sv[j] * scale2 : -INFINITY;
+        if (j & 1)
+          tb = fmaxf(tb, sv[j]);
+        else
+          ta = fmaxf(ta, sv[j]);
       }
-      // the row's maximum over both key halves
-      if (r >= 0) s_xm[(sb * 2 + half) * NQ + r] = tmax;
+      // the row's maximum over its 64 keys: the other lane of the row, then the pair warp
+      float tmax = fmaxf(ta, tb);
+      tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 16));
+      if (sub == 0) s_xm[(sb * 2 + half) * NQ + r] = tmax;
       named_bar(1 + quad, 64);
-      if (r >= 0) tmax = fmaxf(tmax, s_xm[(sb * 2 + (half ^ 1)) * NQ + r]);
+      tmax = fmaxf(tmax, s_xm[(sb * 2 + (half ^ 1)) * NQ + r]);
+      if (warp == 0 && lane == 0 && i == 10) TTRACE(27);
       // this tile's P buffer was read by the PV product of tile i - 2
       if (i >= 2) {
         ok = !dead && mbar_wait(&pv_done[i & 1], ((i - 2) >> 1) & 1, abort);
         dead = !__all_sync(0xffffffffu, ok);
         tc_fence_after();
       }
+      if (warp == 0 && lane == 0 && i == 10) TTRACE(28);
+      // m moves only when the tile's maximum exceeds it by more than 2^RESCALE_LOG2; O then
+      // holds products of earlier tiles exactly when m was already finite. Both decisions
+      // depend only on the row's shared maxima, so all four lanes of a row agree.
       const bool raise = tmax > m_used + RESCALE_LOG2 || (m_used == -INFINITY && tmax > -INFINITY);
+      const bool rescale = raise && m_used != -INFINITY;
       float corr = 1.f;
       if (raise) {
-        corr = (m_used == -INFINITY) ? 0.f : exp2f(m_used - tmax);
+        corr = rescale ? exp2f(m_used - tmax) : 0.f;
         m_used = tmax;
       }
-      if (!dead && __any_sync(0xffffffffu, raise && corr != 0.f && l > 0.f) && i > 0) {
+      if (!dead && i > 0 && __any_sync(0xffffffffu, rescale)) {
         // O holds the products up to tile i - 1: wait for the last one before rescaling
         ok = mbar_wait(&pv_done[(i - 1) & 1], ((i - 1) >> 1) & 1, abort);
         dead = !__all_sync(0xffffffffu, ok);
         tc_fence_after();
         if (!dead) {
-          // rescale this warp's half of its O rows (factor 1 for rows that kept m)
-          const float f = (raise && l > 0.f) ? corr : 1.f;
-          uint32_t rr[64];
+          // this warp's 64 columns of its O rows (lanes 0..15: the first 32, lanes
+          // 16..31: the last 32); factor 1 for rows that kept m
+          const float f = rescale ? corr : 1.f;
+          const uint32_t oa = tmem + tlane + 128 + half * 64;
+          uint32_t rr[32];
+          tmem_ld16x2<32>(oa, rr);
+          tmem_ld16x2<32>(oa + 16, rr + 16);
+          tmem_wait_ld32(rr);
 #pragma unroll
-          for (int j = 0; j < 4; ++j) tmem_ld16_issue(tmem + tlane + 128 + half * 64 + 16 * j, rr + 16 * j);
-          tmem_wait_ld64(rr);
-#pragma unroll
-          for (int j = 0; j < 64; ++j) rr[j] = __float_as_uint(__uint_as_float(rr[j]) * f);
-#pragma unroll
-          for (int j = 0; j < 4; ++j) tmem_st16(tmem + tlane + 128 + half * 64 + 16 * j, rr + 16 * j);
+          for (int j = 0; j < 32; ++j) rr[j] = __float_as_uint(__uint_as_float(rr[j]) * f);
+          tmem_st16x2<32>(oa, rr);
+          tmem_st16x2<32>(oa + 16, rr + 16);
           tmem_wait_st();
         }
       }
       l *= corr;
-      // P = exp(S - m), two-term split into the swizzled P tile (this half's 4 chunks)
+      // P = 2^(S - m), two-term split into the swizzled P tile (this lane's 2 chunks)
       uint8_t* ph = p_buf + (2 * sb) * (NQ * 128);
       uint8_t* pl = ph + NQ * 128;
-      float rsum = 0.f;
+      float ra = 0.f, rb = 0.f;
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
+      for (int c = 0; c < 2; ++c) {
         float pv8[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
           const float x = sv[8 * c + e];
-          pv8[e] = (x == -INFINITY) ? 0.f : exp2f(x - m_used);
-          rsum += pv8[e];
+          pv8[e] = (x == -INFINITY) ? 0.f : ex2_approx(x - m_used);
+          if (e & 1)
+            rb += pv8[e];
+          else
+            ra += pv8[e];
         }
         uint4 hh, ll;
         split_pair(pv8[0], pv8[1], hh.x, ll.x);
         split_pair(pv8[2], pv8[3], hh.y, ll.y);
         split_pair(pv8[4], pv8[5], hh.z, ll.z);
         split_pair(pv8[6], pv8[7], hh.w, ll.w);
-        if (r >= 0 && !dead) {
-          *reinterpret_cast<uint4*>(ph + swz(r, half * 4 + c)) = hh;
-          *reinterpret_cast<uint4*>(pl + swz(r, half * 4 + c)) = ll;
+        if (!dead) {
+          *reinterpret_cast<uint4*>(ph + swz(r, kofs / 8 + c)) = hh;
+          *reinterpret_cast<uint4*>(pl + swz(r, kofs / 8 + c)) = ll;
         }
       }
-      l += rsum;
+      l += ra + rb;
       if (warp == 0 && lane == 0 && i == 10) TTRACE(21);
       if (warp == 0 && lane == 0 && i == 0) TTRACE(7);
       fence_async_smem();
+      if (warp == 0 && lane == 0 && i == 10) TTRACE(29);
       tc_fence_before();
       __syncwarp();
       if (lane == 0 && !dead) mbar_arrive(&p_full[sb]);
     }
-    if (r >= 0) {
+    l += __shfl_xor_sync(0xffffffffu, l, 16);  // the row's sum over this warp's key half
+    if (sub == 0) {
       if (half == 0) s_stat[2 * r] = m_used;
       s_lh[half * NQ + r] = l;
     }
@@ -603,17 +653,18 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
   float* recv = part;                     // [S][rpc][PREC], S * rpc <= NQ + 7 rows (37.5 KB)
   float* s_w = part + (NQ + 8) * PREC;    // [rpc][8] merge weights, past the receive slots
   {
-    const int r = row_of(warp, lane);
     const bool soft = warp < SOFT_WARPS;
+    const int half = (warp >> 2) & 1, sub = lane >> 4;
+    const int r = (warp & 3) * 16 + (lane & 15);
     const bool have = soft && nt > 0 && !*abort;
-    const bool mine = soft && r >= 0 && r < nq;
-    const int half = (warp >> 2) & 1;
-    uint32_t rr[64];
-    if (have) {  // this warp's 64 columns of the O row, while the peers finish
-#pragma unroll
-      for (int j = 0; j < 4; ++j)
-        tmem_ld16_issue(tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16) + 128 + half * 64 + 16 * j, rr + 16 * j);
-      tmem_wait_ld64(rr);
+    const bool mine = soft && r < nq;
+    const int cb = half * 64 + sub * 32;  // this lane's first O column
+    uint32_t rr[32];
+    if (have) {  // this lane's 32 columns of the O row, while the peers finish
+      const uint32_t oa = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16) + 128 + half * 64;
+      tmem_ld16x2<32>(oa, rr);
+      tmem_ld16x2<32>(oa + 16, rr + 16);
+      tmem_wait_ld32(rr);
     }
     __syncwarp();
     if (S > 1) cluster_wait();
@@ -626,13 +677,13 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
       const bool keep = have && lr > 0.f;
       if (mine) {
 #pragma unroll
-        for (int j = 0; j < 64; j += 4) {
+        for (int j = 0; j < 32; j += 4) {
           const float4 v = keep ? make_float4(__uint_as_float(rr[j]), __uint_as_float(rr[j + 1]),
                                               __uint_as_float(rr[j + 2]), __uint_as_float(rr[j + 3]))
                                 : make_float4(0.f, 0.f, 0.f, 0.f);
-          st_dsmem4(dst + static_cast<uint32_t>((half * 64 + j) * 4), v);
+          st_dsmem4(dst + static_cast<uint32_t>((cb + j) * 4), v);
         }
-        if (half == 0) {
+        if (half == 0 && sub == 0) {
           st_dsmem(dst + HD * 4, nt > 0 ? s_stat[2 * r] : -INFINITY);
           st_dsmem(dst + (HD + 1) * 4, nt > 0 ? lr : 0.f);
         }

@@ -179,3 +179,45 @@ def test_attention_tree_masked_paged(dtype, case):
             ref = co.attend(Q[b, i], Ks, Vs)
             err = np.max(np.abs(got[b, i] - ref)) / np.max(np.abs(ref))
             assert err <= tol, (b, i, err)
+
+
+@pytest.mark.parametrize("jump", [40.0, 150.0])
+@pytest.mark.parametrize("splits", [1, 2])
+def test_attention_rescale_after_one_sided_tile(jump, splits):
+    """Online softmax with a far move of the running maximum. Every query row sees the 20
+    context keys, local row 0 and itself, so row 50's first tile has visible keys in its
+    first key half only; its own key (second tile) scores `jump` nats above zero, which
+    moves the maximum by far more than the lazy-rescale threshold (the correction is
+    about 2^-53 at 40 nats and underflows to 0 at 150). All 128 output columns of the
+    row must then be rescaled, whichever key half saw keys before."""
+    import math
+    H, hd, nctx, n_local, nq = 2, 128, 20, 64, 64
+    max_pages = (nctx + n_local + 15) // 16 + 1
+    perm = np.arange(max_pages, dtype=np.int32).reshape(1, max_pages)
+    kv32 = torch.randn(max_pages, H, 2, 16, hd, generator=torch.Generator().manual_seed(7))
+    q = torch.randn(nq, H * hd, generator=torch.Generator().manual_seed(8))
+    anc = [1 | (1 << i) for i in range(n_local)]
+    r, slot = 50, nctx + 50
+    for h in range(H):
+        qv = q[r, h * hd:(h + 1) * hd]
+        kv32[slot // 16, h, 0, slot % 16] = qv * (jump * math.sqrt(hd) / float(qv @ qv))
+    hi = kv32.to(torch.bfloat16)
+    lo = (kv32 - hi.float()).to(torch.bfloat16)
+    pool = torch.stack([hi[:, :, 0], lo[:, :, 0], hi[:, :, 1], lo[:, :, 1]], dim=2).contiguous()
+    out = torch.zeros(nq, H * hd, dtype=torch.bfloat16, device="cuda")
+    out_lo = torch.zeros_like(out)
+    anc_t = torch.tensor(np.array(anc, dtype=np.uint64).view(np.int64), device="cuda")
+    pkg.op_attention(q.cuda(), pool.cuda(), torch.tensor(perm, device="cuda"),
+                     torch.tensor([nctx], dtype=torch.int32, device="cuda"), anc_t, out, nq=nq, q_local0=0,
+                     n_local=n_local, q_rows=nq, n_heads=H, head_dim=hd, splits=splits, out_lo=out_lo)
+    torch.cuda.synchronize()
+    got = (out.float() + out_lo.float()).cpu().numpy().reshape(nq, H, hd)
+    P = kv32.double().numpy()
+    Q = q.double().numpy().reshape(nq, H, hd)
+    for i in range(nq):
+        slots = list(range(nctx)) + [nctx + j for j in range(n_local) if (anc[i] >> j) & 1]
+        Ks = np.array([P[s // 16, :, 0, s % 16] for s in slots])
+        Vs = np.array([P[s // 16, :, 1, s % 16] for s in slots])
+        ref = co.attend(Q[i], Ks, Vs)
+        err = np.max(np.abs(got[i] - ref)) / np.max(np.abs(ref))
+        assert err <= 5e-5, (i, err)
