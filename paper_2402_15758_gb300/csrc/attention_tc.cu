@@ -215,41 +215,34 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  // ---- KV staging (one thread of the loader warp): K or V of tile t into stage st as
-  // 4 pages x KP planes x 2 swizzle atoms of 16 rows; pages at or past kend are
-  // requested out of bounds (zero fill) ----
-  const bool loader = warp == SOFT_WARPS && lane == 0;
+  // ---- KV staging (the loader warp, all lanes together): K or V of tile t into stage st
+  // as 4 pages x KP planes x 2 swizzle atoms of 16 rows, one box per lane; pages at or
+  // past kend are requested out of bounds (zero fill). One thread issues a box only every
+  // ~70 ns, so the 8 KP boxes of a half go out from as many lanes at once. ----
   const long long rows_per_layer = p.pool_layer_stride / HD;
   auto issue_half = [&](int t, int st, int kend, bool is_v) {
     uint64_t* bar = is_v ? &v_full[st] : &k_full[st];
-    mbar_arrive_expect_tx(bar, static_cast<uint32_t>(HALF_BYTES));
-    uint8_t* base = (is_v ? vbuf : kbuf) + st * HALF_BYTES;
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
+    if (lane == 0) mbar_arrive_expect_tx(bar, static_cast<uint32_t>(HALF_BYTES));
+    __syncwarp();
+    if (lane < 8 * KP) {
+      const int u = lane / (2 * KP), plane = (lane >> 1) % KP, a = lane & 1;
       const int kg = t * KT + u * 16;
-      long long y0 = p.pool_rows;  // out of bounds
+      long long y = p.pool_rows;  // out of bounds
       if (kg < kend) {
         const int page = cached ? s_pages[(t - t0) * 4 + u] : p.page_table[b * p.max_pages + t * 4 + u];
-        y0 = static_cast<long long>(p.layer) * rows_per_layer + ((static_cast<long long>(page) * p.H + h) * NP +
-                                                                  (is_v ? KP : 0)) * 16;
+        y = static_cast<long long>(p.layer) * rows_per_layer +
+            ((static_cast<long long>(page) * p.H + h) * NP + (is_v ? KP : 0) + plane) * 16;
       }
-#pragma unroll
-      for (int plane = 0; plane < KP; ++plane) {
-        const long long y = y0 < p.pool_rows ? y0 + plane * 16 : p.pool_rows;
-#pragma unroll
-        for (int a = 0; a < 2; ++a)
-          tma_load_2d(base + plane * TILE64 + a * ATOM_ROWS64 + u * 16 * 128, &args.kv_map, a * 64,
-                      static_cast<int>(y), bar);
-      }
+      uint8_t* base = (is_v ? vbuf : kbuf) + st * HALF_BYTES;
+      tma_load_2d(base + plane * TILE64 + a * ATOM_ROWS64 + u * 16 * 128, &args.kv_map, a * 64,
+                  static_cast<int>(y), bar);
     }
   };
 
-  // L2 prefetch of tile t's page-planes (4 KB each, contiguous), ahead of the ring
+  // L2 prefetch of tile t's page-planes (NP x 4 KB, contiguous per page), one page per lane
   auto prefetch_tile = [&](int t, int kend) {
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      if (t * KT + u * 16 >= kend) break;
-      const int page = cached ? s_pages[(t - t0) * 4 + u] : p.page_table[b * p.max_pages + t * 4 + u];
+    if (lane < 4 && t * KT + lane * 16 < kend) {
+      const int page = cached ? s_pages[(t - t0) * 4 + lane] : p.page_table[b * p.max_pages + t * 4 + lane];
       const bf16* src = pool + (static_cast<size_t>(page) * p.H + h) * NP * 16 * HD;
       prefetch_l2_bulk(src, NP * 16 * HD * 2);
     }
@@ -258,8 +251,9 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
 
   int pre = 0;  // leading tiles (K and V) requested before the dependency wait
   if (p.prewait_kv) {
-    if (loader) {
-      prefetch_tensormap(&args.kv_map);
+    if (warp == SOFT_WARPS) {
+      if (lane == 0) prefetch_tensormap(&args.kv_map);
+      __syncwarp();
       while (pre < nt && pre < STAGES && (t0 + pre + 1) * KT <= nctx) {
         issue_half(t0 + pre, pre, nctx, false);
         issue_half(t0 + pre, pre, nctx, true);
@@ -372,40 +366,53 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
   if (threadIdx.x == 0) TTRACE(2);
 
   if (warp == SOFT_WARPS) {
-    // ---------------- KV loader (lane 0; the other lanes idle) ----------------
-   if (loader) {
-    if (!p.prewait_kv) prefetch_tensormap(&args.kv_map);
+    // ---------------- KV loader (the whole warp; lane 0 polls and decides) ----------------
+    if (!p.prewait_kv && lane == 0) prefetch_tensormap(&args.kv_map);
+    __syncwarp();
     // K of tile j needs the QK product of tile j - 2 done, V of tile j the PV product
     // of tile j - 2; both are polled so that neither waits behind the other
     int nk = pre, nv = pre;
     uint64_t last_progress = global_timer_ns();
-    while ((nk < nt || nv < nt) && !*abort) {
+    while (nk < nt || nv < nt) {
       bool moved = false;
-      if (nk < nt && (nk < STAGES || mbar_test(&k_empty[nk & 1], ((nk - STAGES) >> 1) & 1))) {
-        if (nk == 10) TTRACE(16);
+      const int kgo = __shfl_sync(0xffffffffu, (lane == 0 && nk < nt &&
+                                                (nk < STAGES || mbar_test(&k_empty[nk & 1], ((nk - STAGES) >> 1) & 1))) ? 1 : 0, 0);
+      if (kgo) {
+        if (lane == 0 && nk == 10) TTRACE(16);
+        if (lane == 0 && nk == 11) TTRACE(23);
         issue_half(t0 + nk, nk & 1, total, false);
+        if (lane == 0 && nk == 10) TTRACE(30);
         for (pf = max(pf, nk + 1); pf < nt && pf <= nk + L2_AHEAD; ++pf) prefetch_tile(t0 + pf, total);
+        if (lane == 0 && nk == 10) TTRACE(3);
+        if (lane == 0 && nk == 11) TTRACE(15);
         ++nk;
         moved = true;
       }
-      if (nv < nk && (nv < STAGES || mbar_test(&v_empty[nv & 1], ((nv - STAGES) >> 1) & 1))) {
-        if (nv == 10) TTRACE(17);
+      const int vgo = __shfl_sync(0xffffffffu, (lane == 0 && nv < nk &&
+                                                (nv < STAGES || mbar_test(&v_empty[nv & 1], ((nv - STAGES) >> 1) & 1))) ? 1 : 0, 0);
+      if (vgo) {
+        if (lane == 0 && nv == 10) TTRACE(17);
         issue_half(t0 + nv, nv & 1, total, true);
+        if (lane == 0 && nv == 10) TTRACE(31);
         ++nv;
         moved = true;
       }
-      if (moved) {
-        last_progress = global_timer_ns();
-      } else if (global_timer_ns() - last_progress > 2000000000ull) {
-        *abort = 1;
+      int quit = 0;
+      if (lane == 0) {
+        if (moved)
+          last_progress = global_timer_ns();
+        else if (global_timer_ns() - last_progress > 2000000000ull)
+          *abort = 1;
+        quit = *abort;
       }
+      if (__shfl_sync(0xffffffffu, quit, 0)) break;
     }
     // copies still in flight when the CTA gives up: let them land before it exits
-    if (*abort) {
+    if (lane == 0 && *abort) {
       for (int j = nk - 1; j >= 0 && j >= nk - STAGES; --j) mbar_wait_plain(&k_full[j & 1], (j >> 1) & 1, 200000000ull);
       for (int j = nv - 1; j >= 0 && j >= nv - STAGES; --j) mbar_wait_plain(&v_full[j & 1], (j >> 1) & 1, 200000000ull);
     }
-   }
+    __syncwarp();
   } else if (warp == MMA_WARP) {
     // ---------------- MMA issuer ----------------
     if (lane == 0 && nt > 0) {
