@@ -63,7 +63,7 @@ typedef struct {
   int dtype;            /* 0 = fp32, 1 = bf16 */
   float rms_eps;        /* RMSNorm epsilon (1e-6) */
   float rope_theta;     /* RoPE base (10000) */
-  int n_draft_heads;    /* K, 1..8 */
+  int n_draft_heads;    /* K, 1..4 */
   int tree_nodes;       /* N including the root, 2..64 */
   int topk[8];          /* rank limit per head (1..8); the tree draws ranks < topk[k] */
   int max_batch;        /* sequences per context, 1..64 */
@@ -105,7 +105,10 @@ typedef struct {
 /* Create a context.  `cuda_stream` is a cudaStream_t (NULL: the context creates its
  * own non-blocking stream).  Validates shapes, records the weight pointers and
  * allocates the KV pools (max_batch * max_seq_len slots), scratch and the tree.
- * EINVAL on bad shapes or a NULL weight, ENOMEM on allocation failure. */
+ * It synchronizes the device first, so weights written by earlier work on any stream
+ * are complete before the context reads them; the weights must not change while the
+ * context lives.  EINVAL on bad shapes or a NULL weight, ENOMEM on allocation failure,
+ * ECUDA when the device reports an earlier error. */
 chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
                             void* cuda_stream, chimera_ctx** out);
 

@@ -857,6 +857,12 @@ chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
   ctx->tri_w2 = w->tri_w2;
   ctx->heads.assign(w->heads, w->heads + c.n_draft_heads);
   ctx->num_sms = tc_num_sms();
+  // the weights may have been written on any stream (an own stream is not ordered after
+  // them): let every earlier piece of device work finish before this context reads them
+  if (cudaDeviceSynchronize() != cudaSuccess) {
+    free_ctx(ctx);
+    return CHIMERA_ECUDA;
+  }
 
   if (cuda_stream) {
     ctx->stream = static_cast<cudaStream_t>(cuda_stream);
