@@ -1,6 +1,8 @@
 // Kernel launches with programmatic stream serialization: a kernel may begin launching
 // while its predecessor in the stream drains; every kernel of the library calls
-// pdl_wait() before it touches memory written by earlier kernels.
+// pdl_wait() before it touches memory written by earlier kernels.  No kernel parameter
+// is `const T* __restrict__`: the compiler may treat loads through such a pointer as
+// invariant for the whole kernel and schedule them ahead of the wait.
 #pragma once
 
 #include <cuda_runtime.h>

@@ -11,9 +11,9 @@ namespace {
 constexpr int MT = 16;
 constexpr int WARPS = 8;
 
-__global__ void __launch_bounds__(WARPS * 32) f32_linear_kernel(const float* __restrict__ X, int ldx,
-                                                             const float* __restrict__ W,
-                                                             float* __restrict__ Y, int ldy, int M,
+__global__ void __launch_bounds__(WARPS * 32) f32_linear_kernel(const float* X, int ldx,
+                                                             const float* W,
+                                                             float* Y, int ldy, int M,
                                                              int N, int K, int epi) {
   pdl_trigger();  // the next kernel may start its prologue
   pdl_wait();     // inputs of this kernel are complete

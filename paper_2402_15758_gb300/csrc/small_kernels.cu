@@ -58,12 +58,19 @@ __device__ __forceinline__ float4 load_g4<bf16>(const bf16* g, int i) {
 
 // One block per row; every thread loads its (<= NORM_VEC) float4 of the row at once.
 template <typename T>
-__global__ void __launch_bounds__(NORM_THREADS) rmsnorm_kernel(const float* __restrict__ X, int ldx,
-                                                               const T* __restrict__ g, T* __restrict__ Y,
-                                                               T* __restrict__ Y_lo, float* __restrict__ Y32,
-                                                               int ldy, int d, float eps, float* __restrict__ Z,
+__global__ void __launch_bounds__(NORM_THREADS) rmsnorm_kernel(const float* X, int ldx,
+                                                               const T* g, T* Y,
+                                                               T* Y_lo, float* Y32,
+                                                               int ldy, int d, float eps, float* Z,
                                                                int ldz, int zcols) {
   pdl_trigger();  // the next kernel may start its prologue
+  // the gains are weights (never written by a kernel): load them before the wait
+  float4 gg[NORM_VEC];
+#pragma unroll
+  for (int k = 0; k < NORM_VEC; ++k) {
+    const int i = (threadIdx.x + k * NORM_THREADS) * 4;
+    gg[k] = i < d ? load_g4(g, i) : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
   pdl_wait();     // inputs of this kernel are complete
   __shared__ float red[33];
   const float* x = X + static_cast<size_t>(blockIdx.x) * ldx;
@@ -87,8 +94,8 @@ __global__ void __launch_bounds__(NORM_THREADS) rmsnorm_kernel(const float* __re
   for (int k = 0; k < NORM_VEC; ++k) {
     const int i = (threadIdx.x + k * NORM_THREADS) * 4;
     if (i < d) {
-      const float4 gg = load_g4(g, i);
-      const float4 y = make_float4(v[k].x * r * gg.x, v[k].y * r * gg.y, v[k].z * r * gg.z, v[k].w * r * gg.w);
+      const float4 y = make_float4(v[k].x * r * gg[k].x, v[k].y * r * gg[k].y, v[k].z * r * gg[k].z,
+                                   v[k].w * r * gg[k].w);
       store_act4(Y, Y_lo, row + i, y);
       if (Y32) *reinterpret_cast<float4*>(Y32 + row + i) = y;
     }
@@ -172,8 +179,8 @@ __global__ void rope_kv_kernel(const RopeKvParams p) {
 
 // SwiGLU: h = SiLU(gate) * up, gate in columns [0, F), up in [F, 2F).
 template <typename T>
-__global__ void swiglu_kernel(const float* __restrict__ gu, int ldgu, int F, T* __restrict__ h,
-                              T* __restrict__ h_lo, int ldh) {
+__global__ void swiglu_kernel(const float* gu, int ldgu, int F, T* h,
+                              T* h_lo, int ldh) {
   pdl_trigger();  // the next kernel may start its prologue
   pdl_wait();     // inputs of this kernel are complete
   const float* g = gu + static_cast<size_t>(blockIdx.y) * ldgu;
@@ -186,7 +193,7 @@ __global__ void swiglu_kernel(const float* __restrict__ gu, int ldgu, int F, T* 
 }
 
 template <typename T>
-__global__ void embed_kernel(const T* __restrict__ E, int d, int V, float* __restrict__ x,
+__global__ void embed_kernel(const T* E, int d, int V, float* x,
                              int rows_per_seq, const int* tokens, const int* tok_hist,
                              int hist_stride, const int* n, const int* valid, int* err) {
   pdl_trigger();  // the next kernel may start its prologue
@@ -213,7 +220,7 @@ __device__ __forceinline__ bool better(float v, int i, float bv, int bi) {
   return v > bv || (v == bv && i < bi);
 }
 
-__global__ void __launch_bounds__(512) argmax_kernel(const float* __restrict__ logits, int V, int* __restrict__ out) {
+__global__ void __launch_bounds__(512) argmax_kernel(const float* logits, int V, int* out) {
   pdl_trigger();  // the next kernel may start its prologue
   pdl_wait();     // inputs of this kernel are complete
   __shared__ float sv[32];
@@ -354,10 +361,10 @@ __device__ void topk_block_select(float (&lv)[TOPK_MAX], int (&li)[TOPK_MAX], in
   }
 }
 
-__global__ void __launch_bounds__(TOPK_THREADS) topk_kernel(const float* __restrict__ logits, int V, int k,
-                                                            int* __restrict__ idx, float* __restrict__ val,
-                                                            int out_stride, float* __restrict__ ws_v,
-                                                            int* __restrict__ ws_i, int* __restrict__ counters) {
+__global__ void __launch_bounds__(TOPK_THREADS) topk_kernel(const float* logits, int V, int k,
+                                                            int* idx, float* val,
+                                                            int out_stride, float* ws_v,
+                                                            int* ws_i, int* counters) {
   pdl_trigger();  // the next kernel may start its prologue
   pdl_wait();     // inputs of this kernel are complete
   __shared__ float s_bv[TOPK_MAX];

@@ -12,9 +12,9 @@ namespace {
 // A position before the start of the sequence contributes a zero block.
 // Also zeroes row b of `zero` (d floats): the draft residual that W2 accumulates into.
 template <typename T>
-__global__ void trigram_gather_kernel(const T* __restrict__ E, int d, int V, const int* n_arr,
+__global__ void trigram_gather_kernel(const T* E, int d, int V, const int* n_arr,
                                       const int* tok, int tok_stride, const int* topk, int K,
-                                      int KMAX, int k, T* __restrict__ out, int* err, float* __restrict__ zero) {
+                                      int KMAX, int k, T* out, int* err, float* zero) {
   pdl_trigger();  // the next kernel may start its prologue
   pdl_wait();     // inputs of this kernel are complete
   const int b = blockIdx.x;
@@ -42,9 +42,9 @@ __global__ void trigram_gather_kernel(const T* __restrict__ E, int d, int V, con
 // headin[b][d..2d) = h_full (the draft block output), kept per head for debugging;
 // also zeroes row b of the head's score buffer (V floats) that its linear accumulates into.
 template <typename T>
-__global__ void hfull_store_kernel(const float* __restrict__ dres, int d, T* __restrict__ headin,
-                                   T* __restrict__ headin_lo, float* __restrict__ hlog,
-                                   float* __restrict__ zero, int V) {
+__global__ void hfull_store_kernel(const float* dres, int d, T* headin,
+                                   T* headin_lo, float* hlog,
+                                   float* zero, int V) {
   pdl_trigger();  // the next kernel may start its prologue
   pdl_wait();     // inputs of this kernel are complete
   const int b = blockIdx.x;
@@ -147,9 +147,9 @@ __global__ void compact_kernel(char* pool, long long layer_stride_bytes, int H, 
 // hsel[b][j] = verify hidden (fp32) of path node j (j <= L; later rows repeat the
 // last); headin[b][0..d) = hidden of the last accepted node (h_LLM of the new prefix end).
 template <typename T>
-__global__ void gather_hidden_kernel(const float* __restrict__ hfin, int d, int N, const int* path,
-                                     const int* Lacc, int D1, float* __restrict__ hsel,
-                                     T* __restrict__ headin, T* __restrict__ headin_lo) {
+__global__ void gather_hidden_kernel(const float* hfin, int d, int N, const int* path,
+                                     const int* Lacc, int D1, float* hsel,
+                                     T* headin, T* headin_lo) {
   pdl_trigger();  // the next kernel may start its prologue
   pdl_wait();     // inputs of this kernel are complete
   const int b = blockIdx.x, j = blockIdx.y;
@@ -185,9 +185,9 @@ __global__ void finalize_kernel(int* n_arr, int* tok, int tok_stride, const int*
 
 // Prefill chunk bookkeeping: keep h_LLM of the last prompt row, advance n.
 template <typename T>
-__global__ void prefill_advance_kernel(const float* __restrict__ hfin, int d, int rows_per_seq,
+__global__ void prefill_advance_kernel(const float* hfin, int d, int rows_per_seq,
                                        const int* valid, const int* last, int* n_arr,
-                                       T* __restrict__ headin, T* __restrict__ headin_lo) {
+                                       T* headin, T* headin_lo) {
   pdl_trigger();  // the next kernel may start its prologue
   pdl_wait();     // inputs of this kernel are complete
   const int b = blockIdx.x;
