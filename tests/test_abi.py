@@ -33,3 +33,20 @@ def test_init_rejects_bad_config_without_touching_the_gpu(lib_path):
     assert lib.chimera_init(ctypes.byref(c), None, None, ctypes.byref(h)) == -1
     assert lib.chimera_init(None, None, None, None) == -1
     assert not h.value
+
+
+def test_no_restrict_pointer_in_dependent_launch_kernels():
+    """Every kernel is launched with programmatic dependent launch and reads its inputs
+    only after griddepcontrol.wait.  A `__restrict__` parameter would let the compiler
+    treat its loads as invariant and schedule them ahead of that wait (an fp32 prefill
+    read a stale residual this way), so no kernel source may declare one."""
+    csrc = os.path.join(os.path.dirname(pkg.__file__), "csrc")
+    offenders = []
+    for name in sorted(os.listdir(csrc)):
+        if name.endswith((".cu", ".cuh", ".h")):
+            with open(os.path.join(csrc, name)) as f:
+                for i, line in enumerate(f, 1):
+                    code = line.split("//")[0]
+                    if "__restrict__" in code:
+                        offenders.append(f"{name}:{i}")
+    assert not offenders, offenders
