@@ -47,6 +47,23 @@ def peaks():
     return 6800.0, "fallback"
 
 
+def max_over_ranks(x: float, world: int) -> float:
+    """The largest x over the ranks: a job's time is its slowest replica's."""
+    if world <= 1:
+        return x
+    import torch.distributed as dist
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rate(units_per_rank: float, world: int, ms_job: float) -> float:
+    """Units per second of the whole job: every replica processes units_per_rank in
+    ms_job (the max over ranks)."""
+    return world * units_per_rank / (ms_job * 1e-3)
+
+
 def step_bytes(cfg, n_ctx, kv_elem_bytes=None):
     """Algorithmic HBM bytes of one step at committed length n_ctx (batch 1).
 
@@ -298,12 +315,8 @@ def main():
     torch.cuda.nvtx.range_pop()
     ctx.sync()
     torch.cuda.synchronize()
-    ms = e0.elapsed_time(e1) / args.steps
+    ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, world)
     clk = clocks.stop()
-    if world > 1:
-        t = torch.tensor([ms], device="cuda")
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms = float(t.item())
     n1 = int(ctx.read("n")[0])
     mean_accept = (n1 - n0) / args.steps
 
@@ -333,17 +346,19 @@ def main():
 
     # ---- end to end through chimera_step (host outputs, one sync per step) ----
     ctx.sync()
+    if world > 1:
+        torch.distributed.barrier()
     t0 = time.perf_counter()
     emitted = 0
     for _ in range(args.steps):
         out = ctx.step()
         emitted += sum(len(o) for o in out)
-    t_e2e = (time.perf_counter() - t0) / args.steps
+    t_e2e = max_over_ranks((time.perf_counter() - t0) / args.steps, world)
     d2h = B * 4 + 4 + int(round(4 * emitted / args.steps))
 
     hbm, peak_kind = peaks()
     nb = step_bytes(cfg, (n0 + n1) // 2, kv_elem_bytes=4 if ctx.kv_f32 else None)
-    value = world * B * N / (ms * 1e-3)
+    value = job_rate(B * N, world, ms)
     if lin_ms <= 0:
         raise RuntimeError("per-kernel profile returned no linear time")
     lin_gbs = lin_bytes / (lin_ms * 1e-3) / 1e9
@@ -382,7 +397,7 @@ def main():
                      "traffic_basis": "DRAM bytes read + written by all linear launches of one step (ncu)",
                      "launches_per_step": lin_n, "bytes_per_step": lin_bytes, "ms_per_step": lin_ms},
         "cpu_baseline": cpu,
-        "e2e": {"value": world * B * N / t_e2e, "unit": "tree tokens/s", "h2d_bytes_per_step": 0,
+        "e2e": {"value": job_rate(B * N, world, t_e2e * 1e3), "unit": "tree tokens/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": d2h, "ms_per_step": t_e2e * 1e3},
         "gpu_launches": launches * args.steps,
         "clocks": clk,
