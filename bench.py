@@ -293,7 +293,7 @@ def main():
 
     w = synth.make_weights(cfg, device="cuda")
     torch.cuda.synchronize()
-    total_steps = args.warmup + args.steps + args.profile_steps + args.steps + 8
+    total_steps = args.warmup + 2 * args.steps + args.profile_steps + args.steps + 8
     max_seq = ((len(prompt) + total_steps * 5 + N + 64 + 15) // 16) * 16
     stream = torch.cuda.Stream()
     ctx = pkg.Chimera(cfg, w, max_batch=B, max_seq_len=max_seq, stream=stream)
@@ -319,6 +319,18 @@ def main():
     clk = clocks.stop()
     n1 = int(ctx.read("n")[0])
     mean_accept = (n1 - n0) / args.steps
+
+    # ---- per-step distribution: one event pair around each graph replay ----
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    ev[0].record(stream)
+    for i in range(args.steps):
+        ctx.step_async(1)
+        ev[i + 1].record(stream)
+    ctx.sync()
+    torch.cuda.synchronize()
+    per_step = sorted(ev[i].elapsed_time(ev[i + 1]) for i in range(args.steps))
+    step_median = max_over_ranks(statistics.median(per_step), world)
+    step_p90 = max_over_ranks(per_step[min(len(per_step) - 1, int(round(0.9 * (len(per_step) - 1))))], world)
 
     # ---- per-kernel timing (eager launches with events around each) ----
     recs = []
@@ -383,6 +395,7 @@ def main():
         "breakdown": {
             "verify_ms_eager": phase_ms["verify"], "draft_ms_eager": phase_ms["draft"],
             "commit_ms_eager": phase_ms["commit"], "step_ms_eager": eager_ms,
+            "step_ms_median": step_median, "step_ms_p90": step_p90,
             "kernel_ms_by_kind": {k: round(v, 4) for k, v in sorted(kind_ms.items(), key=lambda t: -t[1])},
             "step_bytes_gb": nb["total"] / 1e9, "verify_bytes_gb": nb["verify"] / 1e9,
             "achieved_step_gbs": nb["total"] / (ms * 1e-3) / 1e9,
