@@ -147,6 +147,11 @@ def block_rows(W: OracleWeights, prefix: str, cfg: dict, x: np.ndarray, pos: np.
     Every row sees all context keys ctx_k/ctx_v[m][H][hd] (already rotated) and the
     local rows j with local_mask[i][j].  Returns (out[R][d], k_local, v_local) where
     k_local is rotated.
+
+    The attention of row i is the softmax over its visible keys (all m context keys,
+    then the visible local rows), written as one score row per (head, query) over the
+    union [context ; local] with the invisible local keys at -inf.  The key rows are
+    never copied, so a context of many thousand rows costs one score matrix per call.
     """
     H, hd, eps, th = cfg["n_heads"], cfg["head_dim"], cfg["rms_eps"], cfg["rope_theta"]
     R, d = x.shape
@@ -155,12 +160,17 @@ def block_rows(W: OracleWeights, prefix: str, cfg: dict, x: np.ndarray, pos: np.
     q = rope(qkv[:, :d].reshape(R, H, hd), pos, th)
     k = rope(qkv[:, d:2 * d].reshape(R, H, hd), pos, th)
     v = qkv[:, 2 * d:].reshape(R, H, hd)
-    att = np.empty((R, H, hd))
-    for i in range(R):
-        sel = np.nonzero(local_mask[i])[0]
-        kk = np.concatenate([ctx_k, k[sel]], axis=0)
-        vv = np.concatenate([ctx_v, v[sel]], axis=0)
-        att[i] = attend(q[i], kk, vv)
+    qh = q.transpose(1, 0, 2)                                   # [H][R][hd]
+    s_ctx = qh @ ctx_k.transpose(1, 2, 0)                      # [H][R][m]
+    s_loc = qh @ k.transpose(1, 2, 0)                          # [H][R][R]
+    s_loc = np.where(np.asarray(local_mask, dtype=bool)[None], s_loc, -np.inf)
+    s = np.concatenate([s_ctx, s_loc], axis=-1) / np.sqrt(hd)
+    s = s - s.max(axis=-1, keepdims=True)
+    p = np.exp(s)
+    p = p / p.sum(axis=-1, keepdims=True)
+    m = ctx_k.shape[0]
+    att = p[..., :m] @ ctx_v.transpose(1, 0, 2) + p[..., m:] @ v.transpose(1, 0, 2)  # [H][R][hd]
+    att = att.transpose(1, 0, 2)
     x = x + att.reshape(R, d) @ W(f"{prefix}.wo").T
     h2 = rmsnorm(x, W(f"{prefix}.ffn_norm"), eps)
     ffn = silu(h2 @ W(f"{prefix}.w_gate").T) * (h2 @ W(f"{prefix}.w_up").T)
@@ -243,18 +253,29 @@ def draft_kv_rows(W: OracleWeights, cfg: dict, hs: np.ndarray, pos: np.ndarray):
     return rope(k, pos, cfg["rope_theta"]), v
 
 
-def prefill(W: OracleWeights, cfg: dict, prompt: list[int], cap: int) -> SeqState:
+def prefill(W: OracleWeights, cfg: dict, prompt: list[int], cap: int, chunk: int | None = None) -> SeqState:
     """Causal forward over the prompt; fills base KV, H_LLM and draft KV; the root is
-    the greedy next token (eq. 1)."""
+    the greedy next token (eq. 1).
+
+    With `chunk`, each layer takes the prompt `chunk` rows at a time: the rows of a
+    chunk attend the keys of all earlier rows of that layer (already computed) plus
+    the causal part of their own chunk, which is the same causal attention as one
+    pass over the whole prompt (every row's softmax still runs over positions
+    0..itself); only the score matrices get smaller, so long prompts fit in memory."""
     R = len(prompt)
     st = SeqState(cfg, cap)
     x = W.rows("embed", prompt)
     pos = np.arange(R)
-    causal = np.tril(np.ones((R, R), dtype=bool))
-    empty = np.zeros((0, cfg["n_heads"], cfg["head_dim"]))
+    C = R if not chunk else int(chunk)
     for l in range(cfg["n_layers"]):
-        x, k, v = block_rows(W, f"layers.{l}", cfg, x, pos, empty, empty, causal)
-        st.K[l, :R], st.V[l, :R] = k, v
+        xs = []
+        for a in range(0, R, C):
+            b = min(R, a + C)
+            causal = np.tril(np.ones((b - a, b - a), dtype=bool))
+            xo, k, v = block_rows(W, f"layers.{l}", cfg, x[a:b], pos[a:b], st.K[l, :a], st.V[l, :a], causal)
+            st.K[l, a:b], st.V[l, a:b] = k, v
+            xs.append(xo)
+        x = np.concatenate(xs, axis=0)
     hs = rmsnorm(x, W("final_norm"), cfg["rms_eps"])
     st.Hs[:R] = hs
     st.dK[:R], st.dV[:R] = draft_kv_rows(W, cfg, hs, pos)

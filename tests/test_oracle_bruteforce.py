@@ -109,3 +109,46 @@ def _force_branch(t, ar, L, V):
         on_branch = all(r == 0 for r in t["nodes"][i])
         toks[i] = want if (on_branch and dep <= L) else (want + 1 + t["rank"][i]) % V
     return toks
+
+
+def test_block_rows_attention_equals_per_row_key_lists(small):
+    # block_rows scores each query against [context ; local] at once; the same rows,
+    # attended one at a time over an explicit list of their visible keys (attend),
+    # must give the same block output
+    cfg, W, _ = small
+    H, hd, d = cfg["n_heads"], cfg["head_dim"], cfg["d_model"]
+    rng = np.random.default_rng(21)
+    R, m = 6, 9
+    x = rng.standard_normal((R, d))
+    pos = np.array([9, 10, 10, 11, 11, 12])
+    ctx_k, ctx_v = rng.standard_normal((m, H, hd)), rng.standard_normal((m, H, hd))
+    parent = [-1, 0, 0, 1, 2, 3]
+    mask = np.zeros((R, R), dtype=bool)
+    for i in range(R):
+        j = i
+        while j >= 0:
+            mask[i, j] = True
+            j = parent[j]
+    out, k, v = co.block_rows(W, "layers.0", cfg, x, pos, ctx_k, ctx_v, mask)
+    p = "layers.0"
+    h = co.rmsnorm(x, W(f"{p}.attn_norm"), cfg["rms_eps"])
+    q = co.rope((h @ W(f"{p}.wqkv").T)[:, :d].reshape(R, H, hd), pos, cfg["rope_theta"])
+    att = np.stack([co.attend(q[i], np.concatenate([ctx_k, k[mask[i]]]), np.concatenate([ctx_v, v[mask[i]]]))
+                    for i in range(R)])
+    x1 = x + att.reshape(R, d) @ W(f"{p}.wo").T
+    h2 = co.rmsnorm(x1, W(f"{p}.ffn_norm"), cfg["rms_eps"])
+    ref = x1 + (co.silu(h2 @ W(f"{p}.w_gate").T) * (h2 @ W(f"{p}.w_up").T)) @ W(f"{p}.w_down").T
+    np.testing.assert_allclose(out, ref, rtol=1e-12, atol=1e-12)
+
+
+@pytest.mark.parametrize("chunk", [1, 4, 5])
+def test_chunked_prefill_equals_one_pass(small, chunk):
+    cfg, W, prompt = small
+    a = co.prefill(W, cfg, prompt, 64)
+    b = co.prefill(W, cfg, prompt, 64, chunk=chunk)
+    n = len(prompt)
+    assert a.tokens == b.tokens
+    np.testing.assert_allclose(b.K[:, :n], a.K[:, :n], rtol=1e-11, atol=1e-12)
+    np.testing.assert_allclose(b.V[:, :n], a.V[:, :n], rtol=1e-11, atol=1e-12)
+    np.testing.assert_allclose(b.Hs[:n], a.Hs[:n], rtol=1e-11, atol=1e-12)
+    np.testing.assert_allclose(b.prefill_logits, a.prefill_logits, rtol=1e-11, atol=1e-12)
