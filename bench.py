@@ -32,10 +32,6 @@ import torch  # noqa: E402
 import synth  # noqa: E402
 
 WORKLOAD = "7b"
-# dram__bytes_read.sum + dram__bytes_write.sum of the 158 linear launches of one step of
-# this workload (ncu, one pass, see profiles/step_7b_bs1_launch_list.md); against the
-# 17.53 GB of weights they stream, 4 % more (the fp32 outputs read by the reductions).
-# Must be re-measured (or set to None) whenever the linear kernel changes.
 LINEAR_DRAM_BYTES_PER_STEP = 18.23e9
 
 

@@ -210,7 +210,10 @@ chimera_status chimera_debug_read_kv(chimera_ctx* ctx, int layer, int seq, int p
  * dtype 1: X, X_lo (optional, NULL = none), W bf16 (K, ldx multiples of 8; 16-byte
  * aligned), tcgen05 kernel; dtype 0: everything fp32, X_lo ignored.  epi 0: Y = acc,
  * 1: Y = SiLU(acc), 2: Y(fp32) += acc.  out_f32 selects an fp32 Y for epi 0/1 with
- * dtype 1.  Device pointers.  Uses a per-process workspace allocated on first use. */
+ * dtype 1.  Device pointers.  Uses a workspace per device, allocated on the first call
+ * made with that device current.  Asynchronous: the status covers the arguments and
+ * the launch; what the kernel flags on the device (a bounded wait that gave up) is
+ * reported by chimera_op_sync. */
 chimera_status chimera_op_linear(int dtype, int epi, int out_f32, int M, int N, int K,
                                  const void* X, const void* X_lo, int ldx, const void* W, void* Y,
                                  int ldy, void* cuda_stream);
@@ -233,6 +236,23 @@ chimera_status chimera_op_attention(int dtype, int kv_split, int batch, int n_he
                                     int max_pages, const int32_t* n_ctx, const uint64_t* anc,
                                     void* out, void* out_lo, int ldo, int splits, void* cuda_stream);
 
+/* Wait until `cuda_stream` (NULL: the default stream) is idle, then read and clear the
+ * device error words of the stateless entry points (chimera_op_linear,
+ * chimera_op_attention, chimera_op_linear_noalloc) on the current device: everything
+ * their kernels flagged since the previous chimera_op_sync.  CHIMERA_ETIMEDOUT when a
+ * bounded wait gave up (the outputs of those calls are undefined; the split counters
+ * of the workspaces are reset, so later calls compute correctly again),
+ * CHIMERA_ECAPACITY / CHIMERA_EINVAL for an out-of-range slot or index, CHIMERA_ECUDA
+ * when a CUDA call fails, else CHIMERA_OK. */
+chimera_status chimera_op_sync(void* cuda_stream);
+
+/* Test hook: limit (ns) of every bounded wait of the tensor-core linear launched by the
+ * stateless entry points from now on (0 restores the default of 2 s).  Contexts always
+ * use the default.  A limit of a few ns makes the waits give up, which exercises the
+ * kernel's clean exit (in-flight copies and MMAs drained, tensor memory freed) and the
+ * CHIMERA_ETIMEDOUT report of chimera_op_sync without any fault. */
+chimera_status chimera_debug_set_wait_limit(uint64_t ns);
+
 /* Same computation as chimera_op_linear with dtype 1 (bf16, tcgen05), but it allocates
  * nothing: for callers that cannot allocate device memory when they call (code running
  * under a fixed per-process memory budget, inside host callbacks or allocator hooks,
@@ -244,7 +264,8 @@ chimera_status chimera_op_attention(int dtype, int kv_split, int batch, int n_he
  * the arrays' device addresses (make that first call outside any stream capture).
  * Every call shares the arrays and keeps the last call's contents; the call clears
  * what must start at zero.  Calls that overlap on the GPU race on the scratch: the
- * caller serialises them (one stream, or explicit synchronisation). */
+ * caller serialises them (one stream, or explicit synchronisation).  A bounded wait
+ * that gives up inside the kernel is reported by the next chimera_op_sync. */
 chimera_status chimera_op_linear_noalloc(int epi, int out_f32, int M, int N, int K, const void* X,
                                          const void* X_lo, int ldx, const void* W, void* Y, int ldy,
                                          void* cuda_stream);

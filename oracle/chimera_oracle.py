@@ -71,6 +71,11 @@ class OracleWeights:
             self._cache[name] = a
         return a
 
+    def subset(self, prefix: str) -> "OracleWeights":
+        """A caching view of the matrices whose names start with `prefix` (one layer):
+        each is up-cast once while the view lives (the prompt chunks of a layer)."""
+        return OracleWeights({k: v for k, v in self._src.items() if k.startswith(prefix)}, cache=True)
+
     def rows(self, name: str, idx) -> np.ndarray:
         """Selected rows of a matrix (the embedding gather), up-cast exactly."""
         t = self._src[name]
@@ -268,11 +273,12 @@ def prefill(W: OracleWeights, cfg: dict, prompt: list[int], cap: int, chunk: int
     pos = np.arange(R)
     C = R if not chunk else int(chunk)
     for l in range(cfg["n_layers"]):
+        Wl = W.subset(f"layers.{l}.") if C < R else W
         xs = []
         for a in range(0, R, C):
             b = min(R, a + C)
             causal = np.tril(np.ones((b - a, b - a), dtype=bool))
-            xo, k, v = block_rows(W, f"layers.{l}", cfg, x[a:b], pos[a:b], st.K[l, :a], st.V[l, :a], causal)
+            xo, k, v = block_rows(Wl, f"layers.{l}", cfg, x[a:b], pos[a:b], st.K[l, :a], st.V[l, :a], causal)
             st.K[l, a:b], st.V[l, a:b] = k, v
             xs.append(xo)
         x = np.concatenate(xs, axis=0)

@@ -77,6 +77,8 @@ _SIGS = {
     "chimera_op_linear_noalloc": (ctypes.c_int, [ctypes.c_int] * 5 + [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int,
                                                                       ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int,
                                                                       ctypes.c_void_p]),
+    "chimera_op_sync": (ctypes.c_int, [ctypes.c_void_p]),
+    "chimera_debug_set_wait_limit": (ctypes.c_int, [ctypes.c_uint64]),
     "chimera_op_attention": (ctypes.c_int, [ctypes.c_int] * 8 + [ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
                                                                  ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p,
                                                                  ctypes.c_int,
@@ -308,6 +310,19 @@ def op_attention(q, pool, page_table, n_ctx, anc, out, nq, q_local0, n_local, q_
                                   _stream_handle(stream))
     if st != 0:
         raise ChimeraError(st, "chimera_op_attention")
+
+
+def op_sync(stream=None):
+    """Wait for the stateless entry points' work and raise what their kernels flagged
+    on the device since the last call (ETIMEDOUT, EINVAL, ...)."""
+    st = load().chimera_op_sync(_stream_handle(stream))
+    if st != 0:
+        raise ChimeraError(st, "chimera_op_sync: the device flagged an error")
+
+
+def set_wait_limit(ns: int = 0):
+    """Test hook: bounded-wait limit of the stateless linear entry points (0: default)."""
+    load().chimera_debug_set_wait_limit(int(ns))
 
 
 def declared_symbols(header: str = HEADER) -> list[str]:

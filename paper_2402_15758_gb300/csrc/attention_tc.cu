@@ -135,13 +135,6 @@ __device__ __forceinline__ void split_pair(float a, float b, uint32_t& hi, uint3
 // Under the M = 64 data-path layout, query rows 16q .. 16q + 15 sit in TMEM lanes 0..15 of
 // sub-partition q (warp w reaches sub-partition w % 4).
 
-#ifdef CHIMERA_ATTN_TRACE
-// per-CTA timestamps of the last launch (instrumented builds only)
-__device__ unsigned long long g_atc_trace[2048][32];
-#define TTRACE(i) g_atc_trace[(blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x][i] = global_timer_ns()
-#else
-#define TTRACE(i)
-#endif
 
 template <bool SPLIT>
 __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_constant__ TcArgs args) {
@@ -197,7 +190,6 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
   }
   if (warp == MMA_WARP) tmem_alloc(tmem_slot, TMEM_COLS);
 
-  if (threadIdx.x == 0) TTRACE(0);
   if (!p.prewait_kv) pdl_wait();
   const int nctx = p.n_ctx[b];
   const int ntiles = (nctx + p.n_local + KT - 1) / KT;
@@ -265,7 +257,6 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
     pdl_wait();
   }
   pdl_trigger();
-  if (threadIdx.x == 0) TTRACE(1);
 
   const int nloc = min(p.n_local_dev ? p.n_local_dev[b] : p.n_local, p.n_local);
   const int nq = p.nq_dev ? p.nq_dev[b] : p.nq;
@@ -363,7 +354,6 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
   fence_async_smem();  // the Q tiles are read by the tensor cores (async proxy)
   __threadfence_block();
   __syncthreads();
-  if (threadIdx.x == 0) TTRACE(2);
 
   if (warp == SOFT_WARPS) {
     // ---------------- KV loader (the whole warp; lane 0 polls and decides) ----------------
@@ -378,22 +368,15 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
       const int kgo = __shfl_sync(0xffffffffu, (lane == 0 && nk < nt &&
                                                 (nk < STAGES || mbar_test(&k_empty[nk & 1], ((nk - STAGES) >> 1) & 1))) ? 1 : 0, 0);
       if (kgo) {
-        if (lane == 0 && nk == 10) TTRACE(16);
-        if (lane == 0 && nk == 11) TTRACE(23);
         issue_half(t0 + nk, nk & 1, total, false);
-        if (lane == 0 && nk == 10) TTRACE(30);
         for (pf = max(pf, nk + 1); pf < nt && pf <= nk + L2_AHEAD; ++pf) prefetch_tile(t0 + pf, total);
-        if (lane == 0 && nk == 10) TTRACE(3);
-        if (lane == 0 && nk == 11) TTRACE(15);
         ++nk;
         moved = true;
       }
       const int vgo = __shfl_sync(0xffffffffu, (lane == 0 && nv < nk &&
                                                 (nv < STAGES || mbar_test(&v_empty[nv & 1], ((nv - STAGES) >> 1) & 1))) ? 1 : 0, 0);
       if (vgo) {
-        if (lane == 0 && nv == 10) TTRACE(17);
         issue_half(t0 + nv, nv & 1, total, true);
-        if (lane == 0 && nv == 10) TTRACE(31);
         ++nv;
         moved = true;
       }
@@ -471,8 +454,6 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
         if (npv < nqk && mbar_test(&p_full[npv & 1], (npv >> 1) & 1) &&
             mbar_test(&v_full[npv & 1], (npv >> 1) & 1)) {
           tc_fence_after();
-          if (npv == 10) TTRACE(22);
-          if (npv == 9) TTRACE(25);
           pv(npv);
           ++npv;
           moved = true;
@@ -480,9 +461,6 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
         if (nqk < nt && nqk <= npv + 1 && mbar_test(&k_full[nqk & 1], (nqk >> 1) & 1) &&
             (nqk < 2 || mbar_test(&s_free[nqk & 1], ((nqk - 2) >> 1) & 1))) {
           tc_fence_after();
-          if (nqk == 0) TTRACE(5);
-          if (nqk == 10) TTRACE(19);
-          if (nqk == 12) TTRACE(24);
           qk(nqk);
           ++nqk;
           moved = true;
@@ -519,8 +497,6 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
       bool ok = !dead && mbar_wait(&s_full[sb], (i >> 1) & 1, abort);
       dead = !__all_sync(0xffffffffu, ok);
       tc_fence_after();
-      if (warp == 0 && lane == 0 && i == 10) TTRACE(20);
-      if (warp == 0 && lane == 0 && i == 0) TTRACE(6);
       float sv[16];
       if (!dead) {
         uint32_t rr[16];
@@ -529,7 +505,6 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
 #pragma unroll
         for (int j = 0; j < 16; ++j) sv[j] = __uint_as_float(rr[j]);
       }
-      if (warp == 0 && lane == 0 && i == 10) TTRACE(26);
       tc_fence_before();
       __syncwarp();
       if (lane == 0 && !dead) mbar_arrive(&s_free[sb]);
@@ -558,14 +533,12 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
       if (sub == 0) s_xm[(sb * 2 + half) * NQ + r] = tmax;
       named_bar(1 + quad, 64);
       tmax = fmaxf(tmax, s_xm[(sb * 2 + (half ^ 1)) * NQ + r]);
-      if (warp == 0 && lane == 0 && i == 10) TTRACE(27);
       // this tile's P buffer was read by the PV product of tile i - 2
       if (i >= 2) {
         ok = !dead && mbar_wait(&pv_done[i & 1], ((i - 2) >> 1) & 1, abort);
         dead = !__all_sync(0xffffffffu, ok);
         tc_fence_after();
       }
-      if (warp == 0 && lane == 0 && i == 10) TTRACE(28);
       // m moves only when the tile's maximum exceeds it by more than 2^RESCALE_LOG2; O then
       // holds products of earlier tiles exactly when m was already finite. Both decisions
       // depend only on the row's shared maxima, so all four lanes of a row agree.
@@ -625,10 +598,7 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
         }
       }
       l += ra + rb;
-      if (warp == 0 && lane == 0 && i == 10) TTRACE(21);
-      if (warp == 0 && lane == 0 && i == 0) TTRACE(7);
       fence_async_smem();
-      if (warp == 0 && lane == 0 && i == 10) TTRACE(29);
       tc_fence_before();
       __syncwarp();
       if (lane == 0 && !dead) mbar_arrive(&p_full[sb]);
@@ -646,10 +616,8 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
   // main loop (split cluster barrier) ----
   if (warp < SOFT_WARPS) {
     if (nt > 0) {
-      if (warp == 0 && lane == 0) TTRACE(14);
       mbar_wait(o_done, 0, abort);
       tc_fence_after();
-      if (warp == 0 && lane == 0) TTRACE(9);
     }
     __syncwarp();
   }
@@ -675,7 +643,6 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
     }
     __syncwarp();
     if (S > 1) cluster_wait();
-    if (threadIdx.x == 0) TTRACE(11);
     if (soft) {
       const int owner = mine ? r / rpc : 0;
       const uint32_t slot = smem_u32(recv + (s * rpc + (mine ? r - owner * rpc : 0)) * PREC);
@@ -706,9 +673,7 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
   }
   if (threadIdx.x == 0 && *abort && p.err) atomicOr(p.err, ERR_TIMEOUT);
   __syncwarp();
-  if (threadIdx.x == 0) TTRACE(12);
   if (S > 1) cluster_sync();  // every push into this CTA is complete and visible
-  if (threadIdx.x == 0) TTRACE(13);
 
   // ---- merge the S partials of this CTA's rows (local shared memory) ----
   bf16* out = static_cast<bf16*>(p.out);
@@ -750,7 +715,6 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
     store_act(out, out_lo, o_idx + 2, acc.z);
     store_act(out, out_lo, o_idx + 3, acc.w);
   }
-  if (threadIdx.x == 0) TTRACE(10);
 }
 
 template <bool SPLIT>
@@ -825,11 +789,6 @@ int tc_splits(int BH, int want) {
 
 }  // namespace
 
-#ifdef CHIMERA_ATTN_TRACE
-extern "C" int chimera_atc_trace(unsigned long long* host, int n) {
-  return cudaMemcpyFromSymbol(host, g_atc_trace, static_cast<size_t>(n) * 32 * 8) == cudaSuccess ? 0 : -1;
-}
-#endif
 
 cudaError_t attention_tc(const AttnParams& p, cudaStream_t s) {
   if (p.hd != HD || p.nq_max > NQ || p.n_local > 64 || p.splits < 1 || p.splits > 8) return cudaErrorInvalidValue;

@@ -5,6 +5,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 namespace chimera {
 
 // ----------------------------------------------------------------------------
@@ -31,9 +33,9 @@ struct TcLinearParams {
   float* ws;         // split partials: [grid][2][128 * BN] fp32
   int* counters;     // [feat_tiles * tok_tiles], all zero between launches
   int* err;          // device error word
+  unsigned long long wait_ns;  // limit of every bounded wait of the launch (ns)
   uint32_t tmem_cols;
   uint32_t acc_stride;  // TMEM column distance between the two accumulators
-  int trace_id;         // call-site id (used by instrumented builds only)
   // optional: [zero, zero + zero_floats) cleared by the epilogue warps after the
   // dependency wait, spread over the CTAs (a later linear's fp32 accumulator)
   float* zero;
@@ -46,6 +48,11 @@ struct TcLinearPlan {
   size_t smem = 0;
   double weight_bytes = 0;  // algorithmic bytes streamed per launch (W once)
 };
+
+// Limit of the linear kernel's bounded waits, taken by every plan encoded afterwards
+// (default 2 s; lowered only by the timeout test hook of the stateless entry points).
+constexpr unsigned long long kDefaultWaitNs = 2000000000ull;
+extern std::atomic<unsigned long long> g_lin_wait_ns;
 
 // Largest grid of the linear kernel (one CTA per SM) and the workspace it needs.
 int tc_num_sms();
@@ -62,6 +69,10 @@ int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, const
                    int* counters, int* err, char* msg, size_t msg_len, const void* W2 = nullptr, int N2 = 0,
                    float* zero = nullptr, long long zero_floats = 0);
 cudaError_t tc_linear_launch(const TcLinearPlan& plan, cudaStream_t s);
+
+// Error word of the allocation-free linear's static scratch on the current device:
+// read into *word and cleared.  0 on success, -1 when a CUDA call failed.
+int noalloc_take_error(int* word);
 
 // ----------------------------------------------------------------------------
 // fp32 linear (SIMT, exact fp32 FMA order per output)

@@ -65,6 +65,26 @@ const NaDevice* na_setup(int dev) {
 }
 
 }  // namespace
+
+// Read and clear the error word of the static scratch on the current device (0 when
+// the device never ran the entry point).  Returns 0, or -1 when a CUDA call failed.
+int noalloc_take_error(int* word) {
+  *word = 0;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= NA_MAX_DEVICES) return -1;
+  int* err = nullptr;
+  {
+    std::lock_guard<std::mutex> lk(g_na_mu);
+    if (!g_na_dev[dev].ready) return 0;
+    err = g_na_dev[dev].err;
+  }
+  int e = 0;
+  if (cudaMemcpy(&e, err, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return -1;
+  if (e && cudaMemset(err, 0, sizeof(int)) != cudaSuccess) return -1;
+  *word = e;
+  return 0;
+}
+
 }  // namespace chimera
 
 using namespace chimera;
@@ -97,10 +117,10 @@ extern "C" chimera_status chimera_op_linear_noalloc(int epi, int out_f32, int M,
     return CHIMERA_EINVAL;
   }
   if (plan.grid > NA_MAX_GRID) plan.grid = NA_MAX_GRID;  // the partition follows gridDim
-  // The counters must start at zero and the error word clean; an aborted earlier call
-  // could have left either set.  The partial tiles are fully written before use.
-  if (cudaMemsetAsync(d->counters, 0, static_cast<size_t>(tiles) * sizeof(int), s) != cudaSuccess ||
-      cudaMemsetAsync(d->err, 0, sizeof(int), s) != cudaSuccess)
+  // The counters must start at zero; an aborted earlier call could have left some
+  // raised.  The partial tiles are fully written before use.  The error word is left
+  // alone: it collects what every call flags until chimera_op_sync reads and clears it.
+  if (cudaMemsetAsync(d->counters, 0, static_cast<size_t>(tiles) * sizeof(int), s) != cudaSuccess)
     return CHIMERA_ECUDA;
   return tc_linear_launch(plan, s) == cudaSuccess ? CHIMERA_OK : CHIMERA_ECUDA;
 }

@@ -22,6 +22,7 @@
 // segment overlap the epilogue of the previous one.
 #include <cstdio>
 #include <cstring>
+#include <atomic>
 #include <mutex>
 
 #include "common.cuh"
@@ -53,19 +54,6 @@ constexpr int PIPE_SMEM = CHIMERA_LIN_PIPE_KB * 1024;
 constexpr int MAX_BN = 256;
 constexpr int MAX_TILES = 8192;
 
-#ifdef CHIMERA_LIN_TRACE
-// Per-CTA timestamps of one launch, and per call site (trace_id) the earliest start,
-// latest first data, latest last MMA and latest end over its CTAs (instrumented builds).
-__device__ unsigned long long g_lin_trace[1024][8];
-__device__ unsigned long long g_lin_tl[4096][4];
-#define TRACE(i) g_lin_trace[blockIdx.x][i] = global_timer_ns()
-#define TL_MIN(i) atomicMin(&g_lin_tl[p.trace_id & 4095][i], global_timer_ns())
-#define TL_MAX(i) atomicMax(&g_lin_tl[p.trace_id & 4095][i], global_timer_ns())
-#else
-#define TRACE(i)
-#define TL_MIN(i)
-#define TL_MAX(i)
-#endif
 
 // Stream-K partition in 32-bit arithmetic (the host checks units * grid < 2^32).
 __device__ __forceinline__ int cta_of_unit(uint32_t u, uint32_t U, uint32_t G) {
@@ -181,10 +169,6 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const _
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  if (threadIdx.x == 0) {
-    TRACE(0);
-    TL_MIN(0);
-  }
 
   const uint32_t U = static_cast<uint32_t>(p.units);
   const uint32_t G = gridDim.x;
@@ -225,7 +209,6 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const _
       for (uint32_t i = 0; i < npre; ++i) {
         uint8_t* sa = smem + i * stage_bytes;
         mbar_arrive_expect_tx(&full[i], static_cast<uint32_t>(stage_bytes));
-        if (i == 0) TRACE(1);
         load_a(u_begin + i, sa, &full[i]);
         issued_mask |= 1u << i;
       }
@@ -235,7 +218,7 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const _
       stage = static_cast<int>(npre % p.stages);
       phase = (npre == static_cast<uint32_t>(p.stages)) ? 1u : 0u;
       for (uint32_t u = u_begin + npre; u < u_end && !*abort; ++u) {
-        if (!mbar_wait(&empty[stage], phase ^ 1u, abort)) break;
+        if (!mbar_wait(&empty[stage], phase ^ 1u, abort, p.wait_ns)) break;
         uint8_t* sa = smem + stage * stage_bytes;
         mbar_arrive_expect_tx(&full[stage], static_cast<uint32_t>(stage_bytes));
         load_a(u, sa, &full[stage]);
@@ -269,16 +252,12 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const _
       for (uint32_t u = u_begin; u < u_end && !*abort;) {
         const int t = static_cast<int>(u / KB);
         const uint32_t seg_end = min(u_end, static_cast<uint32_t>(t + 1) * KB);
-        if (!mbar_wait(&tempty[buf], aphase ^ 1u, abort)) break;
+        if (!mbar_wait(&tempty[buf], aphase ^ 1u, abort, p.wait_ns)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + buf * p.acc_stride;
         bool first = true;
         for (; u < seg_end; ++u) {
-          if (!mbar_wait(&full[stage], phase, abort)) break;
-          if (u == u_begin) {
-            TRACE(2);
-            TL_MAX(1);
-          }
+          if (!mbar_wait(&full[stage], phase, abort, p.wait_ns)) break;
           tc_fence_after();
           const uint32_t sa = smem_u32(smem + stage * stage_bytes);
           const uint32_t sb = sa + a_atom * BKA;
@@ -300,8 +279,6 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const _
           }
         }
         tc_commit(&tfull[buf]);
-        TRACE(3);
-        TL_MAX(2);
         buf ^= 1;
         if (buf == 0) aphase ^= 1u;
       }
@@ -329,9 +306,8 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const _
       const int t = static_cast<int>(u / KB);
       const uint32_t seg_end = min(u_end, static_cast<uint32_t>(t + 1) * KB);
       u = seg_end;
-      const bool ok = mbar_wait(&tfull[buf], aphase, abort);
+      const bool ok = mbar_wait(&tfull[buf], aphase, abort, p.wait_ns);
       if (bar_any(1, 128, !ok)) break;
-      if (threadIdx.x == 64) TRACE(4);
       tc_fence_after();
       const int ft = t / p.tok_tiles, tt = t % p.tok_tiles;
       const uint32_t tu0 = static_cast<uint32_t>(t) * KB;
@@ -370,7 +346,6 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const _
           *s_last = (old == nparts - 1) ? 1 : 0;
         }
         named_bar(1, 128);
-        if (threadIdx.x == 64) TRACE(5);
         if (*s_last) {
           __threadfence();
           // slot of every contributor, computed once (contributor c2 > c_first starts
@@ -405,7 +380,6 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const _
             epi_store16(p, m0 + c0, f, acc);
           }
           if (threadIdx.x == 64) p.counters[t] = 0;
-          if (threadIdx.x == 64) TRACE(6);
         }
         named_bar(1, 128);
       }
@@ -421,10 +395,6 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const _
     tmem_dealloc(tmem_base, p.tmem_cols);
   }
   if (threadIdx.x == 0 && *abort) atomicOr(p.err, ERR_TIMEOUT);
-  if (threadIdx.x == 0) {
-    TRACE(7);
-    TL_MAX(3);
-  }
 }
 
 // ----------------------------------------------------------------------------
@@ -488,28 +458,6 @@ size_t tc_ws_floats(int max_bn) {
 
 int tc_max_tiles() { return MAX_TILES; }
 
-#ifdef CHIMERA_LIN_TRACE
-extern "C" int chimera_lin_timeline(unsigned long long* host, int n, int reset) {
-  if (reset) {
-    static unsigned long long init[4096][4];
-    for (int i = 0; i < 4096; ++i) {
-      init[i][0] = ~0ull;
-      init[i][1] = init[i][2] = init[i][3] = 0;
-    }
-    return cudaMemcpyToSymbol(g_lin_tl, init, sizeof(init)) == cudaSuccess ? 0 : -1;
-  }
-  return cudaMemcpyFromSymbol(host, g_lin_tl, static_cast<size_t>(n) * 4 * sizeof(unsigned long long)) ==
-                 cudaSuccess
-             ? 0
-             : -1;
-}
-extern "C" int chimera_lin_trace(unsigned long long* host, int ctas) {
-  return cudaMemcpyFromSymbol(host, g_lin_trace, static_cast<size_t>(ctas) * 8 * sizeof(unsigned long long)) ==
-                 cudaSuccess
-             ? 0
-             : -1;
-}
-#endif
 
 int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, const void* X_lo, int ldx,
                    const void* W, void* Y, void* Y_lo, int ldy, int epi, int out_f32, float* ws,
@@ -565,6 +513,7 @@ int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, const
   p.ws = ws;
   p.counters = counters;
   p.err = err;
+  p.wait_ns = g_lin_wait_ns.load();
   p.acc_stride = pow2ceil(static_cast<uint32_t>(p.BN));
   p.tmem_cols = pow2ceil(2 * p.acc_stride);
   if (p.tmem_cols < 32) p.tmem_cols = 32;
@@ -582,11 +531,29 @@ int tc_linear_plan(TcLinearPlan* plan, int M, int N, int K, const void* X, const
   return 0;
 }
 
+namespace {
+// The kernel's dynamic shared memory limit is an attribute of the device that is
+// current when it is set: raise it once per device, before the first launch there.
+constexpr int LIN_MAX_DEVICES = 64;
+std::mutex g_attr_mu;
+bool g_attr_set[LIN_MAX_DEVICES];
+}  // namespace
+
+std::atomic<unsigned long long> g_lin_wait_ns{kDefaultWaitNs};
+
 cudaError_t tc_linear_launch(const TcLinearPlan& plan, cudaStream_t s) {
-  static std::once_flag once;
-  std::call_once(once, [] {
-    cudaFuncSetAttribute(tc_linear_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
-  });
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= LIN_MAX_DEVICES) return cudaErrorInvalidDevice;
+  {
+    std::lock_guard<std::mutex> lk(g_attr_mu);
+    if (!g_attr_set[dev]) {
+      e = cudaFuncSetAttribute(tc_linear_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
+      if (e != cudaSuccess) return e;
+      g_attr_set[dev] = true;
+    }
+  }
   launch_pdl(tc_linear_kernel, dim3(plan.grid), dim3(THREADS), plan.smem, s, plan.p);
   return cudaGetLastError();
 }

@@ -230,10 +230,10 @@ struct chimera_ctx {
   cudaGraphExec_t prof_graph = nullptr;  // the step with an event pair around every launch
   size_t prof_count = 0;
   int cur_phase = 0;
+  int last_kind = 0;  // kernel class of the latest launch (CHIMERA_KIND_*)
 
   std::string err;
   std::vector<void*> allocs;
-  int lin_sites = 0;  // call-site ids of the linear plans (instrumented builds)
 };
 
 namespace {
@@ -273,6 +273,7 @@ struct Scope {
   chimera_ctx* c;
   ProfEvent* ev = nullptr;
   Scope(chimera_ctx* ctx, int kind, double bytes) : c(ctx) {
+    c->last_kind = kind;
     if (!c->prof) return;
     if (c->prof_used == c->prof_ev.size()) {
       ProfEvent e{};
@@ -327,7 +328,7 @@ bool make_lin(chimera_ctx* ctx, Lin* l, int M, int N, int K, const void* X, cons
     ctx->err = msg;
     return false;
   }
-  l->tp.p.trace_id = ctx->lin_sites++;
+  l->tp.p.wait_ns = kDefaultWaitNs;  // the timeout hook applies to the stateless entry points only
   return true;
 }
 
@@ -347,12 +348,21 @@ int att_splits(const chimera_ctx* ctx, int B, int nq, int n_keys) {
 }
 
 // With qkv (models where attn_fuses_rope holds) the kernel also rotates q and the nq
-// fresh rows' k (positions n + pos_base + pos_off[i]) and writes their k, v to the pool;
-// its predecessor is always the QKV linear, which triggers only after its own wait.
+// fresh rows' k (positions n + pos_base + pos_off[i]) and writes their k, v to the pool.
+// It then reads n_ctx, the page table and the committed KV rows BEFORE its own
+// dependency wait (prewait_kv).  That is only correct when the launch directly before
+// it is a tensor-core linear: that kernel lets its dependents launch only after its
+// own griddepcontrol.wait, so every earlier kernel has completed by then.  Most row
+// kernels trigger before they wait; one of them directly before this launch could
+// let it read stale KV rows.  The order is checked here (and by a CPU lint test).
 cudaError_t run_attention(chimera_ctx* ctx, bool draft_pool, int layer, int nq, const int* nq_dev, int q_local0,
                           int n_local, const int* n_local_dev, const unsigned long long* anc, int q_rows, int splits,
                           int nq_max, double bytes, const float* qkv = nullptr, int pos_base = 0,
                           const int* pos_off = nullptr) {
+  if (qkv && !(ctx->dtype == 1 && ctx->last_kind == CHIMERA_KIND_LINEAR)) {
+    ctx->err = "attention with early KV reads must directly follow a tensor-core linear";
+    return cudaErrorInvalidValue;
+  }
   Scope sc(ctx, CHIMERA_KIND_ATTENTION, bytes);
   AttnParams p{};
   if (qkv) {
@@ -1042,7 +1052,6 @@ chimera_status chimera_prefill(chimera_ctx* ctx, int batch, const int32_t* token
   }
   ctx->batch = batch;
   ctx->plan_keys = max_len;
-  ctx->lin_sites = 0;
   if (!build_plans(ctx, batch)) return CHIMERA_EINVAL;
   for (int b = 0; b < batch; ++b) {
     chimera_status st = ensure_blocks(ctx, b, lens[b] + need);
@@ -1312,8 +1321,10 @@ chimera_status chimera_debug_read_kv(chimera_ctx* ctx, int layer, int seq, int p
 // stateless kernel-level entry points
 // ---------------------------------------------------------------------------
 namespace {
+// Scratch of the stateless entry points, one set per device (allocated on the first
+// call made with that device current and kept until exit).
 struct OpScratch {
-  int device = -1;
+  bool ready = false;
   float* lin_ws = nullptr;
   int* lin_cnt = nullptr;
   int* err = nullptr;
@@ -1321,27 +1332,39 @@ struct OpScratch {
   size_t att_floats = 0;
   int* att_cnt = nullptr;
 };
+constexpr int OP_MAX_DEVICES = 64;
+constexpr int OP_ATT_COUNTERS = 64 * 256;
 std::mutex g_op_mu;
-OpScratch g_op;
+OpScratch g_op_dev[OP_MAX_DEVICES];
 
-bool op_scratch() {
+// The current device's scratch (nullptr on failure).  Caller holds g_op_mu.
+OpScratch* op_scratch() {
   int dev = 0;
-  cudaGetDevice(&dev);
-  if (g_op.device == dev) return true;
-  OpScratch s;
-  s.device = dev;
-  s.att_floats = static_cast<size_t>(16) << 20;
-  if (cudaMalloc(&s.lin_ws, tc_ws_floats(256) * sizeof(float)) != cudaSuccess) return false;
-  if (cudaMalloc(&s.lin_cnt, tc_max_tiles() * sizeof(int)) != cudaSuccess) return false;
-  if (cudaMalloc(&s.err, sizeof(int)) != cudaSuccess) return false;
-  if (cudaMalloc(&s.att_ws, s.att_floats * sizeof(float)) != cudaSuccess) return false;
-  if (cudaMalloc(&s.att_cnt, 64 * 256 * sizeof(int)) != cudaSuccess) return false;
-  cudaMemset(s.lin_cnt, 0, tc_max_tiles() * sizeof(int));
-  cudaMemset(s.err, 0, sizeof(int));
-  cudaMemset(s.att_cnt, 0, 64 * 256 * sizeof(int));
-  if (cudaDeviceSynchronize() != cudaSuccess) return false;
-  g_op = s;
-  return true;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= OP_MAX_DEVICES) return nullptr;
+  OpScratch& s = g_op_dev[dev];
+  if (s.ready) return &s;
+  OpScratch n;
+  n.att_floats = static_cast<size_t>(16) << 20;
+  bool ok = cudaMalloc(&n.lin_ws, tc_ws_floats(256) * sizeof(float)) == cudaSuccess;
+  ok = ok && cudaMalloc(&n.lin_cnt, tc_max_tiles() * sizeof(int)) == cudaSuccess;
+  ok = ok && cudaMalloc(&n.err, sizeof(int)) == cudaSuccess;
+  ok = ok && cudaMalloc(&n.att_ws, n.att_floats * sizeof(float)) == cudaSuccess;
+  ok = ok && cudaMalloc(&n.att_cnt, OP_ATT_COUNTERS * sizeof(int)) == cudaSuccess;
+  ok = ok && cudaMemset(n.lin_cnt, 0, tc_max_tiles() * sizeof(int)) == cudaSuccess;
+  ok = ok && cudaMemset(n.err, 0, sizeof(int)) == cudaSuccess;
+  ok = ok && cudaMemset(n.att_cnt, 0, OP_ATT_COUNTERS * sizeof(int)) == cudaSuccess;
+  ok = ok && cudaDeviceSynchronize() == cudaSuccess;
+  if (!ok) {
+    cudaFree(n.lin_ws);
+    cudaFree(n.lin_cnt);
+    cudaFree(n.err);
+    cudaFree(n.att_ws);
+    cudaFree(n.att_cnt);
+    return nullptr;
+  }
+  n.ready = true;
+  s = n;
+  return &s;
 }
 }  // namespace
 
@@ -1356,11 +1379,12 @@ chimera_status chimera_op_linear(int dtype, int epi, int out_f32, int M, int N, 
                              ? CHIMERA_OK
                              : CHIMERA_ECUDA;
   std::lock_guard<std::mutex> lk(g_op_mu);
-  if (!op_scratch()) return CHIMERA_ENOMEM;
+  OpScratch* sc = op_scratch();
+  if (!sc) return CHIMERA_ENOMEM;
   TcLinearPlan plan;
   char msg[256];
-  if (tc_linear_plan(&plan, M, N, K, X, X_lo, ldx, W, Y, nullptr, ldy, epi, epi == EPI_RESID ? 1 : out_f32, g_op.lin_ws,
-                     g_op.lin_cnt, g_op.err, msg, sizeof(msg)) != 0)
+  if (tc_linear_plan(&plan, M, N, K, X, X_lo, ldx, W, Y, nullptr, ldy, epi, epi == EPI_RESID ? 1 : out_f32, sc->lin_ws,
+                     sc->lin_cnt, sc->err, msg, sizeof(msg)) != 0)
     return CHIMERA_EINVAL;
   return tc_linear_launch(plan, s) == cudaSuccess ? CHIMERA_OK : CHIMERA_ECUDA;
 }
@@ -1375,7 +1399,8 @@ chimera_status chimera_op_attention(int dtype, int kv_split, int batch, int n_he
       n_blocks < 1)
     return CHIMERA_EINVAL;
   std::lock_guard<std::mutex> lk(g_op_mu);
-  if (!op_scratch()) return CHIMERA_ENOMEM;
+  OpScratch* sc = op_scratch();
+  if (!sc) return CHIMERA_ENOMEM;
   AttnParams p{};
   p.q = q;
   p.ldq = ldq;
@@ -1398,13 +1423,52 @@ chimera_status chimera_op_attention(int dtype, int kv_split, int batch, int n_he
   p.hd = head_dim;
   p.scale = 1.0f / std::sqrt(static_cast<float>(head_dim));
   p.splits = splits;
-  p.ws = g_op.att_ws;
-  p.counters = g_op.att_cnt;
+  p.ws = sc->att_ws;
+  p.counters = sc->att_cnt;
+  p.err = sc->err;
   p.nq_max = nq;
-  if (attn_ws_floats(batch, n_heads, splits, nq, head_dim) > g_op.att_floats) return CHIMERA_EINVAL;
+  if (attn_ws_floats(batch, n_heads, splits, nq, head_dim) > sc->att_floats) return CHIMERA_EINVAL;
   return attention(p, dtype, static_cast<cudaStream_t>(cuda_stream)) == cudaSuccess
              ? CHIMERA_OK
              : CHIMERA_ECUDA;
+}
+
+chimera_status chimera_op_sync(void* cuda_stream) {
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  if (cudaStreamSynchronize(s) != cudaSuccess) return CHIMERA_ECUDA;
+  int word = 0;
+  {
+    std::lock_guard<std::mutex> lk(g_op_mu);
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= OP_MAX_DEVICES) return CHIMERA_ECUDA;
+    OpScratch& sc = g_op_dev[dev];
+    if (sc.ready) {
+      int e = 0;
+      if (cudaMemcpy(&e, sc.err, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return CHIMERA_ECUDA;
+      if (e) {
+        // a launch that gave up can leave split-K or split-merge counters raised
+        if (cudaMemset(sc.err, 0, sizeof(int)) != cudaSuccess ||
+            cudaMemset(sc.lin_cnt, 0, tc_max_tiles() * sizeof(int)) != cudaSuccess ||
+            cudaMemset(sc.att_cnt, 0, OP_ATT_COUNTERS * sizeof(int)) != cudaSuccess ||
+            cudaDeviceSynchronize() != cudaSuccess)
+          return CHIMERA_ECUDA;
+      }
+      word |= e;
+    }
+  }
+  int na = 0;
+  if (noalloc_take_error(&na) != 0) return CHIMERA_ECUDA;
+  word |= na;
+  if (word & ERR_TIMEOUT) return CHIMERA_ETIMEDOUT;
+  if (word & ERR_CAPACITY) return CHIMERA_ECAPACITY;
+  if (word) return CHIMERA_EINVAL;
+  return CHIMERA_OK;
+}
+
+chimera_status chimera_debug_set_wait_limit(uint64_t ns) {
+  if (ns == 0) ns = kDefaultWaitNs;
+  g_lin_wait_ns.store(ns);
+  return CHIMERA_OK;
 }
 
 }  // extern "C"

@@ -132,23 +132,78 @@ def test_tiny_forced_acceptance_and_compaction(tiny, forced):
     assert ctx.read("n")[0] == len(prompt) + len(out)
 
 
-# ----------------------------------------------------------------------------
-# bf16 configs, oracle-driven
-# ----------------------------------------------------------------------------
-def _force_chain(W, cfg, st, tree, toks, L):
-    """Set the rank-0 branch to the base model's greedy continuation for L tokens."""
-    toks = list(toks)
-    chain = [0]
+def _branch_tokens(tree, base, branch, V):
+    """Tree tokens whose nodes on `branch` (a rank tuple, e.g. (1, 0, 0)) carry `base`
+    (AR continuation, base[0] = root); every other node is wrong."""
+    toks = [0] * tree["n"]
     for i in range(1, tree["n"]):
-        if all(r == 0 for r in tree["nodes"][i]):
-            chain.append(i)
-    for j in range(1, min(L, len(chain) - 1) + 1):
-        ver = co.verify(W, cfg, st, tree, toks)
-        toks[chain[j]] = co.argmax_desc(ver["logits"][chain[j - 1]])
+        r, dep = tree["nodes"][i], tree["depth"][i]
+        on = tuple(r) == tuple(branch[:dep])
+        toks[i] = base[dep] if on else (base[dep] + 1 + tree["rank"][i] + 7 * dep) % V
     return toks
 
 
-def _run_bf16(name, n_steps, forced_seq, device_gen="cpu", max_seq=None, precision=1):
+@pytest.mark.parametrize("branch", [(1, 0), (1, 0, 0), (2, 0, 0)])
+def test_tiny_overlapping_compaction(tiny, branch):
+    # accepted path off the rank-0 branch: e.g. "1" -> "10" -> "100" is nodes [0, 2, 7, 12],
+    # so slot n+2 is both the destination of node 7 and the source of node 2; every
+    # layer's compacted KV and the appended draft KV must equal the oracle's
+    cfg, w_dev, W, prompt = tiny
+    tol = tol_of(cfg)
+    tree = ot.build_tree(cfg["topk"], cfg["tree_nodes"])
+    ar = co.ar_generate(W, cfg, prompt, 12)
+    ctx = pkg.Chimera(cfg, w_dev, max_batch=1, max_seq_len=256)
+    ctx.prefill([prompt])
+    st = co.prefill(W, cfg, prompt, 256)
+    out = []
+    for _ in range(2):
+        toks = _branch_tokens(tree, ar[len(out):], branch, cfg["vocab"])
+        ctx.override_tree([toks])
+        n0 = st.n
+        e = ctx.step()[0]
+        rec = co.step(W, cfg, st, tree, toks)
+        L = len(branch)
+        want_path = [0] + [tree["nodes"].index(tuple(branch[:j])) for j in range(1, L + 1)]
+        assert rec["path"] == want_path
+        assert ctx.read("path")[0][: L + 1].tolist() == want_path
+        # some entry's source slot is another entry's destination slot
+        assert any(want_path[j] == j2 for j in range(1, L + 1) for j2 in range(1, L + 1) if j2 != j)
+        assert e == rec["emitted"] == ar[len(out): len(out) + L + 1]
+        for layer in list(range(cfg["n_layers"])) + [-1]:
+            k, v = ctx.read_kv(layer, 0, n0, L + 1)
+            rk = st.dK[n0:n0 + L + 1] if layer < 0 else st.K[layer, n0:n0 + L + 1]
+            rv = st.dV[n0:n0 + L + 1] if layer < 0 else st.V[layer, n0:n0 + L + 1]
+            assert rel_rows(k, rk) <= tol and rel_rows(v, rv) <= tol, layer
+        out += e
+    assert ctx.read("n")[0] == len(prompt) + len(out)
+
+
+# ----------------------------------------------------------------------------
+# bf16 configs, oracle-driven
+# ----------------------------------------------------------------------------
+def _force_chain(W, cfg, st, tree, toks, L, branch=(0, 0, 0, 0)):
+    """Set the nodes of `branch` (a rank tuple; default the rank-0 branch) to the base
+    model's greedy continuation for L tokens; a sibling that happens to carry the same
+    token is moved off it, so the accepted path is exactly that branch."""
+    toks = list(toks)
+    V = cfg["vocab"]
+    chain = [0]
+    for d in range(1, len(branch) + 1):
+        r = tuple(branch[:d])
+        if r not in tree["nodes"]:
+            break
+        chain.append(tree["nodes"].index(r))
+    for j in range(1, min(L, len(chain) - 1) + 1):
+        ver = co.verify(W, cfg, st, tree, toks)
+        t = co.argmax_desc(ver["logits"][chain[j - 1]])
+        toks[chain[j]] = t
+        for c in tree["children"][chain[j - 1]]:
+            if c != chain[j] and toks[c] == t:
+                toks[c] = (t + 1) % V
+    return toks
+
+
+def _run_bf16(name, n_steps, forced_seq, device_gen="cpu", max_seq=None, precision=1, branch=(0, 0, 0, 0)):
     cfg, w_cpu, w_dev = _setup(name, device_gen)
     W = co.OracleWeights(w_cpu, cache=(name != "7b"))
     prompts = synth.make_prompts(cfg)
@@ -173,7 +228,7 @@ def _run_bf16(name, n_steps, forced_seq, device_gen="cpu", max_seq=None, precisi
         for b in range(B):
             dr = co.draft(W, cfg, states[b], kmax)
             toks = co.tree_tokens(tree, states[b].tokens[states[b].n], dr["topk"])
-            toks = _force_chain(W, cfg, states[b], tree, toks, forced_seq[(step + b) % len(forced_seq)])
+            toks = _force_chain(W, cfg, states[b], tree, toks, forced_seq[(step + b) % len(forced_seq)], branch)
             drafts.append(dr)
             toks_all.append(toks)
         n_before = [s.n for s in states]
@@ -210,9 +265,8 @@ def _run_bf16(name, n_steps, forced_seq, device_gen="cpu", max_seq=None, precisi
                 diverged = True
             else:
                 assert emitted[b] == [toks_all[b][i] for i in path]
-                # compacted KV of the accepted rows, first and last layer, and draft KV
-                st = states[b]
-                for layer in (0, cfg["n_layers"] - 1):
+                # compacted KV of the accepted rows in every layer, and draft KV
+                for layer in range(cfg["n_layers"]):
                     k_g, v_g = ctx.read_kv(layer, b, n_before[b], L + 1)
                     assert rel_rows(k_g, ver["k"][layer][path]) <= tol
                     assert rel_rows(v_g, ver["v"][layer][path]) <= tol
@@ -241,6 +295,13 @@ def test_mini_bf16_steps():
 def test_mini_bf16_plain_precision():
     # activations rounded once to bf16 and bf16 KV caches (precision 0)
     _run_bf16("mini", 3, [4, 2, 0], precision=0)
+
+
+def test_mini_overlapping_compaction():
+    # accepted paths along "1" -> "10" -> "100" -> "1000" (nodes 2, 11, 39, 62 of the
+    # 64-node tree): destination slots n+1.. are sources of later path entries
+    acc = _run_bf16("mini", 3, [4, 2, 3], branch=(1, 0, 0, 0))
+    assert max(acc) >= 3
 
 
 def test_mini_b4_ragged_batch():

@@ -47,3 +47,40 @@ def test_noalloc_rejects_sizes_beyond_the_static_limit():
     Y = torch.zeros(33, 128, device="cuda")
     with pytest.raises(pkg.ChimeraError):
         pkg.op_linear_noalloc(X, W, Y, out_f32=True)
+
+
+@pytest.mark.parametrize("M", [17, 32])
+def test_noalloc_split_operand_matches_op_linear(M):
+    # the hi + lo split activation (two MMAs per K slice) changes the stage layout that
+    # the static scratch is used with
+    g = torch.Generator().manual_seed(M)
+    N, K = 1536, 2048
+    X32 = torch.randn(M, K, generator=g)
+    X = X32.to(torch.bfloat16)
+    X_lo = (X32 - X.float()).to(torch.bfloat16)
+    W = (torch.randn(N, K, generator=g) * 0.05).to(torch.bfloat16)
+    X, X_lo, W = X.cuda(), X_lo.cuda(), W.cuda()
+    for call in range(2):
+        ref = torch.zeros(M, N, device="cuda")
+        got = torch.zeros(M, N, device="cuda")
+        pkg.op_linear(X, W, ref, epi=0, out_f32=True, X_lo=X_lo)
+        pkg.op_linear_noalloc(X, W, got, epi=0, out_f32=True, X_lo=X_lo)
+        torch.cuda.synchronize()
+        assert _rel_rows(got.cpu().numpy(), ref.cpu().numpy()) <= 1e-5, (call,)
+
+
+def test_noalloc_calls_leave_device_memory_unchanged():
+    # after a first call (which looks up the static arrays' addresses), further calls
+    # must not change the device's free memory: nothing is allocated per call
+    M, N, K = 16, 4096, 4096
+    X = torch.randn(M, K).to(torch.bfloat16).cuda()
+    W = (torch.randn(N, K) * 0.02).to(torch.bfloat16).cuda()
+    Y = torch.zeros(M, N, device="cuda")
+    pkg.op_linear_noalloc(X, W, Y, epi=0, out_f32=True)
+    torch.cuda.synchronize()
+    free0 = torch.cuda.mem_get_info()[0]
+    for _ in range(4):
+        pkg.op_linear_noalloc(X, W, Y, epi=0, out_f32=True)
+    torch.cuda.synchronize()
+    assert torch.cuda.mem_get_info()[0] == free0
+    pkg.op_sync()  # and no device-side error was flagged
