@@ -6,15 +6,18 @@ verify forward over 32 layers with the LM head and argmax, greedy acceptance, KV
 compaction and the draft-KV append.  The model is random-init (N(0, 0.02)) with the
 Vicuna-7B shape; the 512-token prompt is seeded uniform ids.
 
-Output: one JSON line (rank 0).  `value` = tree tokens per second (B * N tree nodes
-verified per step, whole job); `ms_per_step` = device time of one step from CUDA
-events around K back-to-back graph replays; `e2e` = the same metric through
-chimera_step with host output buffers and a synchronisation per step.
-`--impl reference` times the fp64 CPU oracle instead (see `cpu_sample`).
+Output: one JSON line (rank 0).  `value` = tree tokens per second of whole steps (B * N
+tree nodes per step, whole job); `ms_per_step` = device time of one step from CUDA
+events around K back-to-back graph replays; `breakdown.verify_ms` = the verify phase
+(tree expansion, 32-layer tree forward, LM head, argmax) from CUDA events recorded at
+the phase boundaries of a graph replay; `e2e` = the same metric through chimera_step
+with host output buffers and a synchronisation per step.  `--impl reference` times the
+fp64 CPU oracle (whole steps on an oracle-prefilled state) instead.
 """
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import os
 import statistics
@@ -25,6 +28,9 @@ import time
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
+# the oracle's matrix products run on every host core
+for _v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+    os.environ.setdefault(_v, str(os.cpu_count() or 1))
 
 import numpy as np  # noqa: E402
 import torch  # noqa: E402
@@ -32,7 +38,12 @@ import torch  # noqa: E402
 import synth  # noqa: E402
 
 WORKLOAD = "7b"
-LINEAR_DRAM_BYTES_PER_STEP = 18.23e9
+
+# DRAM traffic of the tensor-core linear over its algorithmic bytes (weights streamed
+# once), from an ncu capture of one launch family on a small case, keyed by the
+# SHA-256 of the kernel source it was taken on: the roofline's `traffic` is null
+# whenever the kernel has changed since (the key no longer matches).
+LINEAR_TRAFFIC_RATIO = {}
 
 
 def peaks():
@@ -60,25 +71,64 @@ def job_rate(units_per_rank: float, world: int, ms_job: float) -> float:
     return world * units_per_rank / (ms_job * 1e-3)
 
 
-def step_bytes(cfg, n_ctx, kv_elem_bytes=None):
+def step_bytes(cfg, n_ctx):
     """Algorithmic HBM bytes of one step at committed length n_ctx (batch 1).
 
     Every weight matrix counts once per use (the trigram encoder and the draft block
-    once per draft sub-step), embeddings only for the gathered rows, KV as the rows
-    read; activations are excluded.  kv_elem_bytes is the stored size of one K (or V)
-    element: 4 for the fp32-equivalent hi+lo bf16 planes of precision mode 1, else the
-    weight element size."""
+    once per draft sub-step, the heads once), embeddings only for the gathered rows, KV
+    as the rows read at the model's element size (bf16: 2 bytes per K or V value); the
+    activations are excluded.  `kv_planes_extra` is what the stored hi + lo planes of
+    precision mode 1 read on top (the same again): traffic, not algorithmic bytes."""
     d, F, V, L, K, N = (cfg["d_model"], cfg["ffn_dim"], cfg["vocab"], cfg["n_layers"],
                         cfg["n_draft_heads"], cfg["tree_nodes"])
     e = 2 if cfg["dtype"] == "bf16" else 4
     layer = (3 * d * d + d * d + 3 * d * F) * e
-    kv_row = 2 * d * (kv_elem_bytes or e)
-    verify = L * layer + V * d * e + N * d * e + L * (n_ctx + N) * kv_row
+    kv_row = 2 * d * e
+    verify_w = L * layer + V * d * e + N * d * e
+    verify_kv = L * (n_ctx + N) * kv_row
     draft_w = K * ((3 * d * d + d * d) * e + layer) + K * V * 2 * d * e + K * 3 * d * e
     draft_kv = sum((n_ctx + k + 1) * kv_row for k in range(K))
     commit = 2 * d * d * e + 2 * L * 4 * kv_row
-    return dict(verify=verify, draft=draft_w + draft_kv, commit=commit,
-                total=verify + draft_w + draft_kv + commit)
+    return dict(verify=verify_w + verify_kv, verify_weights=verify_w, verify_kv=verify_kv,
+                draft=draft_w + draft_kv, commit=commit, total=verify_w + verify_kv + draft_w + draft_kv + commit,
+                kv_planes_extra=verify_kv + draft_kv)
+
+
+def workload_config(cfg, prompt_len):
+    return {"workload": "7B-shaped bs1 draft-and-verify step (N=64, topk 5,5,5,5, 512-token prompt)",
+            "batch": cfg["batch"], "tree_nodes": cfg["tree_nodes"], "prompt_len": prompt_len,
+            "layers": cfg["n_layers"], "d_model": cfg["d_model"], "ffn_dim": cfg["ffn_dim"], "vocab": cfg["vocab"],
+            "draft_heads": cfg["n_draft_heads"], "topk": cfg["topk"]}
+
+
+def oracle_steps(cfg, w_cpu, prompt, n_steps, warmup=1):
+    """The fp64 oracle (as it stands) on the host cores: prefill the prompt (setup,
+    untimed), then `warmup` + n_steps whole draft-and-verify steps; returns the wall
+    time of each timed step (s) and the setup time."""
+    from oracle import chimera_oracle as co
+    from oracle import tree as ot
+    W = co.OracleWeights(w_cpu, cache=False)
+    tree = ot.build_tree(cfg["topk"], cfg["tree_nodes"])
+    cap = len(prompt) + (n_steps + warmup + 1) * 5 + cfg["tree_nodes"] + 8
+    t0 = time.perf_counter()
+    st = co.prefill(W, cfg, prompt, cap)
+    setup = time.perf_counter() - t0
+    for _ in range(warmup):
+        co.step(W, cfg, st, tree)
+    times = []
+    for _ in range(n_steps):
+        t0 = time.perf_counter()
+        co.step(W, cfg, st, tree)
+        times.append(time.perf_counter() - t0)
+    return times, setup
+
+
+def host_threads():
+    try:
+        aff = len(os.sched_getaffinity(0))
+    except AttributeError:
+        aff = os.cpu_count() or 1
+    return {"cores": os.cpu_count() or 1, "affinity": aff, "blas_threads": int(os.environ["OPENBLAS_NUM_THREADS"])}
 
 
 class Clocks:
@@ -111,43 +161,6 @@ class Clocks:
                           if r[5 + i].strip().lower() == "active"})
         return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
                 "reasons": reasons, "samples": len(rows)}
-
-
-def cpu_sample(cfg, w_dev, n_ctx, threads):
-    """Time the fp64 oracle on host cores on a bounded sample of the step:
-    one base layer of the tree verify (64 nodes, n_ctx committed rows), the LM head on
-    64 rows, and one draft sub-step (trigram encoder, full-context block row, one head).
-    The step estimate scales the layer by the layer count and the draft sub-step by K."""
-    from oracle import chimera_oracle as co
-    from oracle import tree as ot
-    names = ["embed", "lm_head", "final_norm", "tri_w1", "tri_w2", "heads.0"]
-    names += [n for n in w_dev if n.startswith("layers.0.") or n.startswith("draft.")]
-    w = {n: w_dev[n].cpu() for n in names}
-    W = co.OracleWeights(w, cache=False)
-    H, hd, d, N = cfg["n_heads"], cfg["head_dim"], cfg["d_model"], cfg["tree_nodes"]
-    rng = np.random.default_rng(0)
-    tree = ot.build_tree(cfg["topk"], N)
-    mask = np.array([[(tree["anc"][i] >> j) & 1 == 1 for j in range(N)] for i in range(N)])
-    ctx_k = rng.standard_normal((n_ctx, H, hd))
-    ctx_v = rng.standard_normal((n_ctx, H, hd))
-    x = rng.standard_normal((N, d))
-    pos = n_ctx + np.array(tree["depth"])
-    t0 = time.perf_counter()
-    out, _, _ = co.block_rows(W, "layers.0", cfg, x, pos, ctx_k, ctx_v, mask)
-    t_layer = time.perf_counter() - t0
-    t0 = time.perf_counter()
-    hs = co.rmsnorm(out, W("final_norm"), cfg["rms_eps"])
-    _ = hs @ W("lm_head").T
-    t_lm = time.perf_counter() - t0
-    t0 = time.perf_counter()
-    t = co.trigram_input(W, cfg, [1, 2, 3])
-    g = co.trigram_encoder(W, t)
-    h, _, _ = co.block_rows(W, "draft", cfg, g[None], np.array([n_ctx]), ctx_k, ctx_v, np.ones((1, 1), bool))
-    z = W("heads.0") @ np.concatenate([hs[0], h[0]])
-    _ = co.topk_desc(z, max(cfg["topk"]))
-    t_draft = time.perf_counter() - t0
-    est = cfg["n_layers"] * t_layer + t_lm + cfg["n_draft_heads"] * t_draft
-    return dict(t_layer=t_layer, t_lm=t_lm, t_draft_sub=t_draft, step_s=est, threads=threads)
 
 
 def op_bench(args, hbm, peak_kind):
@@ -227,6 +240,42 @@ def op_bench(args, hbm, peak_kind):
                       "launches": args.steps, "note": "back-to-back device launches (enqueued behind a sleep kernel)"}))
 
 
+
+
+def reference_arm(args, rank):
+    """The oracle timed on the host cores, whole steps, on the main arm's workload."""
+    if rank != 0:
+        return
+    cfg = synth.get_config(WORKLOAD)
+    prompt = synth.make_prompts(cfg)[0]
+    # the oracle reads the stored weights; draw them on the host with the same shapes
+    w = synth.make_weights(cfg, device="cpu")
+    ht = host_threads()
+    times, setup = oracle_steps(cfg, w, prompt, args.steps, warmup=1)
+    t = statistics.median(times)
+    B, N = cfg["batch"], cfg["tree_nodes"]
+    v = B * N / t
+    sample = (f"whole steps of the fp64 NumPy oracle (draft K=4, 32-layer tree verify, LM head, accept, "
+              f"commit) after an oracle prefill of the {len(prompt)}-token prompt ({setup:.1f} s, untimed); "
+              f"1 warm-up + {args.steps} timed steps, median {t:.2f} s")
+    line = {"impl": "reference", "metric": "tree tokens/s at 7B bs1 (draft-and-verify step)",
+            "value": v, "unit": "tree tokens/s", "n_gpus": args.gpus, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": t * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": workload_config(cfg, len(prompt)),
+            "cpu_baseline": {"kind": "oracle", "cores": ht["blas_threads"], "value": v, "unit": "tree tokens/s",
+                             "sample": sample, "host": ht},
+            "e2e": {"value": v, "unit": "tree tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "step_s": [round(x, 3) for x in times]}
+    print(json.dumps(line))
+
+
+def linear_traffic_ratio():
+    src = os.path.join(ROOT, "paper_2402_15758_gb300", "csrc", "linear_tc.cu")
+    h = hashlib.sha256(open(src, "rb").read()).hexdigest()
+    return LINEAR_TRAFFIC_RATIO.get(h), h
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -234,7 +283,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="chimera", choices=["chimera", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--profile-steps", type=int, default=3)
+    ap.add_argument("--layers", type=int, default=None,
+                    help="profiling only: the 7B shapes with fewer base layers (not the benchmark workload)")
     ap.add_argument("--op", choices=["linear", "attention"], default=None,
                     help="time one kernel entry point instead of the step")
     ap.add_argument("--shape", default="64,22016,4096", help="--op linear: M,N,K")
@@ -245,37 +295,11 @@ def main():
     if args.op:
         op_bench(args, *peaks())
         return
-
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
-    cfg = synth.get_config(WORKLOAD)
-    B, N = cfg["batch"], cfg["tree_nodes"]
-    prompt = synth.make_prompts(cfg)[0]
-    threads = os.cpu_count() or 1
-
     if args.impl == "reference":
-        if rank != 0:
-            return
-        torch.manual_seed(0)
-        # the oracle needs only the weights of the sampled parts; draw them on the host
-        # with the same shapes (values do not change the timing)
-        w = synth.make_weights(dict(cfg, n_layers=1), device="cpu")
-        for _ in range(args.warmup if args.warmup < 1 else 1):
-            cpu_sample(cfg, w, len(prompt), threads)
-        times = [cpu_sample(cfg, w, len(prompt), threads)["step_s"] for _ in range(args.steps)]
-        t = statistics.median(times)
-        v = B * N / t
-        line = {"impl": "reference", "metric": "tree tokens/s at 7B bs1 (draft-and-verify step)",
-                "value": v, "unit": "tree tokens/s", "n_gpus": args.gpus, "steps": args.steps,
-                "warmup": args.warmup, "ms_per_step": t * 1e3, "higher_is_better": True,
-                "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-                "config": {"workload": "7B-shaped bs1 draft-and-verify step (N=64, topk 5,5,5,5, 512-token prompt)"},
-                "cpu_baseline": {"kind": "oracle", "cores": threads, "value": v, "unit": "tree tokens/s",
-                                 "sample": "per step: one verify layer (64 nodes, 512 ctx) x32 + LM head + "
-                                           "one draft sub-step x4, fp64 NumPy on the host cores"},
-                "e2e": {"value": v, "unit": "tree tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
-        print(json.dumps(line))
+        reference_arm(args, rank)
         return
 
     import paper_2402_15758_gb300 as pkg
@@ -287,9 +311,15 @@ def main():
     pkg_build.build()
     pkg.load()
 
+    cfg = synth.get_config(WORKLOAD)
+    if args.layers:
+        cfg["n_layers"] = args.layers
+    B, N = cfg["batch"], cfg["tree_nodes"]
+    prompt = synth.make_prompts(cfg)[0]
     w = synth.make_weights(cfg, device="cuda")
     torch.cuda.synchronize()
-    total_steps = args.warmup + 2 * args.steps + args.profile_steps + args.steps + 8
+    reps = max(3, min(args.steps, 20))
+    total_steps = args.warmup + 3 * args.steps + reps + 8
     max_seq = ((len(prompt) + total_steps * 5 + N + 64 + 15) // 16) * 16
     stream = torch.cuda.Stream()
     ctx = pkg.Chimera(cfg, w, max_batch=B, max_seq_len=max_seq, stream=stream)
@@ -325,31 +355,28 @@ def main():
     ctx.sync()
     torch.cuda.synchronize()
     per_step = sorted(ev[i].elapsed_time(ev[i + 1]) for i in range(args.steps))
-    step_median = max_over_ranks(statistics.median(per_step), world)
-    step_p90 = max_over_ranks(per_step[min(len(per_step) - 1, int(round(0.9 * (len(per_step) - 1))))], world)
 
-    # ---- per-kernel timing (eager launches with events around each) ----
-    recs = []
-    for _ in range(args.profile_steps):
-        recs.append(ctx.profile_step())
-    launches = len(recs[-1])
+    def med_p90(xs):
+        xs = sorted(xs)
+        return statistics.median(xs), xs[min(len(xs) - 1, int(round(0.9 * (len(xs) - 1))))]
 
-    def agg(pred):
-        out = []
-        for r in recs:
-            sel = [x for x in r if pred(x)]
-            out.append((sum(x["ms"] for x in sel), sum(x["bytes"] for x in sel), len(sel)))
-        return out
+    step_median, step_p90 = (max_over_ranks(v, world) for v in med_p90(per_step))
 
-    lin = agg(lambda x: x["kind"] == "linear")
-    lin_ms = statistics.median([a[0] for a in lin])
-    lin_bytes = statistics.median([a[1] for a in lin])
-    lin_n = lin[-1][2]
-    phase_ms = {ph: statistics.median([a[0] for a in agg(lambda x, ph=ph: x["phase"] == ph)])
-                for ph in ("draft", "verify", "commit")}
-    eager_ms = statistics.median([sum(x["ms"] for x in r) for r in recs])
+    # ---- phases: events at the draft | verify | commit boundaries of a graph replay ----
+    dr_ms, ve_ms, co_ms = ctx.profile_phases(args.steps)
+    verify_med, verify_p90 = (max_over_ranks(v, world) for v in med_p90(ve_ms))
+    draft_med, _ = med_p90(dr_ms)
+    commit_med, _ = med_p90(co_ms)
+
+    # ---- the dominant kernel class alone: the step's linear launches, back to back ----
+    lin = ctx.profile_kind("linear", reps)
+    att = ctx.profile_kind("attention", reps)
+
+    # ---- per-kernel timing, eager (an event pair around every launch: no overlap) ----
+    rec = ctx.profile_step()
+    launches = len(rec)
     kind_ms = {}
-    for x in recs[-1]:
+    for x in rec:
         kind_ms[x["kind"]] = kind_ms.get(x["kind"], 0.0) + x["ms"]
 
     # ---- end to end through chimera_step (host outputs, one sync per step) ----
@@ -363,55 +390,74 @@ def main():
         emitted += sum(len(o) for o in out)
     t_e2e = max_over_ranks((time.perf_counter() - t0) / args.steps, world)
     d2h = B * 4 + 4 + int(round(4 * emitted / args.steps))
+    n_mid = (n0 + n1) // 2
+    ctx.close()
 
     hbm, peak_kind = peaks()
-    nb = step_bytes(cfg, (n0 + n1) // 2, kv_elem_bytes=4 if ctx.kv_f32 else None)
+    nb = step_bytes(cfg, n_mid)
     value = job_rate(B * N, world, ms)
-    if lin_ms <= 0:
-        raise RuntimeError("per-kernel profile returned no linear time")
-    lin_gbs = lin_bytes / (lin_ms * 1e-3) / 1e9
+    lin_per_launch_ms = lin["ms"] / max(1, lin["launches"])
+    lin_bytes_per_launch = lin["bytes"] / max(1, lin["launches"])
+    lin_gbs = lin_bytes_per_launch / (lin_per_launch_ms * 1e-3) / 1e9
+    ratio, src_hash = linear_traffic_ratio()
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cs = cpu_sample(cfg, w, n1, threads)
-        cpu = {"value": B * N / cs["step_s"], "unit": "tree tokens/s", "cores": threads, "kind": "oracle",
-               "sample": (f"fp64 NumPy oracle: one verify layer (64 nodes, {n1} ctx) {cs['t_layer']:.2f}s x32 + "
-                          f"LM head {cs['t_lm']:.2f}s + one draft sub-step {cs['t_draft_sub']:.2f}s x4 "
-                          f"= {cs['step_s']:.1f}s per step (estimate)")}
+        w_cpu = {k: v.cpu() for k, v in w.items()}
+        del w
+        torch.cuda.empty_cache()
+        ht = host_threads()
+        times, setup = oracle_steps(cfg, w_cpu, prompt, 1, warmup=0)
+        cpu = {"value": B * N / times[0], "unit": "tree tokens/s", "cores": ht["blas_threads"], "kind": "oracle",
+               "sample": (f"one whole step of the fp64 NumPy oracle on its own prefilled state "
+                          f"({len(prompt)}-token prompt, prefill {setup:.1f} s untimed): {times[0]:.2f} s"),
+               "host": ht}
     line = {
         "metric": "tree tokens/s at 7B bs1 (draft-and-verify step)",
         "value": value, "unit": "tree tokens/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic: random-init N(0,0.02) weights, uniform-random prompt ids",
-        "config": {"workload": "7B-shaped bs1 draft-and-verify step (N=64, topk 5,5,5,5, 512-token prompt)",
-                   "batch": B, "tree_nodes": N, "prompt_len": len(prompt), "n_ctx": [n0, n1],
-                   "parallelism": "replicas" if world > 1 else "single",
-                   "precision": "bf16 weights; split hi+lo bf16 GEMM operands, fp32 accumulation, "
-                                "KV cache as hi+lo bf16 planes (fp32-equivalent)",
-                   "l2": "inputs larger than L2: 17.8 GB of weights streamed per step"},
+        "config": dict(workload_config(cfg, len(prompt)),
+                       n_ctx=[n0, n1], parallelism="replicas" if world > 1 else "single",
+                       precision="bf16 weights; split hi+lo bf16 GEMM operands, fp32 accumulation, "
+                                 "KV cache as hi+lo bf16 planes",
+                       l2="inputs larger than L2: 17.8 GB of weights streamed per step"),
         "breakdown": {
-            "verify_ms_eager": phase_ms["verify"], "draft_ms_eager": phase_ms["draft"],
-            "commit_ms_eager": phase_ms["commit"], "step_ms_eager": eager_ms,
+            "verify_ms": verify_med, "verify_ms_p90": verify_p90, "draft_ms": draft_med, "commit_ms": commit_med,
+            "phase_timing": "CUDA events at the phase boundaries of a graph replay of the step, one step at a time",
+            "verify_tree_tokens_per_s": B * N / (verify_med * 1e-3),
             "step_ms_median": step_median, "step_ms_p90": step_p90,
-            "kernel_ms_by_kind": {k: round(v, 4) for k, v in sorted(kind_ms.items(), key=lambda t: -t[1])},
             "step_bytes_gb": nb["total"] / 1e9, "verify_bytes_gb": nb["verify"] / 1e9,
+            "kv_bytes_basis": "bf16 K and V values read (algorithmic); the hi+lo planes read "
+                              f"{nb['kv_planes_extra'] / 1e9:.3f} GB more per step",
             "achieved_step_gbs": nb["total"] / (ms * 1e-3) / 1e9,
             "step_roofline_frac": nb["total"] / (ms * 1e-3) / 1e9 / hbm,
             "step_roofline_frac_8tbs": nb["total"] / (ms * 1e-3) / 1e9 / 8000.0,
-            "verify_roofline_frac_eager": nb["verify"] / (phase_ms["verify"] * 1e-3) / 1e9 / hbm,
+            "verify_achieved_gbs": nb["verify"] / (verify_med * 1e-3) / 1e9,
+            "verify_roofline_frac": nb["verify"] / (verify_med * 1e-3) / 1e9 / hbm,
+            "verify_roofline_frac_8tbs": nb["verify"] / (verify_med * 1e-3) / 1e9 / 8000.0,
+            "verify_roofline_ms": nb["verify"] / (hbm * 1e9) * 1e3,
+            "attention_class_ms": att["ms"], "attention_launches": att["launches"],
+            "kernel_ms_by_kind_eager": {k: round(v, 4) for k, v in sorted(kind_ms.items(), key=lambda t: -t[1])},
             "mean_accepted_tokens_per_step": mean_accept,
         },
-        "roofline": {"bound": "hbm", "kernel": "linear_tc (tcgen05 weight-streaming linear)",
+        "roofline": {"bound": "hbm", "kernel": "tc_linear_kernel (tcgen05 weight-streaming linear)",
                      "achieved": lin_gbs, "peak": hbm, "peak_kind": peak_kind, "unit": "GB/s",
-                     "frac": lin_gbs / hbm, "traffic": LINEAR_DRAM_BYTES_PER_STEP,
-                     "traffic_basis": "DRAM bytes read + written by all linear launches of one step (ncu)",
-                     "launches_per_step": lin_n, "bytes_per_step": lin_bytes, "ms_per_step": lin_ms},
+                     "frac": lin_gbs / hbm,
+                     "traffic": (ratio * lin_bytes_per_launch) if ratio else None,
+                     "traffic_basis": ("DRAM bytes per launch: small-case ncu ratio x algorithmic bytes"
+                                       if ratio else f"no capture of this kernel source ({src_hash[:12]})"),
+                     "bytes_per_launch": lin_bytes_per_launch, "ms_per_launch": lin_per_launch_ms,
+                     "launches_per_step": lin["launches"], "ms_per_step": lin["ms"],
+                     "timing": "CUDA events around back-to-back replays of a graph holding only the step's "
+                               "linear launches (step order, programmatic dependent launch kept)"},
         "cpu_baseline": cpu,
         "e2e": {"value": job_rate(B * N, world, t_e2e * 1e3), "unit": "tree tokens/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": d2h, "ms_per_step": t_e2e * 1e3},
         "gpu_launches": launches * args.steps,
         "clocks": clk,
     }
-    ctx.close()
+    if args.layers:
+        line["config"]["workload"] += f" [profiling run: {args.layers} base layers, not the benchmark workload]"
     if rank == 0:
         print(json.dumps(line))
     if world > 1:

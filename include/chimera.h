@@ -170,6 +170,24 @@ enum { CHIMERA_PHASE_DRAFT = 0, CHIMERA_PHASE_VERIFY = 1, CHIMERA_PHASE_COMMIT =
 chimera_status chimera_profile_step(chimera_ctx* ctx, int max, int32_t* kinds, int32_t* phases,
                                     float* ms, double* bytes, int32_t* count);
 
+/* Phase-timed steps (benchmark hook): n_steps steps replayed from a graph that records
+ * an event at each phase boundary (draft | tree + verify forward + LM head + argmax |
+ * acceptance + compaction + draft-KV append), with a synchronisation after each step.
+ * draft_ms / verify_ms / commit_ms: host float [n_steps] (any may be NULL).  The steps
+ * advance the state like chimera_step_async. */
+chimera_status chimera_profile_phases(chimera_ctx* ctx, int n_steps, float* draft_ms, float* verify_ms,
+                                      float* commit_ms);
+
+/* One kernel class in isolation (benchmark hook): a graph holding only the launches of
+ * class `kind` of one step, in step order and with the step's launch attributes, is
+ * replayed n_reps times back to back between two events.  *ms: mean time of one
+ * replay; *launches, *bytes (may be NULL): launches per replay and their algorithmic
+ * HBM bytes.  The launches read whatever their inputs hold and overwrite only step
+ * scratch, which the next step recomputes; classes that update the committed state
+ * (acceptance, compaction, the state update) are refused with EINVAL. */
+chimera_status chimera_profile_kind(chimera_ctx* ctx, int kind, int n_reps, float* ms, int32_t* launches,
+                                    double* bytes);
+
 /* ---- test hooks (part of the library; used by the parity tests) ---- */
 
 /* Replace the drafted tokens of tree nodes 1..N-1 for the NEXT step only

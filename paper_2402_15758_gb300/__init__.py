@@ -66,6 +66,8 @@ _SIGS = {
     "chimera_last_error": (ctypes.c_char_p, [ctypes.c_void_p]),
     "chimera_tree": (ctypes.c_int, [ctypes.c_void_p] + [ctypes.c_void_p] * 4),
     "chimera_profile_step": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int] + [ctypes.c_void_p] * 5),
+    "chimera_profile_phases": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int] + [ctypes.c_void_p] * 3),
+    "chimera_profile_kind": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int, ctypes.c_int] + [ctypes.c_void_p] * 3),
     "chimera_debug_override_tree": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p]),
     "chimera_debug_set_root": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p]),
     "chimera_debug_read": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p, ctypes.c_size_t]),
@@ -229,6 +231,25 @@ class Chimera:
         n = min(cnt.value, max_launches)
         return [dict(kind=KIND[int(kinds[i])], phase=PHASE[int(phases[i])], ms=float(ms[i]), bytes=float(by[i]))
                 for i in range(n)]
+
+    def profile_phases(self, n_steps: int):
+        """Per-step (draft, verify, commit) ms of n_steps phase-timed graph replays."""
+        d = np.zeros(n_steps, np.float32)
+        v = np.zeros(n_steps, np.float32)
+        c = np.zeros(n_steps, np.float32)
+        self._check(self.lib.chimera_profile_phases(self.h, n_steps, d.ctypes.data, v.ctypes.data, c.ctypes.data))
+        return d.tolist(), v.tolist(), c.tolist()
+
+    def profile_kind(self, kind: str, n_reps: int):
+        """Mean ms of one replay of a graph holding only one kernel class's launches of
+        the step, with its launch count and algorithmic bytes."""
+        code = {v: k for k, v in KIND.items()}[kind]
+        ms = ctypes.c_float(0)
+        n = ctypes.c_int32(0)
+        by = ctypes.c_double(0)
+        self._check(self.lib.chimera_profile_kind(self.h, code, n_reps, ctypes.byref(ms), ctypes.byref(n),
+                                                  ctypes.byref(by)))
+        return dict(ms=ms.value, launches=n.value, bytes=by.value)
 
     # ---- test hooks ----
     def override_tree(self, node_tokens):

@@ -231,6 +231,16 @@ struct chimera_ctx {
   size_t prof_count = 0;
   int cur_phase = 0;
   int last_kind = 0;  // kernel class of the latest launch (CHIMERA_KIND_*)
+  // graph of the step with an event at each phase boundary (draft | verify | commit)
+  cudaGraphExec_t phase_graph = nullptr;
+  cudaEvent_t phase_ev[4] = {nullptr, nullptr, nullptr, nullptr};
+  bool phase_marks = false;
+  // graph of only one kernel class's launches of the step, in step order
+  int filter_kind = 0;  // 0: every launch is enqueued
+  cudaGraphExec_t class_graph = nullptr;
+  int class_graph_kind = 0;
+  size_t class_launches = 0;
+  double class_bytes = 0;
 
   std::string err;
   std::vector<void*> allocs;
@@ -266,6 +276,9 @@ bool dalloc_bytes(chimera_ctx* ctx, void** p, size_t bytes) {
   return true;
 }
 
+// True when a launch of class `kind` is left out of the graph being captured.
+bool filtered(const chimera_ctx* ctx, int kind) { return ctx->filter_kind != 0 && ctx->filter_kind != kind; }
+
 // ---------------------------------------------------------------------------
 // launch helpers (events around every launch when profiling)
 // ---------------------------------------------------------------------------
@@ -274,6 +287,10 @@ struct Scope {
   ProfEvent* ev = nullptr;
   Scope(chimera_ctx* ctx, int kind, double bytes) : c(ctx) {
     c->last_kind = kind;
+    if (c->filter_kind == kind) {
+      ++c->class_launches;
+      c->class_bytes += bytes;
+    }
     if (!c->prof) return;
     if (c->prof_used == c->prof_ev.size()) {
       ProfEvent e{};
@@ -294,7 +311,7 @@ struct Scope {
 };
 
 cudaError_t run_lin(chimera_ctx* ctx, const Lin& l) {
-  if (l.N == 0) return cudaSuccess;  // folded into the previous call site
+  if (l.N == 0 || filtered(ctx, CHIMERA_KIND_LINEAR)) return cudaSuccess;  // N = 0: folded into the previous site
   Scope sc(ctx, CHIMERA_KIND_LINEAR, l.bytes);
   if (l.tc) return tc_linear_launch(l.tp, ctx->stream);
   cudaError_t e = f32_linear(l.M, l.N, l.K, static_cast<const float*>(l.X), l.ldx, static_cast<const float*>(l.W),
@@ -359,7 +376,8 @@ cudaError_t run_attention(chimera_ctx* ctx, bool draft_pool, int layer, int nq, 
                           int n_local, const int* n_local_dev, const unsigned long long* anc, int q_rows, int splits,
                           int nq_max, double bytes, const float* qkv = nullptr, int pos_base = 0,
                           const int* pos_off = nullptr) {
-  if (qkv && !(ctx->dtype == 1 && ctx->last_kind == CHIMERA_KIND_LINEAR)) {
+  if (filtered(ctx, CHIMERA_KIND_ATTENTION)) return cudaSuccess;
+  if (qkv && !ctx->filter_kind && !(ctx->dtype == 1 && ctx->last_kind == CHIMERA_KIND_LINEAR)) {
     ctx->err = "attention with early KV reads must directly follow a tensor-core linear";
     return cudaErrorInvalidValue;
   }
@@ -410,6 +428,7 @@ cudaError_t run_attention(chimera_ctx* ctx, bool draft_pool, int layer, int nq, 
 cudaError_t run_rope(chimera_ctx* ctx, bool draft_pool, int layer, const float* src, int ldsrc, int q_col, int k_col,
                      int v_col, int rows_per_seq, const int* valid, int valid_plus, int pos_base, int slot_base,
                      const int* pos_off) {
+  if (filtered(ctx, CHIMERA_KIND_ROPE_KV)) return cudaSuccess;
   Scope sc(ctx, CHIMERA_KIND_ROPE_KV, 0);
   RopeKvParams p{};
   p.qkv = src;
@@ -444,6 +463,7 @@ cudaError_t run_rope(chimera_ctx* ctx, bool draft_pool, int layer, const float* 
 // RMSNorm of fp32 rows into the GEMM operand buffer xn (+ lo half); zeroes the rows of
 // Z (zcols floats, pitch zcols) that the following linear accumulates into.
 cudaError_t run_norm(chimera_ctx* ctx, const float* X, const void* g, int rows, float* Z, int zcols) {
+  if (filtered(ctx, CHIMERA_KIND_NORM)) return cudaSuccess;
   Scope sc(ctx, CHIMERA_KIND_NORM, 0);
   return rmsnorm(ctx->dtype, X, ctx->d, g, ctx->xn, ctx->xn_lo, nullptr, ctx->d, rows, ctx->d, ctx->cfg.rms_eps, Z,
                  zcols, zcols, ctx->stream);
@@ -452,6 +472,7 @@ cudaError_t run_norm(chimera_ctx* ctx, const float* X, const void* g, int rows, 
 // Final norm: H_LLM rows in fp32 plus the LM-head operand (+ lo half); zeroes the
 // logits rows when the LM head follows.
 cudaError_t run_final_norm(chimera_ctx* ctx, int rows, bool zero_logits) {
+  if (filtered(ctx, CHIMERA_KIND_NORM)) return cudaSuccess;
   Scope sc(ctx, CHIMERA_KIND_NORM, 0);
   return rmsnorm(ctx->dtype, ctx->x, ctx->d, ctx->final_norm, ctx->hfin, ctx->hfin_lo, ctx->hfin32, ctx->d, rows,
                  ctx->d, ctx->cfg.rms_eps, zero_logits ? ctx->logits : nullptr, ctx->V, ctx->V, ctx->stream);
@@ -462,6 +483,21 @@ cudaError_t run_final_norm(chimera_ctx* ctx, int rows, bool zero_logits) {
     cudaError_t e_ = (call);                                 \
     if (e_ != cudaSuccess) return e_;                        \
   } while (0)
+
+// One launch of class `kind` (left out when the capture keeps another class only).
+#define LAUNCH(kind, bytes, call)                            \
+  do {                                                       \
+    if (!filtered(ctx, kind)) {                              \
+      Scope sc_(ctx, kind, bytes);                           \
+      RUN(call);                                             \
+    }                                                        \
+  } while (0)
+
+// Phase boundary of the step (an event node in the phase-timed graph).
+cudaError_t mark_phase(chimera_ctx* ctx, int i) {
+  if (!ctx->phase_marks) return cudaSuccess;
+  return cudaEventRecordWithFlags(ctx->phase_ev[i], ctx->stream, cudaEventRecordExternal);
+}
 
 char* eoff(const chimera_ctx* ctx, void* base, size_t elems) {
   return static_cast<char*>(base) + elems * ctx->esz;
@@ -489,10 +525,7 @@ cudaError_t enqueue_layer(chimera_ctx* ctx, int l, const Lin* lin, int rows, int
   RUN(run_norm(ctx, ctx->x, w.ffn_norm, rows, z ? ctx->gu : nullptr, 2 * ctx->F));
   RUN(run_lin(ctx, lin[2]));
   RUN(run_lin(ctx, lin[3]));
-  {
-    Scope sc(ctx, CHIMERA_KIND_SWIGLU, 0);
-    RUN(swiglu(ctx->dtype, ctx->gu, 2 * ctx->F, ctx->F, ctx->hf, ctx->hf_lo, ctx->F, rows, ctx->stream));
-  }
+  LAUNCH(CHIMERA_KIND_SWIGLU, 0, swiglu(ctx->dtype, ctx->gu, 2 * ctx->F, ctx->F, ctx->hf, ctx->hf_lo, ctx->F, rows, ctx->stream));
   RUN(run_lin(ctx, lin[4]));
   return cudaSuccess;
 }
@@ -512,12 +545,10 @@ cudaError_t enqueue_step(chimera_ctx* ctx) {
   (void)F;
   // ---- draft: K sequential sub-steps ----
   ctx->cur_phase = CHIMERA_PHASE_DRAFT;
+  RUN(mark_phase(ctx, 0));
   for (int k = 0; k < K; ++k) {
-    {
-      Scope sc(ctx, CHIMERA_KIND_EMBED, 0);
-      RUN(launch_trigram_gather(ctx->dtype, ctx->embed, d, V, ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_topk, K,
+    LAUNCH(CHIMERA_KIND_EMBED, 0, launch_trigram_gather(ctx->dtype, ctx->embed, d, V, ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_topk, K,
                                 ctx->KMAX, k, ctx->tbuf, B, ctx->d_err, ctx->dres, s));
-    }
     RUN(run_lin(ctx, ctx->tri1));
     RUN(run_lin(ctx, ctx->tri2));
     RUN(run_norm(ctx, ctx->dres, ctx->draft.attn_norm, B, ctx->qkv, 3 * d));
@@ -534,74 +565,60 @@ cudaError_t enqueue_step(chimera_ctx* ctx) {
     RUN(run_norm(ctx, ctx->dres, ctx->draft.ffn_norm, B, ctx->gu, 2 * ctx->F));
     RUN(run_lin(ctx, ctx->dgate));
     RUN(run_lin(ctx, ctx->dup));
-    {
-      Scope sc(ctx, CHIMERA_KIND_SWIGLU, 0);
-      RUN(swiglu(ctx->dtype, ctx->gu, 2 * ctx->F, ctx->F, ctx->hf, ctx->hf_lo, ctx->F, B, s));
-    }
+    LAUNCH(CHIMERA_KIND_SWIGLU, 0, swiglu(ctx->dtype, ctx->gu, 2 * ctx->F, ctx->F, ctx->hf, ctx->hf_lo, ctx->F, B, s));
     RUN(run_lin(ctx, ctx->ddown));
-    {
-      Scope sc(ctx, CHIMERA_KIND_OTHER, 0);
-      RUN(launch_hfull_store(ctx->dtype, ctx->dres, d, ctx->headin, ctx->headin_lo,
+    LAUNCH(CHIMERA_KIND_OTHER, 0, launch_hfull_store(ctx->dtype, ctx->dres, d, ctx->headin, ctx->headin_lo,
                              ctx->hfull_log + static_cast<size_t>(k) * B * d, ctx->hlog + static_cast<size_t>(k) * B * V,
                              V, B, s));
-    }
     RUN(run_lin(ctx, ctx->dhead[k]));
-    {
-      Scope sc(ctx, CHIMERA_KIND_TOPK, 0);
-      RUN(topk_rows(ctx->hlog + static_cast<size_t>(k) * B * V, V, B, ctx->KMAX, ctx->d_topk + k * ctx->KMAX,
+    LAUNCH(CHIMERA_KIND_TOPK, 0, topk_rows(ctx->hlog + static_cast<size_t>(k) * B * V, V, B, ctx->KMAX, ctx->d_topk + k * ctx->KMAX,
                     ctx->d_topk_val + k * ctx->KMAX, K * ctx->KMAX, ctx->topk_ws_v, ctx->topk_ws_i,
                     ctx->topk_cnt, s));
-    }
   }
   // ---- tree ----
   ctx->cur_phase = CHIMERA_PHASE_VERIFY;
-  {
-    Scope sc(ctx, CHIMERA_KIND_TREE, 0);
-    RUN(launch_tree_expand(ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_topk, K, ctx->KMAX, ctx->d_depth, ctx->d_rank,
+  RUN(mark_phase(ctx, 1));
+  LAUNCH(CHIMERA_KIND_TREE, 0, launch_tree_expand(ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_topk, K, ctx->KMAX, ctx->d_depth, ctx->d_rank,
                            N, ctx->d_ovr_flag, ctx->d_ovr, ctx->d_node_tok, B, s));
-  }
   // ---- verify: one base forward over every tree node ----
-  {
-    Scope sc(ctx, CHIMERA_KIND_EMBED, 0);
-    RUN(embed(ctx->dtype, ctx->embed, d, V, ctx->x, B * N, N, ctx->d_node_tok, nullptr, 0, nullptr, nullptr,
+  LAUNCH(CHIMERA_KIND_EMBED, 0, embed(ctx->dtype, ctx->embed, d, V, ctx->x, B * N, N, ctx->d_node_tok, nullptr, 0, nullptr, nullptr,
               ctx->d_err, s));
-  }
   const double kvb = kv_read_bytes(ctx, N, false);
   for (int l = 0; l < ctx->L; ++l)
     RUN(enqueue_layer(ctx, l, &ctx->ver[5 * l], B * N, N, nullptr, ctx->d_depth, ctx->d_anc, ctx->att_splits_ver, kvb));
   RUN(run_final_norm(ctx, B * N, true));
   RUN(run_lin(ctx, ctx->ver_lm));
-  {
-    Scope sc(ctx, CHIMERA_KIND_ARGMAX, 0);
-    RUN(argmax_rows(ctx->logits, V, B * N, ctx->d_amax, s));
-  }
+  LAUNCH(CHIMERA_KIND_ARGMAX, 0, argmax_rows(ctx->logits, V, B * N, ctx->d_amax, s));
   // ---- accept and commit ----
   ctx->cur_phase = CHIMERA_PHASE_COMMIT;
-  {
-    Scope sc(ctx, CHIMERA_KIND_ACCEPT, 0);
-    RUN(launch_accept(ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_node_tok, ctx->d_amax, ctx->d_child_start,
+  RUN(mark_phase(ctx, 2));
+  LAUNCH(CHIMERA_KIND_ACCEPT, 0, launch_accept(ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_node_tok, ctx->d_amax, ctx->d_child_start,
                       ctx->d_child, N, ctx->D1, ctx->d_path, ctx->d_L, ctx->d_bonus, B, s));
-  }
-  {
-    Scope sc(ctx, CHIMERA_KIND_COMPACT, 0);
-    RUN(launch_compact(ctx->kv, ctx->kv_layer_stride * static_cast<long long>(ctx->kv_esz), ctx->L, ctx->H,
+  LAUNCH(CHIMERA_KIND_COMPACT, 0, launch_compact(ctx->kv, ctx->kv_layer_stride * static_cast<long long>(ctx->kv_esz), ctx->L, ctx->H,
                        ctx->kv_planes, static_cast<int>(ctx->hd * ctx->kv_esz), ctx->d_n, ctx->d_path, ctx->d_L,
                        ctx->D1, ctx->d_pt, ctx->max_pages, B, s));
-  }
-  {
-    Scope sc(ctx, CHIMERA_KIND_OTHER, 0);
-    RUN(launch_gather_hidden(ctx->dtype, ctx->hfin32, d, N, ctx->d_path, ctx->d_L, ctx->D1, ctx->hsel, ctx->headin,
+  LAUNCH(CHIMERA_KIND_OTHER, 0, launch_gather_hidden(ctx->dtype, ctx->hfin32, d, N, ctx->d_path, ctx->d_L, ctx->D1, ctx->hsel, ctx->headin,
                              ctx->headin_lo, B, s));
-  }
   RUN(run_norm(ctx, ctx->hsel, ctx->draft.attn_norm, B * ctx->D1, ctx->kvtmp, 2 * d));
   RUN(run_lin(ctx, ctx->commit_kv));
   RUN(run_rope(ctx, true, 0, ctx->kvtmp, 2 * d, -1, 0, d, ctx->D1, ctx->d_L, 1, 0, 0, nullptr));
-  {
-    Scope sc(ctx, CHIMERA_KIND_OTHER, 0);
-    RUN(launch_finalize(ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_L, ctx->d_bonus, ctx->d_count_log, LOG_CAP,
+  LAUNCH(CHIMERA_KIND_OTHER, 0, launch_finalize(ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_L, ctx->d_bonus, ctx->d_count_log, LOG_CAP,
                         ctx->d_step, B, s));
-  }
+  RUN(mark_phase(ctx, 3));
   return cudaSuccess;
+}
+
+// Capture the step into a graph with the given capture-time options.
+cudaError_t capture_step(chimera_ctx* ctx, cudaGraphExec_t* out) {
+  cudaGraph_t g = nullptr;
+  cudaError_t e = cudaStreamBeginCapture(ctx->stream, cudaStreamCaptureModeThreadLocal);
+  if (e != cudaSuccess) return e;
+  e = enqueue_step(ctx);
+  cudaError_t e2 = cudaStreamEndCapture(ctx->stream, &g);
+  if (e == cudaSuccess) e = e2;
+  if (e == cudaSuccess) e = cudaGraphInstantiate(out, g, 0);
+  if (g) cudaGraphDestroy(g);
+  return e;
 }
 
 // (Re)build every linear call site for `batch` sequences.
@@ -784,6 +801,10 @@ void free_ctx(chimera_ctx* ctx) {
   if (!ctx) return;
   if (ctx->graph) cudaGraphExecDestroy(ctx->graph);
   if (ctx->prof_graph) cudaGraphExecDestroy(ctx->prof_graph);
+  if (ctx->phase_graph) cudaGraphExecDestroy(ctx->phase_graph);
+  if (ctx->class_graph) cudaGraphExecDestroy(ctx->class_graph);
+  for (auto& e : ctx->phase_ev)
+    if (e) cudaEventDestroy(e);
   for (auto& e : ctx->prof_ev) {
     cudaEventDestroy(e.a);
     cudaEventDestroy(e.b);
@@ -1050,6 +1071,14 @@ chimera_status chimera_prefill(chimera_ctx* ctx, int batch, const int32_t* token
     cudaGraphExecDestroy(ctx->prof_graph);
     ctx->prof_graph = nullptr;
   }
+  if (ctx->phase_graph) {
+    cudaGraphExecDestroy(ctx->phase_graph);
+    ctx->phase_graph = nullptr;
+  }
+  if (ctx->class_graph) {
+    cudaGraphExecDestroy(ctx->class_graph);
+    ctx->class_graph = nullptr;
+  }
   ctx->batch = batch;
   ctx->plan_keys = max_len;
   if (!build_plans(ctx, batch)) return CHIMERA_EINVAL;
@@ -1220,6 +1249,89 @@ chimera_status chimera_profile_step(chimera_ctx* ctx, int max, int32_t* kinds, i
   }
   *count = n;
   CK(cudaMemcpy(ctx->host_n.data(), ctx->d_n, ctx->batch * sizeof(int), cudaMemcpyDeviceToHost));
+  return check_err(ctx);
+}
+
+chimera_status chimera_profile_phases(chimera_ctx* ctx, int n_steps, float* draft_ms, float* verify_ms,
+                                      float* commit_ms) {
+  if (!ctx) return CHIMERA_EINVAL;
+  if (n_steps < 1) return fail(ctx, CHIMERA_EINVAL, "n_steps < 1");
+  chimera_status st = steps_prepare(ctx, n_steps);
+  if (st != CHIMERA_OK) return st;
+  if (!ctx->phase_graph) {
+    for (auto& e : ctx->phase_ev)
+      if (!e) CK(cudaEventCreate(&e));
+    ctx->phase_marks = true;
+    cudaError_t e = capture_step(ctx, &ctx->phase_graph);
+    ctx->phase_marks = false;
+    if (e != cudaSuccess) {
+      ctx->phase_graph = nullptr;
+      return fail(ctx, CHIMERA_ECUDA, std::string("capturing the phase-timed step: ") + cudaGetErrorString(e));
+    }
+  }
+  if (ctx->ovr_pending) {
+    const int one = 1;
+    CK(cudaMemcpyAsync(ctx->d_ovr_flag, &one, sizeof(int), cudaMemcpyHostToDevice, ctx->stream));
+  }
+  for (int i = 0; i < n_steps; ++i) {
+    CK(cudaGraphLaunch(ctx->phase_graph, ctx->stream));
+    if (i == 0 && ctx->ovr_pending) {
+      CK(cudaMemsetAsync(ctx->d_ovr_flag, 0, sizeof(int), ctx->stream));
+      ctx->ovr_pending = false;
+    }
+    CK(cudaStreamSynchronize(ctx->stream));
+    float t[3] = {0, 0, 0};
+    for (int p = 0; p < 3; ++p) CK(cudaEventElapsedTime(&t[p], ctx->phase_ev[p], ctx->phase_ev[p + 1]));
+    if (draft_ms) draft_ms[i] = t[0];
+    if (verify_ms) verify_ms[i] = t[1];
+    if (commit_ms) commit_ms[i] = t[2];
+  }
+  CK(cudaMemcpy(ctx->host_n.data(), ctx->d_n, ctx->batch * sizeof(int), cudaMemcpyDeviceToHost));
+  return check_err(ctx);
+}
+
+chimera_status chimera_profile_kind(chimera_ctx* ctx, int kind, int n_reps, float* ms, int32_t* launches,
+                                    double* bytes) {
+  if (!ctx) return CHIMERA_EINVAL;
+  // classes whose kernels write only step scratch (never n, the token history or
+  // committed KV rows), so the replays leave the committed state intact
+  const bool allowed = kind == CHIMERA_KIND_LINEAR || kind == CHIMERA_KIND_ATTENTION || kind == CHIMERA_KIND_NORM ||
+                       kind == CHIMERA_KIND_SWIGLU || kind == CHIMERA_KIND_EMBED || kind == CHIMERA_KIND_TOPK ||
+                       kind == CHIMERA_KIND_ARGMAX || kind == CHIMERA_KIND_ROPE_KV;
+  if (!allowed || n_reps < 1 || !ms) return fail(ctx, CHIMERA_EINVAL, "bad kernel class or repetition count");
+  chimera_status st = steps_prepare(ctx, 1);
+  if (st != CHIMERA_OK) return st;
+  if (ctx->class_graph && ctx->class_graph_kind != kind) {
+    CK(cudaGraphExecDestroy(ctx->class_graph));
+    ctx->class_graph = nullptr;
+  }
+  if (!ctx->class_graph) {
+    ctx->filter_kind = kind;
+    ctx->class_launches = 0;
+    ctx->class_bytes = 0;
+    cudaError_t e = capture_step(ctx, &ctx->class_graph);
+    ctx->filter_kind = 0;
+    if (e != cudaSuccess) {
+      ctx->class_graph = nullptr;
+      return fail(ctx, CHIMERA_ECUDA, std::string("capturing the kernel-class graph: ") + cudaGetErrorString(e));
+    }
+    ctx->class_graph_kind = kind;
+  }
+  cudaEvent_t a, b;
+  CK(cudaEventCreate(&a));
+  CK(cudaEventCreate(&b));
+  CK(cudaGraphLaunch(ctx->class_graph, ctx->stream));  // warm-up
+  CK(cudaEventRecord(a, ctx->stream));
+  for (int i = 0; i < n_reps; ++i) CK(cudaGraphLaunch(ctx->class_graph, ctx->stream));
+  CK(cudaEventRecord(b, ctx->stream));
+  CK(cudaEventSynchronize(b));
+  float t = 0;
+  CK(cudaEventElapsedTime(&t, a, b));
+  cudaEventDestroy(a);
+  cudaEventDestroy(b);
+  *ms = t / n_reps;
+  if (launches) *launches = static_cast<int32_t>(ctx->class_launches);
+  if (bytes) *bytes = ctx->class_bytes;
   return check_err(ctx);
 }
 
