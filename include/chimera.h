@@ -136,6 +136,16 @@ chimera_status chimera_generate(chimera_ctx* ctx, int n_steps, int32_t* out_toke
  * (no host output; capacity checked for the worst case).  For timing. */
 chimera_status chimera_step_async(chimera_ctx* ctx, int n_steps);
 
+/* n_steps plain autoregressive steps (eq. 1 with argmax: one base forward per token),
+ * the baseline that speculative decoding accelerates.  Each step runs the base model
+ * on every sequence's root x[n] at position n, emits that root, writes its KV at slot n,
+ * appends its draft-layer KV and makes the argmax the next root: the same state update
+ * as a draft-and-verify step that accepts no drafted token, so the two kinds of step
+ * can be mixed and produce the same stream.  out_tokens: host int32 [batch][n_steps]
+ * (NULL: enqueue only, for timing; then out_count is ignored and chimera_sync
+ * completes the steps); out_count: host int32 [batch] (= n_steps). */
+chimera_status chimera_ar_generate(chimera_ctx* ctx, int n_steps, int32_t* out_tokens, int32_t* out_count);
+
 /* Block until the context stream is idle and report device-side errors. */
 chimera_status chimera_sync(chimera_ctx* ctx);
 

@@ -314,8 +314,17 @@ def draft(W: OracleWeights, cfg: dict, st: SeqState, kmax: int) -> dict:
     """K sequential sub-steps (reading R5).  Sub-step k encodes the trigram ending at
     x[n+k] (x[n] = root, x[n+1+j] = head j's top-1), runs the full-context block on
     it at position n+k against the committed draft KV (0..n-1) plus the trigram rows
-    of sub-steps 0..k, and scores head k on [H_LLM[n-1]; h_full]."""
+    of sub-steps 0..k, and scores head k on [H_LLM[n-1]; h_full].
+
+    cfg["draft_mode"] selects the ablation variants of the draft (Section "Residual
+    decoding heads" and its ablation):
+      bit 0 (one pass): only sub-step 0 runs; every head k scores h_full_{n+1}
+        (the alternative reading of eq. "residual decoding head" with one trigram row);
+      bit 1 (no residual): head k scores h_full alone, Theta_k in R^{|V| x d}
+        (the "w/o residual" variant of the ablation figure)."""
     n, K = st.n, cfg["n_draft_heads"]
+    mode = cfg.get("draft_mode", 0)
+    one_pass, no_resid = bool(mode & 1), bool(mode & 2)
     chain = [st.tokens[n]]
     tk, tv, top, logits, hfull, htri = [], [], [], [], [], []
 
@@ -325,21 +334,23 @@ def draft(W: OracleWeights, cfg: dict, st: SeqState, kmax: int) -> dict:
         return st.tokens[i] if i <= n else chain[i - n]
 
     for k in range(K):
-        t = trigram_input(W, cfg, [tok(n - 2 + k), tok(n - 1 + k), tok(n + k)])
-        g = trigram_encoder(W, t)
-        htri.append(g)
-        # incremental full-context block: new row at position n+k
-        # the new row sees the committed draft KV, the earlier trigram rows (given
-        # as context) and itself (its only local row).
-        ctx_k = np.concatenate([st.dK[:n]] + [kk[None] for kk in tk], axis=0)
-        ctx_v = np.concatenate([st.dV[:n]] + [vv[None] for vv in tv], axis=0)
-        out, k_new, v_new = block_rows(W, "draft", cfg, g[None, :], np.array([n + k]),
-                                       ctx_k, ctx_v, np.ones((1, 1), dtype=bool))
-        tk.append(k_new[0])
-        tv.append(v_new[0])
-        h = out[0]
+        if k == 0 or not one_pass:
+            t = trigram_input(W, cfg, [tok(n - 2 + k), tok(n - 1 + k), tok(n + k)])
+            g = trigram_encoder(W, t)
+            htri.append(g)
+            # incremental full-context block: new row at position n+k
+            # the new row sees the committed draft KV, the earlier trigram rows (given
+            # as context) and itself (its only local row).
+            ctx_k = np.concatenate([st.dK[:n]] + [kk[None] for kk in tk], axis=0)
+            ctx_v = np.concatenate([st.dV[:n]] + [vv[None] for vv in tv], axis=0)
+            out, k_new, v_new = block_rows(W, "draft", cfg, g[None, :], np.array([n + k]),
+                                           ctx_k, ctx_v, np.ones((1, 1), dtype=bool))
+            tk.append(k_new[0])
+            tv.append(v_new[0])
+            h = out[0]
         hfull.append(h)
-        z = W(f"heads.{k}") @ np.concatenate([st.Hs[n - 1], h])
+        head_in = h if no_resid else np.concatenate([st.Hs[n - 1], h])
+        z = W(f"heads.{k}") @ head_in
         logits.append(z)
         idx = topk_desc(z, kmax)
         top.append(idx)
@@ -404,6 +415,43 @@ def accept(tree: dict, node_tokens: list[int], logits: np.ndarray):
         path.append(cur)
 
 
+def typical_threshold(z: np.ndarray, eps: float, delta: float) -> tuple[np.ndarray, float]:
+    """Probabilities at temperature 1 of a score row and the typical-acceptance
+    threshold min(eps, delta * exp(-H(p))), H the entropy in nats (the typical decoding
+    of the verification step, Section "Verification"; criterion of the cited work)."""
+    z = np.asarray(z, dtype=np.float64)
+    e = np.exp(z - z.max())
+    p = e / e.sum()
+    nz = p > 0
+    H = -float(np.sum(p[nz] * np.log(p[nz])))
+    return p, min(eps, delta * np.exp(-H))
+
+
+def accept_typical(tree: dict, node_tokens: list[int], logits: np.ndarray, eps: float, delta: float):
+    """Typical acceptance (T = 1): a node is acceptable when its parent is and its token
+    has probability above the parent's typical threshold under the base model's
+    distribution at the parent.  The accepted path ends at the deepest acceptable node
+    (ties: the smallest node index, i.e. the lexicographically first rank tuple); the
+    bonus token is the base argmax there.  Returns (path, bonus)."""
+    N = tree["n"]
+    ok = [False] * N
+    ok[0] = True
+    probs = [typical_threshold(logits[i], eps, delta) for i in range(N)]
+    for c in range(1, N):
+        par = tree["parent"][c]
+        p, thr = probs[par]
+        ok[c] = ok[par] and p[node_tokens[c]] > thr
+    best = 0
+    for c in range(1, N):
+        if ok[c] and tree["depth"][c] > tree["depth"][best]:
+            best = c
+    path, j = [], best
+    while j >= 0:
+        path.append(j)
+        j = tree["parent"][j]
+    return path[::-1], argmax_desc(logits[best])
+
+
 def commit(W: OracleWeights, cfg: dict, st: SeqState, node_tokens: list[int], ver: dict,
            path: list[int], bonus: int) -> list[int]:
     """State update (reading R13): the path's tokens, base KV and H_LLM rows become
@@ -424,7 +472,9 @@ def commit(W: OracleWeights, cfg: dict, st: SeqState, node_tokens: list[int], ve
 
 def step(W: OracleWeights, cfg: dict, st: SeqState, tree: dict, override=None) -> dict:
     """One draft-and-verify step.  `override` replaces the drafted node tokens
-    (nodes 1..N-1) to force acceptance lengths in tests."""
+    (nodes 1..N-1) to force acceptance lengths in tests.  cfg["accept_mode"] = 1 takes
+    the typical acceptance (thresholds cfg["typical_eps"], cfg["typical_delta"])
+    instead of the greedy one."""
     kmax = max(cfg["topk"])
     dr = draft(W, cfg, st, kmax)
     toks = tree_tokens(tree, st.tokens[st.n], dr["topk"])
@@ -432,7 +482,10 @@ def step(W: OracleWeights, cfg: dict, st: SeqState, tree: dict, override=None) -
         toks = [toks[0]] + [int(t) for t in override[1:]]
     n_before = st.n
     ver = verify(W, cfg, st, tree, toks)
-    path, bonus = accept(tree, toks, ver["logits"])
+    if cfg.get("accept_mode", 0) == 1:
+        path, bonus = accept_typical(tree, toks, ver["logits"], cfg["typical_eps"], cfg["typical_delta"])
+    else:
+        path, bonus = accept(tree, toks, ver["logits"])
     emitted = commit(W, cfg, st, toks, ver, path, bonus)
     return dict(draft=dr, node_tokens=toks, verify=ver, path=path, bonus=bonus,
                 emitted=emitted, n_before=n_before)

@@ -62,6 +62,7 @@ _SIGS = {
     "chimera_generate": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p]),
     "chimera_step_async": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int]),
     "chimera_sync": (ctypes.c_int, [ctypes.c_void_p]),
+    "chimera_ar_generate": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p]),
     "chimera_free": (None, [ctypes.c_void_p]),
     "chimera_last_error": (ctypes.c_char_p, [ctypes.c_void_p]),
     "chimera_tree": (ctypes.c_int, [ctypes.c_void_p] + [ctypes.c_void_p] * 4),
@@ -213,6 +214,16 @@ class Chimera:
         cnt = np.zeros(self.batch, np.int32)
         self._check(self.lib.chimera_generate(self.h, n_steps, out.ctypes.data, cnt.ctypes.data))
         return [out[b, : cnt[b]].tolist() for b in range(self.batch)]
+
+    def ar_generate(self, n_steps: int):
+        """n_steps plain autoregressive steps; per sequence the n_steps emitted tokens."""
+        out = np.zeros((self.batch, n_steps), np.int32)
+        cnt = np.zeros(self.batch, np.int32)
+        self._check(self.lib.chimera_ar_generate(self.h, n_steps, out.ctypes.data, cnt.ctypes.data))
+        return [out[b, : cnt[b]].tolist() for b in range(self.batch)]
+
+    def ar_step_async(self, n_steps: int = 1):
+        self._check(self.lib.chimera_ar_generate(self.h, n_steps, None, None))
 
     def step_async(self, n_steps: int = 1):
         self._check(self.lib.chimera_step_async(self.h, n_steps))

@@ -211,12 +211,14 @@ struct chimera_ctx {
   // plan of the current batch
   int batch = 0;
   std::vector<int> host_n;
-  std::vector<Lin> ver, pre;  // 5 per layer: qkv, wo, gate, up, down
-  Lin ver_lm, pre_lm, pre_dkv, tri1, tri2, dqkv, dwo, dgate, dup, ddown, commit_kv;
+  std::vector<Lin> ver, pre, ar;  // 5 per layer: qkv, wo, gate, up, down
+  Lin ver_lm, pre_lm, ar_lm, pre_dkv, tri1, tri2, dqkv, dwo, dgate, dup, ddown, commit_kv;
   std::vector<Lin> dhead;
-  int att_splits_ver = 1, att_splits_pre = 1, att_splits_draft = 1;
+  int att_splits_ver = 1, att_splits_pre = 1, att_splits_draft = 1, att_splits_ar = 1;
   int plan_keys = 0;  // longest prompt of the batch (sizes the attention splits)
   cudaGraphExec_t graph = nullptr;
+  cudaGraphExec_t ar_graph = nullptr;  // one plain autoregressive step (eq. 1)
+  int *d_one = nullptr, *d_child_start1 = nullptr, *d_child1 = nullptr;  // a one-node tree
   bool prefilled = false;
   bool ovr_pending = false;
 
@@ -608,12 +610,44 @@ cudaError_t enqueue_step(chimera_ctx* ctx) {
   return cudaSuccess;
 }
 
+// One plain autoregressive step (eq. 1 with argmax; the baseline that speculative
+// decoding accelerates): the base forward of each sequence's root x[n] at position n
+// (one query row attending the committed rows and itself), LM head, argmax -> the next
+// root; the root's base KV is written at slot n, its draft-layer KV appended and
+// h_LLM_n refreshed, exactly as a draft-and-verify step that accepts nothing.
+cudaError_t enqueue_ar_step(chimera_ctx* ctx) {
+  const int B = ctx->batch, d = ctx->d, V = ctx->V;
+  cudaStream_t s = ctx->stream;
+  ctx->cur_phase = CHIMERA_PHASE_VERIFY;
+  LAUNCH(CHIMERA_KIND_EMBED, 0, embed(ctx->dtype, ctx->embed, d, V, ctx->x, B, 1, nullptr, ctx->d_tok, ctx->tok_stride,
+                                      ctx->d_n, ctx->d_one, ctx->d_err, s));
+  const double kvb = kv_read_bytes(ctx, 1, false);
+  for (int l = 0; l < ctx->L; ++l)
+    RUN(enqueue_layer(ctx, l, &ctx->ar[5 * l], B, 1, nullptr, nullptr, ctx->d_chain, ctx->att_splits_ar, kvb));
+  RUN(run_final_norm(ctx, B, true));
+  RUN(run_lin(ctx, ctx->ar_lm));
+  LAUNCH(CHIMERA_KIND_ARGMAX, 0, argmax_rows(ctx->logits, V, B, ctx->d_amax, s));
+  ctx->cur_phase = CHIMERA_PHASE_COMMIT;
+  // a tree of the root alone: the path is [root], the bonus is its argmax
+  LAUNCH(CHIMERA_KIND_ACCEPT, 0, launch_accept(ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_node_tok, ctx->d_amax,
+                                               ctx->d_child_start1, ctx->d_child1, 1, ctx->D1, ctx->d_path, ctx->d_L,
+                                               ctx->d_bonus, B, s));
+  LAUNCH(CHIMERA_KIND_OTHER, 0, launch_gather_hidden(ctx->dtype, ctx->hfin32, d, 1, ctx->d_path, ctx->d_L, ctx->D1,
+                                                     ctx->hsel, ctx->headin, ctx->headin_lo, B, s));
+  RUN(run_norm(ctx, ctx->hsel, ctx->draft.attn_norm, B * ctx->D1, ctx->kvtmp, 2 * d));
+  RUN(run_lin(ctx, ctx->commit_kv));
+  RUN(run_rope(ctx, true, 0, ctx->kvtmp, 2 * d, -1, 0, d, ctx->D1, ctx->d_L, 1, 0, 0, nullptr));
+  LAUNCH(CHIMERA_KIND_OTHER, 0, launch_finalize(ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_L, ctx->d_bonus,
+                                                ctx->d_count_log, LOG_CAP, ctx->d_step, B, s));
+  return cudaSuccess;
+}
+
 // Capture the step into a graph with the given capture-time options.
-cudaError_t capture_step(chimera_ctx* ctx, cudaGraphExec_t* out) {
+cudaError_t capture_step(chimera_ctx* ctx, cudaGraphExec_t* out, bool ar = false) {
   cudaGraph_t g = nullptr;
   cudaError_t e = cudaStreamBeginCapture(ctx->stream, cudaStreamCaptureModeThreadLocal);
   if (e != cudaSuccess) return e;
-  e = enqueue_step(ctx);
+  e = ar ? enqueue_ar_step(ctx) : enqueue_step(ctx);
   cudaError_t e2 = cudaStreamEndCapture(ctx->stream, &g);
   if (e == cudaSuccess) e = e2;
   if (e == cudaSuccess) e = cudaGraphInstantiate(out, g, 0);
@@ -627,6 +661,7 @@ bool build_plans(chimera_ctx* ctx, int B) {
   const int f32 = 1, tb = ctx->dtype == 0 ? 1 : 0;  // bf16 storage -> out_f32 = 0
   ctx->ver.assign(5 * ctx->L, Lin());
   ctx->pre.assign(5 * ctx->L, Lin());
+  ctx->ar.assign(5 * ctx->L, Lin());
   // fp32 outputs accumulate (split-K partials added atomically) into buffers that the
   // preceding kernel zeroed, or into the residual stream itself
   constexpr int ACC = EPI_RESID;
@@ -652,6 +687,10 @@ bool build_plans(chimera_ctx* ctx, int B) {
     return true;
   };
   if (!layer_plans(ctx->ver, B * N)) return false;
+  if (!layer_plans(ctx->ar, B)) return false;
+  if (!make_lin(ctx, &ctx->ar_lm, B, V, d, ctx->hfin, ctx->hfin_lo, d, ctx->lm_head, ctx->logits, nullptr, V, ACC,
+                f32))
+    return false;
   if (!layer_plans(ctx->pre, B * CHUNK)) return false;
   if (!make_lin(ctx, &ctx->ver_lm, B * N, V, d, ctx->hfin, ctx->hfin_lo, d, ctx->lm_head, ctx->logits, nullptr, V,
                 ACC, f32))
@@ -686,6 +725,7 @@ bool build_plans(chimera_ctx* ctx, int B) {
   ctx->att_splits_ver = att_splits(ctx, B, N, ctx->plan_keys + N);
   ctx->att_splits_pre = att_splits(ctx, B, CHUNK, ctx->plan_keys);
   ctx->att_splits_draft = att_splits(ctx, B, 1, ctx->plan_keys);
+  ctx->att_splits_ar = att_splits(ctx, B, 1, ctx->plan_keys + 1);
   return true;
 }
 
@@ -803,6 +843,7 @@ void free_ctx(chimera_ctx* ctx) {
   if (ctx->prof_graph) cudaGraphExecDestroy(ctx->prof_graph);
   if (ctx->phase_graph) cudaGraphExecDestroy(ctx->phase_graph);
   if (ctx->class_graph) cudaGraphExecDestroy(ctx->class_graph);
+  if (ctx->ar_graph) cudaGraphExecDestroy(ctx->ar_graph);
   for (auto& e : ctx->phase_ev)
     if (e) cudaEventDestroy(e);
   for (auto& e : ctx->prof_ev) {
@@ -967,6 +1008,9 @@ chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
   ok = ok && dalloc(ctx, &ctx->d_chain, 64);
   ok = ok && dalloc(ctx, &ctx->d_child_start, N + 1);
   ok = ok && dalloc(ctx, &ctx->d_child, ctx->tree.child.size());
+  ok = ok && dalloc(ctx, &ctx->d_one, B);
+  ok = ok && dalloc(ctx, &ctx->d_child_start1, 2);
+  ok = ok && dalloc(ctx, &ctx->d_child1, 1);
   if (ctx->dtype == 1) {
     ok = ok && dalloc(ctx, &ctx->lin_ws, tc_ws_floats(256));
     ok = ok && dalloc(ctx, &ctx->lin_cnt, static_cast<size_t>(tc_max_tiles()));
@@ -1025,6 +1069,10 @@ chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
   zok = zok && cudaMemcpyAsync(ctx->d_child_start, t.child_start.data(), (N + 1) * sizeof(int), cudaMemcpyHostToDevice, s) == cudaSuccess;
   zok = zok && cudaMemcpyAsync(ctx->d_child, t.child.data(), t.child.size() * sizeof(int), cudaMemcpyHostToDevice, s) == cudaSuccess;
   zok = zok && cudaMemcpyAsync(ctx->d_rope, rope.data(), rope.size() * sizeof(float2), cudaMemcpyHostToDevice, s) == cudaSuccess;
+  const std::vector<int> ones(B, 1);
+  zok = zok && cudaMemcpyAsync(ctx->d_one, ones.data(), B * sizeof(int), cudaMemcpyHostToDevice, s) == cudaSuccess;
+  zok = zok && cudaMemsetAsync(ctx->d_child_start1, 0, 2 * sizeof(int), s) == cudaSuccess;
+  zok = zok && cudaMemsetAsync(ctx->d_child1, 0, sizeof(int), s) == cudaSuccess;
   zok = zok && cudaStreamSynchronize(s) == cudaSuccess;
   if (!zok) {
     free_ctx(ctx);
@@ -1078,6 +1126,10 @@ chimera_status chimera_prefill(chimera_ctx* ctx, int batch, const int32_t* token
   if (ctx->class_graph) {
     cudaGraphExecDestroy(ctx->class_graph);
     ctx->class_graph = nullptr;
+  }
+  if (ctx->ar_graph) {
+    cudaGraphExecDestroy(ctx->ar_graph);
+    ctx->ar_graph = nullptr;
   }
   ctx->batch = batch;
   ctx->plan_keys = max_len;
@@ -1174,6 +1226,24 @@ chimera_status chimera_step_async(chimera_ctx* ctx, int n_steps) {
   if (st != CHIMERA_OK) return st;
   // host_n is refreshed by chimera_sync
   return CHIMERA_OK;
+}
+
+chimera_status chimera_ar_generate(chimera_ctx* ctx, int n_steps, int32_t* out_tokens, int32_t* out_count) {
+  if (!ctx) return CHIMERA_EINVAL;
+  if (n_steps < 1) return fail(ctx, CHIMERA_EINVAL, "n_steps < 1");
+  chimera_status st = steps_prepare(ctx, n_steps);
+  if (st != CHIMERA_OK) return st;
+  if (!ctx->ar_graph) {
+    cudaError_t e = capture_step(ctx, &ctx->ar_graph, true);
+    if (e != cudaSuccess) {
+      ctx->ar_graph = nullptr;
+      return fail(ctx, CHIMERA_ECUDA, std::string("capturing the autoregressive step: ") + cudaGetErrorString(e));
+    }
+  }
+  for (int i = 0; i < n_steps; ++i) CK(cudaGraphLaunch(ctx->ar_graph, ctx->stream));
+  if (!out_tokens) return CHIMERA_OK;  // timing: no host output, no synchronisation
+  if (!out_count) return fail(ctx, CHIMERA_EINVAL, "NULL count");
+  return read_new_tokens(ctx, out_tokens, n_steps, out_count);
 }
 
 chimera_status chimera_sync(chimera_ctx* ctx) {

@@ -107,8 +107,9 @@ def weight_shapes(cfg: dict) -> list[tuple[str, tuple[int, ...]]]:
     out += [("final_norm", (d,)), ("lm_head", (v, d))]
     out += [("tri_w1", (d, 3 * d)), ("tri_w2", (d, d))]
     block("draft")
+    head_in = d if cfg.get("draft_mode", 0) & 2 else 2 * d  # no-residual heads read h_full alone
     for k in range(cfg["n_draft_heads"]):
-        out.append((f"heads.{k}", (v, 2 * d)))
+        out.append((f"heads.{k}", (v, head_in)))
     return out
 
 

@@ -320,3 +320,70 @@ def _host_mem_gb():
 def test_7b_full_size_step():
     # the benchmark's workload: 7B shape, bs1, 512-token prompt, 64-node tree
     _run_bf16("7b", 1, [2], device_gen="cuda", max_seq=1024)
+
+
+# ----------------------------------------------------------------------------
+# plain autoregressive steps (eq. 1): the baseline path on the same kernels
+# ----------------------------------------------------------------------------
+def test_tiny_ar_generation_matches_oracle(tiny):
+    cfg, w_dev, W, prompt = tiny
+    T = cfg["gen_tokens"]
+    ctx = pkg.Chimera(cfg, w_dev, max_batch=1, max_seq_len=256)
+    ctx.prefill([prompt])
+    out = ctx.ar_generate(T)[0]
+    assert out == co.ar_generate(W, cfg, prompt, T)
+    ctx.close()
+
+
+def test_tiny_ar_and_spec_steps_mix(tiny):
+    # both kinds of step leave the same state: any interleaving emits the AR stream
+    cfg, w_dev, W, prompt = tiny
+    ref = co.ar_generate(W, cfg, prompt, 40)
+    ctx = pkg.Chimera(cfg, w_dev, max_batch=1, max_seq_len=256)
+    ctx.prefill([prompt])
+    out = []
+    for kind in ["ar", "spec", "spec", "ar", "ar", "spec", "ar", "spec"]:
+        out += ctx.ar_generate(2)[0] if kind == "ar" else ctx.step()[0]
+    assert out == ref[: len(out)]
+    n = int(ctx.read("n")[0])
+    assert n == len(prompt) + len(out)
+    # the committed KV rows equal a from-scratch prefill of the committed tokens
+    st = co.prefill(W, cfg, prompt + out, 256)
+    for layer in list(range(cfg["n_layers"])) + [-1]:
+        k, v = ctx.read_kv(layer, 0, 0, n)
+        rk = st.dK[:n] if layer < 0 else st.K[layer, :n]
+        rv = st.dV[:n] if layer < 0 else st.V[layer, :n]
+        assert rel_rows(k, rk) <= tol_of(cfg) and rel_rows(v, rv) <= tol_of(cfg), layer
+    ctx.close()
+
+
+@pytest.mark.parametrize("name", ["mini", "mini_b4"])
+def test_bf16_ar_steps_match_oracle(name):
+    cfg, w_cpu, w_dev = _setup(name)
+    W = co.OracleWeights(w_cpu)
+    prompts = synth.make_prompts(cfg)
+    B, tol = len(prompts), tol_of(cfg)
+    ctx = pkg.Chimera(cfg, w_dev, max_batch=B, max_seq_len=256)
+    ctx.prefill(prompts)
+    seqs = [list(p) for p in prompts]
+    flags = 0
+    for b in range(B):  # the roots: the oracle's greedy next token (a near-tie may differ)
+        _, lg = co.causal_forward(W, cfg, seqs[b])
+        flags += check_choice(int(ctx.read("tokens")[b, len(seqs[b])]), lg[-1], co.argmax_desc(lg[-1]))
+        seqs[b].append(co.argmax_desc(lg[-1]))
+    ctx.set_root([s[-1] for s in seqs])
+    for step in range(5):
+        out = ctx.ar_generate(1)
+        logits = ctx.read("prefill_logits")  # the LM-head rows of the step's B query rows
+        toks = ctx.read("tokens")
+        for b in range(B):
+            assert out[b] == [seqs[b][-1]]
+            _, lg = co.causal_forward(W, cfg, seqs[b])
+            assert rel_rows(logits[b], lg[-1]) <= tol, (step, b)
+            ref = co.argmax_desc(lg[-1])
+            flags += check_choice(int(toks[b, len(seqs[b])]), lg[-1], ref)
+            seqs[b].append(ref)
+        ctx.set_root([s[-1] for s in seqs])
+    assert ctx.read("n").tolist() == [len(s) - 1 for s in seqs]
+    ctx.close()
+    print(f"{name} AR: 5 steps x {B} seqs, near-tie flags {flags}")
