@@ -75,6 +75,26 @@ typedef struct {
                            taken term by term with fp32 accumulation (~fp32 accuracy);
                            0: activations and KV entries rounded once to bf16.
                            fp32 models ignore it. */
+  int draft_mode;       /* 0: the draft of the method (K sequential sub-steps, residual heads).
+                           Ablation variants (Section "Residual decoding heads" and its
+                           ablation): bit 0 = one-pass draft (the trigram encoder and the
+                           full-context block run once, every head scores h_full_{n+1});
+                           bit 1 = heads without the residual input (Theta_k is
+                           [vocab][d_model] on h_full alone). */
+  int accept_mode;      /* 0: greedy acceptance (lossless); 1: typical acceptance at temperature
+                           1 (Section "Verification"): node c is acceptable when its parent is
+                           and p_parent(token_c) > min(typical_eps, typical_delta * exp(-H)),
+                           H the entropy of the parent's distribution; the path ends at the
+                           deepest acceptable node (smallest index among the deepest) and the
+                           bonus token is the base argmax there.  Not lossless. */
+  float typical_eps;    /* typical acceptance: hard threshold (e.g. 0.09) */
+  float typical_delta;  /* typical acceptance: entropy factor (e.g. 0.3) */
+  int trigram_cache;    /* entries of the device trigram cache (Section "Trigram encoder",
+                           lookup table): 0 = off; else a multiple of 4 with a power-of-two
+                           number of 4-way sets, <= 65536.  Each entry keeps one h_tri row
+                           (d_model fp32 values) keyed by its three token ids; the least
+                           recently used way of a set is replaced.  A sub-step whose trigrams
+                           all hit skips the encoder's two linears; results are unchanged. */
 } chimera_config;
 
 /* One Llama block: RMSNorm gains [d]; wqkv [3d][d] (rows q, then k, then v; head h
@@ -219,8 +239,13 @@ enum {
   CHIMERA_DBG_HFULL = 9,          /* f32 [K][batch][d] full-context outputs */
   CHIMERA_DBG_N = 10,             /* int32 [batch] committed length n */
   CHIMERA_DBG_TOKENS = 11,        /* int32 [batch][max_seq_len + 1] token history */
-  CHIMERA_DBG_PREFILL_LOGITS = 12 /* f32 [batch][V] LM-head scores of the last prompt row
-                                     (valid until the first step) */
+  CHIMERA_DBG_PREFILL_LOGITS = 12, /* f32 [batch][V] LM-head scores of the last prompt row
+                                      (until the first step; after chimera_ar_generate: the
+                                      scores of its last step's rows) */
+  CHIMERA_DBG_TRIGRAM_HITS = 13,  /* int32 [K][batch] 1 where the last step's sub-step hit the
+                                     trigram cache (trigram_cache > 0 only) */
+  CHIMERA_DBG_HTRI = 14           /* f32 [K][batch][d] the last step's h_tri rows (trigram_cache
+                                     > 0 only) */
 };
 /* Copy a device buffer of the context to host memory; `bytes` must equal its size. */
 chimera_status chimera_debug_read(chimera_ctx* ctx, int what, void* host_dst, size_t bytes);

@@ -19,7 +19,7 @@ HEADER = os.path.join(os.path.dirname(_PKG), "include", "chimera.h")
 STATUS = {0: "OK", -1: "EINVAL", -2: "ENOMEM", -3: "ECAPACITY", -4: "ECUDA", -5: "ETIMEDOUT", -6: "ESTATE"}
 
 DBG = dict(node_tokens=1, verify_logits=2, verify_hidden=3, argmax=4, path=5, accept_len=6,
-           draft_logits=7, topk=8, hfull=9, n=10, tokens=11, prefill_logits=12)
+           draft_logits=7, topk=8, hfull=9, n=10, tokens=11, prefill_logits=12, trigram_hits=13, htri=14)
 KIND = {1: "linear", 2: "attention", 3: "norm", 4: "rope_kv", 5: "swiglu", 6: "embed", 7: "topk",
         8: "argmax", 9: "tree", 10: "accept", 11: "compact", 12: "other"}
 PHASE = {0: "draft", 1: "verify", 2: "commit"}
@@ -37,7 +37,9 @@ class Config(ctypes.Structure):
                 ("dtype", ctypes.c_int), ("rms_eps", ctypes.c_float), ("rope_theta", ctypes.c_float),
                 ("n_draft_heads", ctypes.c_int), ("tree_nodes", ctypes.c_int),
                 ("topk", ctypes.c_int * 8), ("max_batch", ctypes.c_int), ("max_seq_len", ctypes.c_int),
-                ("kv_block", ctypes.c_int), ("precision", ctypes.c_int)]
+                ("kv_block", ctypes.c_int), ("precision", ctypes.c_int), ("draft_mode", ctypes.c_int),
+                ("accept_mode", ctypes.c_int), ("typical_eps", ctypes.c_float), ("typical_delta", ctypes.c_float),
+                ("trigram_cache", ctypes.c_int)]
 
 
 class BlockWeights(ctypes.Structure):
@@ -132,6 +134,11 @@ def make_config(cfg: dict, max_batch: int | None = None, max_seq_len: int | None
     c.max_seq_len = max_seq_len or cfg.get("max_seq_len", 4096)
     c.kv_block = 16
     c.precision = cfg.get("precision", 1) if precision is None else precision
+    c.draft_mode = cfg.get("draft_mode", 0)
+    c.accept_mode = cfg.get("accept_mode", 0)
+    c.typical_eps = cfg.get("typical_eps", 0.09)
+    c.typical_delta = cfg.get("typical_delta", 0.3)
+    c.trigram_cache = cfg.get("trigram_cache", 0)
     return c
 
 
@@ -284,7 +291,8 @@ class Chimera:
                       draft_logits=((K, B, V), torch.float32), topk=((B, K, kmax), torch.int32),
                       hfull=((K, B, d), torch.float32), n=((B,), torch.int32),
                       tokens=((B, self.c.max_seq_len + 1), torch.int32),
-                      prefill_logits=((B, V), torch.float32))
+                      prefill_logits=((B, V), torch.float32), trigram_hits=((K, B), torch.int32),
+                      htri=((K, B, d), torch.float32))
         shape, dt = shapes[what]
         t = torch.empty(shape, dtype=dt)
         self._check(self.lib.chimera_debug_read(self.h, DBG[what], t.data_ptr(), t.numel() * t.element_size()))

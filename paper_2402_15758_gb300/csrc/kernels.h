@@ -34,6 +34,7 @@ struct TcLinearParams {
   int* counters;     // [feat_tiles * tok_tiles], all zero between launches
   int* err;          // device error word
   unsigned long long wait_ns;  // limit of every bounded wait of the launch (ns)
+  const int* skip;   // optional device flag: nonzero at run time -> the launch does nothing
   uint32_t tmem_cols;
   uint32_t acc_stride;  // TMEM column distance between the two accumulators
   // optional: [zero, zero + zero_floats) cleared by the epilogue warps after the
@@ -77,8 +78,10 @@ int noalloc_take_error(int* word);
 // ----------------------------------------------------------------------------
 // fp32 linear (SIMT, exact fp32 FMA order per output)
 // ----------------------------------------------------------------------------
+// skip (optional, device): when *skip != 0 at run time the launch does nothing (its
+// output was provided another way, e.g. by the trigram cache).
 cudaError_t f32_linear(int M, int N, int K, const float* X, int ldx, const float* W, float* Y,
-                       int ldy, int epi, cudaStream_t s);
+                       int ldy, int epi, cudaStream_t s, const int* skip = nullptr);
 
 // ----------------------------------------------------------------------------
 // attention over the paged KV cache with a per-query ancestor bitmask
@@ -186,7 +189,9 @@ cudaError_t embed(int dtype, const void* E, int d, int V, float* x, int rows, in
                   const int* tokens, const int* tok_hist, int hist_stride, const int* n,
                   const int* valid, int* err, cudaStream_t s);
 
-cudaError_t argmax_rows(const float* logits, int V, int rows, int* out, cudaStream_t s);
+// Argmax of each row (larger value first, then smaller index); with `stats` also the
+// row's max m, log sum exp(z - m) and entropy of softmax(z) in nats: stats[row][3].
+cudaError_t argmax_rows(const float* logits, int V, int rows, int* out, cudaStream_t s, float* stats = nullptr);
 // Top-k (k <= 8) of each row, larger score first, then smaller index.  Scratch:
 // ws_v / ws_i [rows][TOPK_MAX_BLOCKS][8], counters [rows] (zero between launches).
 constexpr int TOPK_MAX_BLOCKS = 64;  // V <= 64 * 2048

@@ -121,6 +121,15 @@ __device__ __forceinline__ bool bar_any(int id, int nthreads, bool pred) {
 
 
 __global__ void __launch_bounds__(THREADS, CTAS_PER_SM) tc_linear_kernel(const __grid_constant__ TcLinearParams p) {
+  if (p.skip) {
+    // the flag is written by the previous kernel: read it after the dependency wait,
+    // before any weight is requested (a skipped launch streams nothing)
+    pdl_wait();
+    if (*reinterpret_cast<const volatile int*>(p.skip)) {
+      pdl_trigger();
+      return;
+    }
+  }
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));

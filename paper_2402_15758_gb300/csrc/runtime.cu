@@ -32,6 +32,7 @@ struct Lin {
   const void* W2 = nullptr;  // optional second weight: outputs at columns N .. N+N2-1
   int N2 = 0;
   void* Y = nullptr;
+  const int* skip = nullptr;  // device flag: nonzero -> the launch does nothing
   double bytes = 0;
 };
 
@@ -154,6 +155,20 @@ struct chimera_ctx {
   const void* tri_w1 = nullptr;
   const void* tri_w2 = nullptr;
   std::vector<const void*> heads;
+
+  // variants of the method (see chimera_config)
+  int draft_mode = 0;   // bit 0: one-pass draft; bit 1: heads without the residual input
+  int accept_mode = 0;  // 0: greedy, 1: typical acceptance
+  float typ_eps = 0.f, typ_delta = 0.f;
+  // trigram cache: keys / LRU stamps / h_tri rows of tc_entries ways (4 per set)
+  int tc_entries = 0, tc_nsets = 0;
+  unsigned long long* tc_keys = nullptr;
+  int *tc_stamp = nullptr, *tc_hit = nullptr, *tc_slot = nullptr, *tc_skip = nullptr, *tc_clock = nullptr;
+  int* tc_hit_log = nullptr;     // [K][B] hits of the last step's sub-steps
+  float* tc_vals = nullptr;
+  float* htri_log = nullptr;     // [K][B][d] h_tri rows of the last step (cache on)
+  float* d_stats = nullptr;      // [B*N][3] softmax stats of the verify rows (typical acceptance)
+  int* d_parent = nullptr;
 
   Tree tree;
   std::vector<uint64_t> chain;
@@ -317,15 +332,15 @@ cudaError_t run_lin(chimera_ctx* ctx, const Lin& l) {
   Scope sc(ctx, CHIMERA_KIND_LINEAR, l.bytes);
   if (l.tc) return tc_linear_launch(l.tp, ctx->stream);
   cudaError_t e = f32_linear(l.M, l.N, l.K, static_cast<const float*>(l.X), l.ldx, static_cast<const float*>(l.W),
-                             static_cast<float*>(l.Y), l.ldy, l.epi, ctx->stream);
+                             static_cast<float*>(l.Y), l.ldy, l.epi, ctx->stream, l.skip);
   if (e != cudaSuccess || !l.W2) return e;
   return f32_linear(l.M, l.N2, l.K, static_cast<const float*>(l.X), l.ldx, static_cast<const float*>(l.W2),
-                    static_cast<float*>(l.Y) + l.N, l.ldy, l.epi, ctx->stream);
+                    static_cast<float*>(l.Y) + l.N, l.ldy, l.epi, ctx->stream, l.skip);
 }
 
 bool make_lin(chimera_ctx* ctx, Lin* l, int M, int N, int K, const void* X, const void* X_lo, int ldx,
               const void* W, void* Y, void* Y_lo, int ldy, int epi, int out_f32, const void* W2 = nullptr,
-              int N2 = 0, float* zero = nullptr, long long zero_floats = 0) {
+              int N2 = 0, float* zero = nullptr, long long zero_floats = 0, const int* skip = nullptr) {
   l->M = M;
   l->N = N;
   l->K = K;
@@ -339,6 +354,7 @@ bool make_lin(chimera_ctx* ctx, Lin* l, int M, int N, int K, const void* X, cons
   l->W2 = W2;
   l->N2 = W2 ? N2 : 0;
   l->bytes = static_cast<double>(N + l->N2) * K * ctx->esz;
+  l->skip = skip;
   l->tc = ctx->dtype == 1;
   if (!l->tc) return true;
   char msg[256];
@@ -348,6 +364,7 @@ bool make_lin(chimera_ctx* ctx, Lin* l, int M, int N, int K, const void* X, cons
     return false;
   }
   l->tp.p.wait_ns = kDefaultWaitNs;  // the timeout hook applies to the stateless entry points only
+  l->tp.p.skip = skip;
   return true;
 }
 
@@ -548,11 +565,31 @@ cudaError_t enqueue_step(chimera_ctx* ctx) {
   // ---- draft: K sequential sub-steps ----
   ctx->cur_phase = CHIMERA_PHASE_DRAFT;
   RUN(mark_phase(ctx, 0));
+  const bool one_pass = (ctx->draft_mode & 1) != 0;
   for (int k = 0; k < K; ++k) {
+    if (k > 0 && one_pass) {  // every head scores h_full_{n+1}: only the head k launch below
+      LAUNCH(CHIMERA_KIND_OTHER, 0, launch_hfull_store(ctx->dtype, ctx->dres, d, ctx->headin, ctx->headin_lo,
+                                 ctx->hfull_log + static_cast<size_t>(k) * B * d, ctx->hlog + static_cast<size_t>(k) * B * V,
+                                 V, B, s));
+      RUN(run_lin(ctx, ctx->dhead[k]));
+      LAUNCH(CHIMERA_KIND_TOPK, 0, topk_rows(ctx->hlog + static_cast<size_t>(k) * B * V, V, B, ctx->KMAX,
+                                             ctx->d_topk + k * ctx->KMAX, ctx->d_topk_val + k * ctx->KMAX, K * ctx->KMAX,
+                                             ctx->topk_ws_v, ctx->topk_ws_i, ctx->topk_cnt, s));
+      continue;
+    }
     LAUNCH(CHIMERA_KIND_EMBED, 0, launch_trigram_gather(ctx->dtype, ctx->embed, d, V, ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_topk, K,
                                 ctx->KMAX, k, ctx->tbuf, B, ctx->d_err, ctx->dres, s));
+    if (ctx->tc_entries)
+      LAUNCH(CHIMERA_KIND_OTHER, 0, launch_trigram_lookup(ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_topk, K, ctx->KMAX, k,
+                                                          B, d, ctx->tc_nsets, ctx->tc_keys, ctx->tc_stamp, ctx->tc_vals,
+                                                          ctx->dres, ctx->tc_hit, ctx->tc_slot, ctx->tc_skip,
+                                                          ctx->tc_clock, ctx->tc_hit_log, s));
     RUN(run_lin(ctx, ctx->tri1));
     RUN(run_lin(ctx, ctx->tri2));
+    if (ctx->tc_entries)
+      LAUNCH(CHIMERA_KIND_OTHER, 0, launch_trigram_insert(ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_topk, K, ctx->KMAX, k,
+                                                          B, d, ctx->tc_keys, ctx->tc_stamp, ctx->tc_vals, ctx->dres,
+                                                          ctx->tc_hit, ctx->tc_slot, ctx->tc_clock, ctx->htri_log, s));
     RUN(run_norm(ctx, ctx->dres, ctx->draft.attn_norm, B, ctx->qkv, 3 * d));
     RUN(run_lin(ctx, ctx->dqkv));
     if (attn_fuses_rope(ctx->dtype, ctx->hd)) {
@@ -590,12 +627,18 @@ cudaError_t enqueue_step(chimera_ctx* ctx) {
     RUN(enqueue_layer(ctx, l, &ctx->ver[5 * l], B * N, N, nullptr, ctx->d_depth, ctx->d_anc, ctx->att_splits_ver, kvb));
   RUN(run_final_norm(ctx, B * N, true));
   RUN(run_lin(ctx, ctx->ver_lm));
-  LAUNCH(CHIMERA_KIND_ARGMAX, 0, argmax_rows(ctx->logits, V, B * N, ctx->d_amax, s));
+  LAUNCH(CHIMERA_KIND_ARGMAX, 0, argmax_rows(ctx->logits, V, B * N, ctx->d_amax, s, ctx->d_stats));
   // ---- accept and commit ----
   ctx->cur_phase = CHIMERA_PHASE_COMMIT;
   RUN(mark_phase(ctx, 2));
-  LAUNCH(CHIMERA_KIND_ACCEPT, 0, launch_accept(ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_node_tok, ctx->d_amax, ctx->d_child_start,
-                      ctx->d_child, N, ctx->D1, ctx->d_path, ctx->d_L, ctx->d_bonus, B, s));
+  if (ctx->accept_mode == 1)
+    LAUNCH(CHIMERA_KIND_ACCEPT, 0, launch_accept_typical(ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_node_tok, ctx->d_amax,
+                                                         ctx->logits, V, ctx->d_stats, ctx->d_parent, ctx->d_depth, N,
+                                                         ctx->D1, ctx->typ_eps, ctx->typ_delta, ctx->d_path, ctx->d_L,
+                                                         ctx->d_bonus, B, s));
+  else
+    LAUNCH(CHIMERA_KIND_ACCEPT, 0, launch_accept(ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_node_tok, ctx->d_amax, ctx->d_child_start,
+                        ctx->d_child, N, ctx->D1, ctx->d_path, ctx->d_L, ctx->d_bonus, B, s));
   LAUNCH(CHIMERA_KIND_COMPACT, 0, launch_compact(ctx->kv, ctx->kv_layer_stride * static_cast<long long>(ctx->kv_esz), ctx->L, ctx->H,
                        ctx->kv_planes, static_cast<int>(ctx->hd * ctx->kv_esz), ctx->d_n, ctx->d_path, ctx->d_L,
                        ctx->D1, ctx->d_pt, ctx->max_pages, B, s));
@@ -705,10 +748,13 @@ bool build_plans(chimera_ctx* ctx, int B) {
                 f32))
     return false;
   // draft (M = B rows); the trigram input is a gather of bf16 embeddings: exact, no lo half
+  // W2 stores h_tri (partials summed in a fixed order): the same trigram always gives
+  // the same row, so a cached row equals a recomputed one bit for bit
   if (!make_lin(ctx, &ctx->tri1, B, d, 3 * d, ctx->tbuf, nullptr, 3 * d, ctx->tri_w1, ctx->ubuf, ctx->ubuf_lo, d,
-                EPI_SILU, tb))
+                EPI_SILU, tb, nullptr, 0, nullptr, 0, ctx->tc_skip))
     return false;
-  if (!make_lin(ctx, &ctx->tri2, B, d, d, ctx->ubuf, ctx->ubuf_lo, d, ctx->tri_w2, ctx->dres, nullptr, d, ACC, f32))
+  if (!make_lin(ctx, &ctx->tri2, B, d, d, ctx->ubuf, ctx->ubuf_lo, d, ctx->tri_w2, ctx->dres, nullptr, d, EPI_STORE,
+                f32, nullptr, 0, nullptr, 0, ctx->tc_skip))
     return false;
   const chimera_block_weights& w = ctx->draft;
   if (!make_lin(ctx, &ctx->dqkv, B, 3 * d, d, xn, xl, d, w.wqkv, ctx->qkv, nullptr, 3 * d, ACC, f32)) return false;
@@ -718,8 +764,13 @@ bool build_plans(chimera_ctx* ctx, int B) {
   ctx->dup = Lin();
   if (!make_lin(ctx, &ctx->ddown, B, d, F, hf, hl, F, w.w_down, ctx->dres, nullptr, d, ACC, f32)) return false;
   ctx->dhead.assign(ctx->K, Lin());
+  // residual heads read [h_LLM_n ; h_full] (2d); heads without the residual h_full alone
+  const bool no_resid = (ctx->draft_mode & 2) != 0;
+  const int hk = no_resid ? d : 2 * d;
+  const void* hx = no_resid ? eoff(ctx, ctx->headin, d) : ctx->headin;
+  const void* hx_lo = ctx->headin_lo ? (no_resid ? eoff(ctx, ctx->headin_lo, d) : ctx->headin_lo) : nullptr;
   for (int k = 0; k < ctx->K; ++k)
-    if (!make_lin(ctx, &ctx->dhead[k], B, V, 2 * d, ctx->headin, ctx->headin_lo, 2 * d, ctx->heads[k],
+    if (!make_lin(ctx, &ctx->dhead[k], B, V, hk, hx, hx_lo, 2 * d, ctx->heads[k],
                   ctx->hlog + static_cast<size_t>(k) * B * V, nullptr, V, ACC, f32))
       return false;
   ctx->att_splits_ver = att_splits(ctx, B, N, ctx->plan_keys + N);
@@ -882,6 +933,11 @@ chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
       (c.precision != 0 && c.precision != 1))
     return CHIMERA_EINVAL;
   if (c.dtype == 1 && (c.d_model % 64 != 0 || c.ffn_dim % 128 != 0)) return CHIMERA_EINVAL;
+  if (c.draft_mode < 0 || c.draft_mode > 3 || (c.accept_mode != 0 && c.accept_mode != 1)) return CHIMERA_EINVAL;
+  if (c.accept_mode == 1 && (!(c.typical_eps >= 0.f) || !(c.typical_delta >= 0.f))) return CHIMERA_EINVAL;
+  if (c.trigram_cache < 0 || c.trigram_cache > 65536 ||
+      (c.trigram_cache && (c.trigram_cache % 4 || ((c.trigram_cache / 4) & (c.trigram_cache / 4 - 1)))))
+    return CHIMERA_EINVAL;
   // row kernels read 16-byte vectors; the top-k covers at most 64 slices of 2048 scores
   if ((c.d_model & 3) || (c.ffn_dim & 3) || (c.vocab & 3) || c.vocab > TOPK_MAX_BLOCKS * 2048) return CHIMERA_EINVAL;
   for (int k = 0; k < c.n_draft_heads; ++k)
@@ -920,6 +976,12 @@ chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
     return CHIMERA_EINVAL;
   }
   ctx->D1 = ctx->tree.depth_max + 1;
+  ctx->draft_mode = c.draft_mode;
+  ctx->accept_mode = c.accept_mode;
+  ctx->typ_eps = c.typical_eps;
+  ctx->typ_delta = c.typical_delta;
+  ctx->tc_entries = c.trigram_cache;
+  ctx->tc_nsets = c.trigram_cache / 4;
   ctx->embed = w->embed;
   ctx->layers.assign(w->layers, w->layers + c.n_layers);
   ctx->draft = w->draft;
@@ -1009,6 +1071,19 @@ chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
   ok = ok && dalloc(ctx, &ctx->d_child_start, N + 1);
   ok = ok && dalloc(ctx, &ctx->d_child, ctx->tree.child.size());
   ok = ok && dalloc(ctx, &ctx->d_one, B);
+  ok = ok && dalloc(ctx, &ctx->d_parent, N);
+  if (ctx->accept_mode == 1) ok = ok && dalloc(ctx, &ctx->d_stats, static_cast<size_t>(B) * N * 3);
+  if (ctx->tc_entries) {
+    ok = ok && dalloc(ctx, &ctx->tc_keys, ctx->tc_entries);
+    ok = ok && dalloc(ctx, &ctx->tc_stamp, ctx->tc_entries);
+    ok = ok && dalloc(ctx, &ctx->tc_vals, static_cast<size_t>(ctx->tc_entries) * d);
+    ok = ok && dalloc(ctx, &ctx->tc_hit, B);
+    ok = ok && dalloc(ctx, &ctx->tc_slot, B);
+    ok = ok && dalloc(ctx, &ctx->tc_skip, 1);
+    ok = ok && dalloc(ctx, &ctx->tc_clock, 1);
+    ok = ok && dalloc(ctx, &ctx->tc_hit_log, static_cast<size_t>(K) * B);
+    ok = ok && dalloc(ctx, &ctx->htri_log, static_cast<size_t>(K) * B * d);
+  }
   ok = ok && dalloc(ctx, &ctx->d_child_start1, 2);
   ok = ok && dalloc(ctx, &ctx->d_child1, 1);
   if (ctx->dtype == 1) {
@@ -1073,6 +1148,13 @@ chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
   zok = zok && cudaMemcpyAsync(ctx->d_one, ones.data(), B * sizeof(int), cudaMemcpyHostToDevice, s) == cudaSuccess;
   zok = zok && cudaMemsetAsync(ctx->d_child_start1, 0, 2 * sizeof(int), s) == cudaSuccess;
   zok = zok && cudaMemsetAsync(ctx->d_child1, 0, sizeof(int), s) == cudaSuccess;
+  zok = zok && cudaMemcpyAsync(ctx->d_parent, t.parent.data(), N * sizeof(int), cudaMemcpyHostToDevice, s) == cudaSuccess;
+  if (ctx->tc_entries) {
+    zok = zok && cudaMemsetAsync(ctx->tc_keys, 0, ctx->tc_entries * sizeof(unsigned long long), s) == cudaSuccess;
+    zok = zok && cudaMemsetAsync(ctx->tc_stamp, 0, ctx->tc_entries * sizeof(int), s) == cudaSuccess;
+    zok = zok && cudaMemsetAsync(ctx->tc_clock, 0, sizeof(int), s) == cudaSuccess;
+    zok = zok && cudaMemsetAsync(ctx->tc_hit_log, 0, static_cast<size_t>(K) * B * sizeof(int), s) == cudaSuccess;
+  }
   zok = zok && cudaStreamSynchronize(s) == cudaSuccess;
   if (!zok) {
     free_ctx(ctx);
@@ -1448,8 +1530,11 @@ chimera_status chimera_debug_read(chimera_ctx* ctx, int what, void* dst, size_t 
     case CHIMERA_DBG_N: src = ctx->d_n; need = B * 4; break;
     case CHIMERA_DBG_TOKENS: src = ctx->d_tok; need = B * ctx->tok_stride * 4; break;
     case CHIMERA_DBG_PREFILL_LOGITS: src = ctx->logits; need = B * V * 4; break;
+    case CHIMERA_DBG_TRIGRAM_HITS: src = ctx->tc_hit_log; need = K * B * 4; break;
+    case CHIMERA_DBG_HTRI: src = ctx->htri_log; need = K * B * d * 4; break;
     default: return fail(ctx, CHIMERA_EINVAL, "unknown debug buffer");
   }
+  if (!src) return fail(ctx, CHIMERA_EINVAL, "debug buffer not kept in this configuration");
   if (bytes != need)
     return fail(ctx, CHIMERA_EINVAL, "debug read: expected " + std::to_string(need) + " bytes, got " + std::to_string(bytes));
   CK(cudaStreamSynchronize(ctx->stream));

@@ -220,7 +220,7 @@ __device__ __forceinline__ bool better(float v, int i, float bv, int bi) {
   return v > bv || (v == bv && i < bi);
 }
 
-__global__ void __launch_bounds__(512) argmax_kernel(const float* logits, int V, int* out) {
+__global__ void __launch_bounds__(512) argmax_kernel(const float* logits, int V, int* out, float* stats) {
   pdl_trigger();  // the next kernel may start its prologue
   pdl_wait();     // inputs of this kernel are complete
   __shared__ float sv[32];
@@ -276,7 +276,50 @@ __global__ void __launch_bounds__(512) argmax_kernel(const float* logits, int V,
         bi = oi;
       }
     }
-    if (lane == 0) out[blockIdx.x] = bi < V ? bi : 0;
+    if (lane == 0) {
+      out[blockIdx.x] = bi < V ? bi : 0;
+      sv[0] = bv;
+    }
+  }
+  if (!stats) return;
+  // softmax statistics of the row at temperature 1: with e_i = exp(z_i - m),
+  // S = sum e_i, A = sum e_i (z_i - m): log S and the entropy H = log S - A / S
+  __syncthreads();
+  const float m = sv[0];
+  float S = 0.f, A = 0.f;
+  for (int i4 = threadIdx.x; i4 < V4; i4 += blockDim.x) {
+    const float4 v = *reinterpret_cast<const float4*>(z + 4 * i4);
+    const float a = v.x - m, b = v.y - m, c = v.z - m, d = v.w - m;
+    const float ea = expf(a), eb = expf(b), ec = expf(c), ed = expf(d);
+    S += (ea + eb) + (ec + ed);
+    A += (ea * a + eb * b) + (ec * c + ed * d);
+  }
+  for (int i = 4 * V4 + threadIdx.x; i < V; i += blockDim.x) {
+    const float a = z[i] - m, ea = expf(a);
+    S += ea;
+    A += ea * a;
+  }
+  __shared__ float red[2][33];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    S += __shfl_xor_sync(0xffffffffu, S, o);
+    A += __shfl_xor_sync(0xffffffffu, A, o);
+  }
+  if (lane == 0) {
+    red[0][warp] = S;
+    red[1][warp] = A;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float s2 = 0.f, a2 = 0.f;
+    for (int w = 0; w < static_cast<int>(blockDim.x >> 5); ++w) {
+      s2 += red[0][w];
+      a2 += red[1][w];
+    }
+    const float lse = logf(s2);
+    stats[3 * blockIdx.x] = m;
+    stats[3 * blockIdx.x + 1] = lse;
+    stats[3 * blockIdx.x + 2] = lse - a2 / s2;
   }
 }
 
@@ -486,10 +529,10 @@ cudaError_t embed(int dtype, const void* E, int d, int V, float* x, int rows, in
   return cudaGetLastError();
 }
 
-cudaError_t argmax_rows(const float* logits, int V, int rows, int* out, cudaStream_t s) {
+cudaError_t argmax_rows(const float* logits, int V, int rows, int* out, cudaStream_t s, float* stats) {
   if (rows <= 0) return cudaSuccess;
   if (V & 3) return cudaErrorInvalidValue;  // rows are read as float4
-  launch_pdl(argmax_kernel, dim3(rows), dim3(512), 0, s, logits, V, out);
+  launch_pdl(argmax_kernel, dim3(rows), dim3(512), 0, s, logits, V, out, stats);
   return cudaGetLastError();
 }
 

@@ -207,6 +207,158 @@ __global__ void set_root_kernel(const int* n_arr, int* tok, int tok_stride, cons
   if (b < B) tok[static_cast<size_t>(b) * tok_stride + n_arr[b]] = amax[b];
 }
 
+// ---------------------------------------------------------------------------
+// Trigram cache (the lookup table of the trigram encoder's outputs): a 4-way set-
+// associative table of h_tri rows keyed by the three token ids, least recently used
+// way replaced.  Key = (x_{i-2}+1) << 42 | (x_{i-1}+1) << 21 | x_i (a missing leading
+// token is -1, so its field is 0); 0 marks an empty way.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ int trigram_id(const int* tok, int tok_stride, const int* topk, int K, int KMAX, int b,
+                                          int n, int i) {
+  if (i < 0) return -1;
+  return i <= n ? tok[static_cast<size_t>(b) * tok_stride + i] : topk[(b * K + (i - n - 1)) * KMAX];
+}
+
+__device__ __forceinline__ unsigned long long trigram_key(int a, int b, int c) {
+  return (static_cast<unsigned long long>(a + 1) << 42) | (static_cast<unsigned long long>(b + 1) << 21) |
+         static_cast<unsigned long long>(c);
+}
+
+// One block for the batch.  For sequence b: the trigram of sub-step k; on a hit its
+// row is copied into dres[b] (the h_tri the encoder would produce) and its stamp
+// refreshed; on a miss the way to replace is recorded.  skip = every sequence hit
+// (the encoder's two linears then do nothing).
+__global__ void trigram_lookup_kernel(const int* n_arr, const int* tok, int tok_stride, const int* topk, int K,
+                                      int KMAX, int k, int B, int d, int nsets,
+                                      const unsigned long long* keys, int* stamp, const float* vals,
+                                      float* dres, int* hit, int* slot, int* skip, int* clock, int* hit_log) {
+  pdl_trigger();  // the next kernel may start its prologue
+  pdl_wait();     // inputs of this kernel are complete
+  __shared__ int s_all;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+  if (threadIdx.x == 0) s_all = 1;
+  __syncthreads();
+  const int now = *clock;
+  for (int b = warp; b < B; b += nw) {
+    const int n = n_arr[b];
+    const int x0 = trigram_id(tok, tok_stride, topk, K, KMAX, b, n, n - 2 + k);
+    const int x1 = trigram_id(tok, tok_stride, topk, K, KMAX, b, n, n - 1 + k);
+    const int x2 = trigram_id(tok, tok_stride, topk, K, KMAX, b, n, n + k);
+    const unsigned long long key = trigram_key(x0, x1, x2);
+    const int set = static_cast<int>((key * 0x9E3779B97F4A7C15ull) >> 40) & (nsets - 1);
+    int found = -1, victim = 0, oldest = 0x7fffffff;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+      const int e = set * 4 + w;
+      const unsigned long long kk = keys[e];
+      if (kk == key && found < 0) found = e;
+      const int age = kk == 0ull ? -1 : stamp[e];  // an empty way is replaced first
+      if (age < oldest) {
+        oldest = age;
+        victim = e;
+      }
+    }
+    if (found >= 0) {
+      const float4* src = reinterpret_cast<const float4*>(vals + static_cast<size_t>(found) * d);
+      float4* dst = reinterpret_cast<float4*>(dres + static_cast<size_t>(b) * d);
+      for (int c = lane; c < d / 4; c += 32) dst[c] = src[c];
+    }
+    if (lane == 0) {
+      hit[b] = found >= 0 ? 1 : 0;
+      slot[b] = found >= 0 ? found : victim;
+      if (found >= 0) stamp[found] = now;
+      else s_all = 0;
+      if (hit_log) hit_log[k * B + b] = found >= 0 ? 1 : 0;
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    *skip = s_all;
+    *clock = now + 1;
+  }
+}
+
+// After the encoder ran: store each missed sequence's h_tri row (dres[b]) in the way
+// chosen by the lookup.  Sequences are taken in order, so two of them that picked the
+// same way leave one consistent entry.  Also logs every h_tri row of the sub-step.
+__global__ void trigram_insert_kernel(const int* n_arr, const int* tok, int tok_stride, const int* topk, int K,
+                                      int KMAX, int k, int B, int d, unsigned long long* keys, int* stamp,
+                                      float* vals, const float* dres, const int* hit, const int* slot,
+                                      const int* clock, float* htri_log) {
+  pdl_trigger();  // the next kernel may start its prologue
+  pdl_wait();     // inputs of this kernel are complete
+  const int now = *clock - 1;
+  for (int b = 0; b < B; ++b) {
+    const float4* src = reinterpret_cast<const float4*>(dres + static_cast<size_t>(b) * d);
+    if (htri_log) {
+      float4* lg = reinterpret_cast<float4*>(htri_log + (static_cast<size_t>(k) * B + b) * d);
+      for (int c = threadIdx.x; c < d / 4; c += blockDim.x) lg[c] = src[c];
+    }
+    if (hit[b]) continue;
+    const int e = slot[b];
+    float4* dst = reinterpret_cast<float4*>(vals + static_cast<size_t>(e) * d);
+    for (int c = threadIdx.x; c < d / 4; c += blockDim.x) dst[c] = src[c];
+    if (threadIdx.x == 0) {
+      const int n = n_arr[b];
+      const int x0 = trigram_id(tok, tok_stride, topk, K, KMAX, b, n, n - 2 + k);
+      const int x1 = trigram_id(tok, tok_stride, topk, K, KMAX, b, n, n - 1 + k);
+      const int x2 = trigram_id(tok, tok_stride, topk, K, KMAX, b, n, n + k);
+      keys[e] = trigram_key(x0, x1, x2);
+      stamp[e] = now;
+    }
+    __syncthreads();
+  }
+}
+
+// Typical acceptance (Section "Verification", temperature 1): node c is acceptable
+// when its parent is and p_parent(token_c) > min(eps, delta exp(-H_parent)), p the
+// softmax of the parent's logits and H its entropy (stats from the argmax kernel:
+// max, log-sum-exp, entropy).  The path ends at the deepest acceptable node (the
+// smallest index among the deepest); the bonus is the base argmax there.  Writes the
+// path and the accepted tokens into the token history at x[n+1..n+L].
+__global__ void accept_typical_kernel(const int* n_arr, int* tok, int tok_stride, const int* node_tok,
+                                      const int* amax, const float* logits, int V, const float* stats,
+                                      const int* parent, const int* depth, int N, int D1, float eps, float delta,
+                                      int* path, int* Lacc, int* bonus) {
+  pdl_trigger();  // the next kernel may start its prologue
+  pdl_wait();     // inputs of this kernel are complete
+  const int b = blockIdx.x;
+  __shared__ int s_ok[64];
+  // thread c decides node c against its parent's distribution
+  const int c = threadIdx.x;
+  int pass = 0;
+  if (c < N) {
+    if (c == 0) {
+      pass = 1;
+    } else {
+      const int par = parent[c];
+      const size_t row = static_cast<size_t>(b) * N + par;
+      const float m = stats[3 * row], lse = stats[3 * row + 1], H = stats[3 * row + 2];
+      const int t = node_tok[b * N + c];
+      const float p = expf(logits[row * V + t] - m - lse);
+      const float thr = fminf(eps, delta * expf(-H));
+      pass = p > thr ? 1 : 0;
+    }
+    s_ok[c] = pass;
+  }
+  __syncthreads();
+  if (threadIdx.x != 0) return;
+  // parents precede children: fold the ancestors' decisions in node order
+  for (int i = 1; i < N; ++i) s_ok[i] = s_ok[i] && s_ok[parent[i]];
+  int best = 0;
+  for (int i = 1; i < N; ++i)
+    if (s_ok[i] && depth[i] > depth[best]) best = i;
+  const int L = depth[best];
+  const int n = n_arr[b];
+  for (int j = L, i = best; j >= 0; --j, i = parent[i]) {
+    path[b * D1 + j] = i;
+    if (j >= 1) tok[static_cast<size_t>(b) * tok_stride + n + j] = node_tok[b * N + i];
+  }
+  for (int j = L + 1; j < D1; ++j) path[b * D1 + j] = best;
+  Lacc[b] = L;
+  bonus[b] = amax[b * N + best];
+}
+
 }  // namespace
 
 cudaError_t launch_trigram_gather(int dtype, const void* E, int d, int V, const int* n, const int* tok,
@@ -243,6 +395,33 @@ cudaError_t launch_accept(const int* n, int* tok, int tok_stride, const int* nod
                           int* bonus, int B, cudaStream_t s) {
   launch_pdl(accept_kernel, dim3(B), dim3(32), 0, s, n, tok, tok_stride, node_tok, amax, child_start, child, N, D1, path, Lacc,
                                  bonus);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_trigram_lookup(const int* n, const int* tok, int tok_stride, const int* topk, int K, int KMAX, int k,
+                                  int B, int d, int nsets, const unsigned long long* keys, int* stamp,
+                                  const float* vals, float* dres, int* hit, int* slot, int* skip, int* clock,
+                                  int* hit_log, cudaStream_t s) {
+  launch_pdl(trigram_lookup_kernel, dim3(1), dim3(256), 0, s, n, tok, tok_stride, topk, K, KMAX, k, B, d, nsets, keys,
+             stamp, vals, dres, hit, slot, skip, clock, hit_log);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_trigram_insert(const int* n, const int* tok, int tok_stride, const int* topk, int K, int KMAX, int k,
+                                  int B, int d, unsigned long long* keys, int* stamp, float* vals, const float* dres,
+                                  const int* hit, const int* slot, const int* clock, float* htri_log, cudaStream_t s) {
+  launch_pdl(trigram_insert_kernel, dim3(1), dim3(256), 0, s, n, tok, tok_stride, topk, K, KMAX, k, B, d, keys, stamp,
+             vals, dres, hit, slot, clock, htri_log);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_accept_typical(const int* n, int* tok, int tok_stride, const int* node_tok, const int* amax,
+                                  const float* logits, int V, const float* stats, const int* parent, const int* depth,
+                                  int N, int D1, float eps, float delta, int* path, int* Lacc, int* bonus, int B,
+                                  cudaStream_t s) {
+  if (N > 64) return cudaErrorInvalidValue;
+  launch_pdl(accept_typical_kernel, dim3(B), dim3(64), 0, s, n, tok, tok_stride, node_tok, amax, logits, V, stats, parent,
+             depth, N, D1, eps, delta, path, Lacc, bonus);
   return cudaGetLastError();
 }
 

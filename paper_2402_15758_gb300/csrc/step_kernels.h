@@ -16,6 +16,20 @@ cudaError_t launch_tree_expand(const int* n, const int* tok, int tok_stride, con
 cudaError_t launch_accept(const int* n, int* tok, int tok_stride, const int* node_tok, const int* amax,
                           const int* child_start, const int* child, int N, int D1, int* path, int* Lacc,
                           int* bonus, int B, cudaStream_t s);
+// Trigram cache: look up the trigram of draft sub-step k for every sequence (hits fill
+// dres and set *skip when all hit), then store the misses after the encoder ran.
+cudaError_t launch_trigram_lookup(const int* n, const int* tok, int tok_stride, const int* topk, int K, int KMAX, int k,
+                                  int B, int d, int nsets, const unsigned long long* keys, int* stamp,
+                                  const float* vals, float* dres, int* hit, int* slot, int* skip, int* clock,
+                                  int* hit_log, cudaStream_t s);
+cudaError_t launch_trigram_insert(const int* n, const int* tok, int tok_stride, const int* topk, int K, int KMAX, int k,
+                                  int B, int d, unsigned long long* keys, int* stamp, float* vals, const float* dres,
+                                  const int* hit, const int* slot, const int* clock, float* htri_log, cudaStream_t s);
+// Typical acceptance over the verify logits (stats: per row max, log-sum-exp, entropy).
+cudaError_t launch_accept_typical(const int* n, int* tok, int tok_stride, const int* node_tok, const int* amax,
+                                  const float* logits, int V, const float* stats, const int* parent, const int* depth,
+                                  int N, int D1, float eps, float delta, int* path, int* Lacc, int* bonus, int B,
+                                  cudaStream_t s);
 cudaError_t launch_compact(void* pool, long long layer_stride_bytes, int n_layers, int H, int planes, int row_bytes,
                            const int* n, const int* path, const int* Lacc, int D1, const int* page_table,
                            int max_pages, int B, cudaStream_t s);
