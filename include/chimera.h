@@ -194,7 +194,8 @@ enum {
   CHIMERA_KIND_TREE = 9,
   CHIMERA_KIND_ACCEPT = 10,
   CHIMERA_KIND_COMPACT = 11,
-  CHIMERA_KIND_OTHER = 12
+  CHIMERA_KIND_OTHER = 12,
+  CHIMERA_KIND_CHAIN = 13  /* a persistent chain of linears and row steps (bf16 models) */
 };
 enum { CHIMERA_PHASE_DRAFT = 0, CHIMERA_PHASE_VERIFY = 1, CHIMERA_PHASE_COMMIT = 2 };
 chimera_status chimera_profile_step(chimera_ctx* ctx, int max, int32_t* kinds, int32_t* phases,

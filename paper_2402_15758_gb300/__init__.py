@@ -21,7 +21,7 @@ STATUS = {0: "OK", -1: "EINVAL", -2: "ENOMEM", -3: "ECAPACITY", -4: "ECUDA", -5:
 DBG = dict(node_tokens=1, verify_logits=2, verify_hidden=3, argmax=4, path=5, accept_len=6,
            draft_logits=7, topk=8, hfull=9, n=10, tokens=11, prefill_logits=12, trigram_hits=13, htri=14)
 KIND = {1: "linear", 2: "attention", 3: "norm", 4: "rope_kv", 5: "swiglu", 6: "embed", 7: "topk",
-        8: "argmax", 9: "tree", 10: "accept", 11: "compact", 12: "other"}
+        8: "argmax", 9: "tree", 10: "accept", 11: "compact", 12: "other", 13: "chain"}
 PHASE = {0: "draft", 1: "verify", 2: "commit"}
 
 

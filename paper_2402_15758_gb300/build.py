@@ -13,7 +13,7 @@ CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libchimera.so")
 SOURCES = ["linear_tc.cu", "linear_f32.cu", "attention.cu", "attention_tc.cu", "small_kernels.cu", "step_kernels.cu",
-           "runtime.cu", "linear_static.cu"]
+           "runtime.cu", "linear_static.cu", "chain_tc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2"]
 

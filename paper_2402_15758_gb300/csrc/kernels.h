@@ -76,6 +76,68 @@ cudaError_t tc_linear_launch(const TcLinearPlan& plan, cudaStream_t s);
 int noalloc_take_error(int* word);
 
 // ----------------------------------------------------------------------------
+// Persistent chain of bf16 linears and row steps in one launch (chain_tc.cu)
+// ----------------------------------------------------------------------------
+constexpr int CHAIN_MAX_GEMM = 4;
+constexpr int CHAIN_MAX_ROW = 4;
+constexpr int CHAIN_MAX_STEPS = 8;
+enum : int { CH_GEMM = 0, CH_NORM = 1, CH_SWIGLU = 2, CH_COPY = 3 };
+
+// One linear of a chain: Y[M][N] (fp32) += X[M][K] . W[N][K]^T (X bf16, optional lo half).
+struct ChainGemm {
+  CUtensorMap tmA, tmA2, tmB, tmB2;  // W, optional W2 (outputs N1..), X, X_lo
+  int N, K, ft_split, feat_tiles, kblocks;
+  uint32_t units;                    // feat_tiles * tok_tiles * kblocks
+  float* Y;
+  int ldy;
+};
+// One row step: CH_NORM  y = RMSNorm(X row; gains g, eps) -> Y (+ Y_lo), Y32; Z row cleared
+//               CH_SWIGLU y = SiLU(X[:, :cols]) * X[:, cols:2 cols] -> Y (+ Y_lo)
+//               CH_COPY  y = X row -> Y (+ Y_lo), Y32; Z row cleared
+struct ChainRow {
+  const float* X;
+  int ldx;
+  const void* g;
+  void* Y;
+  void* Y_lo;
+  int ldy;
+  float* Y32;
+  int ld32;
+  float* Z;
+  int ldz, zcols;
+  int rows, cols;
+  float eps;
+};
+struct ChainParams {
+  ChainGemm gemm[CHAIN_MAX_GEMM];
+  ChainRow row[CHAIN_MAX_ROW];
+  int n_steps, n_gemm, n_row;
+  int kind[CHAIN_MAX_STEPS];       // CH_*
+  int idx[CHAIN_MAX_STEPS];        // index into gemm[] or row[]
+  int wait[CHAIN_MAX_STEPS];       // step whose completion the step's input needs (-1: none)
+  int gemm_step[CHAIN_MAX_GEMM];   // step of each linear
+  int M, BN, tok_tiles, has_lo, stages;
+  int* bars;                       // [CHAIN_MAX_STEPS + 1] counters, all zero between launches
+  int* err;
+  unsigned long long wait_ns;
+  uint32_t tmem_cols, acc_stride;
+};
+struct ChainPlan {
+  ChainParams p;
+  int grid = 0;
+  size_t smem = 0;
+  double weight_bytes = 0;
+};
+// Start a plan for M token rows (has_lo: the activations are hi + lo bf16 pairs).
+int chain_plan(ChainPlan* plan, int M, int has_lo, char* msg, size_t msg_len);
+// Append a linear / a row step that waits for step `wait` (-1: none); returns the new
+// step's index, or -1 with a message.
+int chain_add_gemm(ChainPlan* plan, int wait, const void* X, const void* X_lo, int ldx, int K, const void* W, int N,
+                   const void* W2, int N2, float* Y, int ldy, char* msg, size_t msg_len);
+int chain_add_row(ChainPlan* plan, int kind, int wait, const ChainRow& row, char* msg, size_t msg_len);
+cudaError_t chain_launch(const ChainPlan& plan, cudaStream_t s);
+
+// ----------------------------------------------------------------------------
 // fp32 linear (SIMT, exact fp32 FMA order per output)
 // ----------------------------------------------------------------------------
 // skip (optional, device): when *skip != 0 at run time the launch does nothing (its

@@ -4,6 +4,7 @@
 #include <algorithm>
 #include <cmath>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <functional>
 #include <mutex>
@@ -22,6 +23,8 @@ namespace {
 constexpr int CHUNK = 64;        // prefill rows per sequence per pass (one 64-bit mask)
 constexpr int LOG_CAP = 4096;    // per-step accepted-count log
 constexpr int MAX_KMAX = 8;
+constexpr int CHAIN_BAR_INTS = 16;     // >= CHAIN_MAX_STEPS + 1 counters per chain launch
+constexpr int CHAIN_BAR_BLOCKS = 256;  // chain launches with their own counters
 
 struct Lin {
   bool tc = false;
@@ -229,6 +232,13 @@ struct chimera_ctx {
   std::vector<Lin> ver, pre, ar;  // 5 per layer: qkv, wo, gate, up, down
   Lin ver_lm, pre_lm, ar_lm, pre_dkv, tri1, tri2, dqkv, dwo, dgate, dup, ddown, commit_kv;
   std::vector<Lin> dhead;
+  // persistent chains (bf16 models): the linears and row steps between two attentions
+  // in one launch each (chain_tc.cu)
+  bool use_chain = false;
+  std::vector<ChainPlan> ver_chain, ar_chain, draft_chain_a, draft_chain_b;
+  ChainPlan commit_chain;
+  int* chain_bars = nullptr;  // [CHAIN_BAR_BLOCKS][CHAIN_BAR_INTS] step counters, zero between launches
+  int chain_bar_next = 0;
   int att_splits_ver = 1, att_splits_pre = 1, att_splits_draft = 1, att_splits_ar = 1;
   int plan_keys = 0;  // longest prompt of the batch (sizes the attention splits)
   cudaGraphExec_t graph = nullptr;
@@ -396,8 +406,9 @@ cudaError_t run_attention(chimera_ctx* ctx, bool draft_pool, int layer, int nq, 
                           int nq_max, double bytes, const float* qkv = nullptr, int pos_base = 0,
                           const int* pos_off = nullptr) {
   if (filtered(ctx, CHIMERA_KIND_ATTENTION)) return cudaSuccess;
-  if (qkv && !ctx->filter_kind && !(ctx->dtype == 1 && ctx->last_kind == CHIMERA_KIND_LINEAR)) {
-    ctx->err = "attention with early KV reads must directly follow a tensor-core linear";
+  if (qkv && !ctx->filter_kind &&
+      !(ctx->dtype == 1 && (ctx->last_kind == CHIMERA_KIND_LINEAR || ctx->last_kind == CHIMERA_KIND_CHAIN))) {
+    ctx->err = "attention with early KV reads must directly follow a tensor-core linear or chain";
     return cudaErrorInvalidValue;
   }
   Scope sc(ctx, CHIMERA_KIND_ATTENTION, bytes);
@@ -522,6 +533,27 @@ char* eoff(const chimera_ctx* ctx, void* base, size_t elems) {
   return static_cast<char*>(base) + elems * ctx->esz;
 }
 
+cudaError_t run_chain(chimera_ctx* ctx, const ChainPlan& c) {
+  if (filtered(ctx, CHIMERA_KIND_CHAIN)) return cudaSuccess;
+  Scope sc(ctx, CHIMERA_KIND_CHAIN, c.weight_bytes);
+  return chain_launch(c, ctx->stream);
+}
+
+// The base layers as chains: chain 0 (RMSNorm + QKV of layer 0), then per layer its
+// tree attention and the chain to the next attention (O .. down, the next layer's
+// RMSNorm and QKV; after the last layer the final norm and the LM head).
+cudaError_t enqueue_layers_chain(chimera_ctx* ctx, const std::vector<ChainPlan>& ch, int rows_per_seq,
+                                 const int* valid, const int* pos_off, const unsigned long long* anc, int splits,
+                                 double kv_bytes) {
+  RUN(run_chain(ctx, ch[0]));
+  for (int l = 0; l < ctx->L; ++l) {
+    RUN(run_attention(ctx, false, l, rows_per_seq, valid, 0, rows_per_seq, valid, anc, rows_per_seq, splits,
+                      rows_per_seq, kv_bytes, ctx->qkv, 0, pos_off));
+    RUN(run_chain(ctx, ch[l + 1]));
+  }
+  return cudaSuccess;
+}
+
 // One Llama layer over the rows of `plan` (5 linears), shared by verify and prefill.
 cudaError_t enqueue_layer(chimera_ctx* ctx, int l, const Lin* lin, int rows, int rows_per_seq, const int* valid,
                           const int* pos_off, const unsigned long long* anc, int splits, double kv_bytes) {
@@ -567,6 +599,13 @@ cudaError_t enqueue_step(chimera_ctx* ctx) {
   RUN(mark_phase(ctx, 0));
   const bool one_pass = (ctx->draft_mode & 1) != 0;
   for (int k = 0; k < K; ++k) {
+    if (k > 0 && one_pass && ctx->use_chain) {  // every head scores h_full_{n+1}
+      RUN(run_chain(ctx, ctx->draft_chain_b[k]));
+      LAUNCH(CHIMERA_KIND_TOPK, 0, topk_rows(ctx->hlog + static_cast<size_t>(k) * B * V, V, B, ctx->KMAX,
+                                             ctx->d_topk + k * ctx->KMAX, ctx->d_topk_val + k * ctx->KMAX, K * ctx->KMAX,
+                                             ctx->topk_ws_v, ctx->topk_ws_i, ctx->topk_cnt, s));
+      continue;
+    }
     if (k > 0 && one_pass) {  // every head scores h_full_{n+1}: only the head k launch below
       LAUNCH(CHIMERA_KIND_OTHER, 0, launch_hfull_store(ctx->dtype, ctx->dres, d, ctx->headin, ctx->headin_lo,
                                  ctx->hfull_log + static_cast<size_t>(k) * B * d, ctx->hlog + static_cast<size_t>(k) * B * V,
@@ -590,6 +629,16 @@ cudaError_t enqueue_step(chimera_ctx* ctx) {
       LAUNCH(CHIMERA_KIND_OTHER, 0, launch_trigram_insert(ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_topk, K, ctx->KMAX, k,
                                                           B, d, ctx->tc_keys, ctx->tc_stamp, ctx->tc_vals, ctx->dres,
                                                           ctx->tc_hit, ctx->tc_slot, ctx->tc_clock, ctx->htri_log, s));
+    if (ctx->use_chain) {
+      RUN(run_chain(ctx, ctx->draft_chain_a[k]));
+      RUN(run_attention(ctx, true, 0, 1, nullptr, k, k + 1, nullptr, ctx->d_chain, 1, ctx->att_splits_draft, 1,
+                        kv_read_bytes(ctx, k + 1, true), ctx->qkv, k, nullptr));
+      RUN(run_chain(ctx, ctx->draft_chain_b[k]));
+      LAUNCH(CHIMERA_KIND_TOPK, 0, topk_rows(ctx->hlog + static_cast<size_t>(k) * B * V, V, B, ctx->KMAX,
+                                             ctx->d_topk + k * ctx->KMAX, ctx->d_topk_val + k * ctx->KMAX, K * ctx->KMAX,
+                                             ctx->topk_ws_v, ctx->topk_ws_i, ctx->topk_cnt, s));
+      continue;
+    }
     RUN(run_norm(ctx, ctx->dres, ctx->draft.attn_norm, B, ctx->qkv, 3 * d));
     RUN(run_lin(ctx, ctx->dqkv));
     if (attn_fuses_rope(ctx->dtype, ctx->hd)) {
@@ -623,10 +672,15 @@ cudaError_t enqueue_step(chimera_ctx* ctx) {
   LAUNCH(CHIMERA_KIND_EMBED, 0, embed(ctx->dtype, ctx->embed, d, V, ctx->x, B * N, N, ctx->d_node_tok, nullptr, 0, nullptr, nullptr,
               ctx->d_err, s));
   const double kvb = kv_read_bytes(ctx, N, false);
-  for (int l = 0; l < ctx->L; ++l)
-    RUN(enqueue_layer(ctx, l, &ctx->ver[5 * l], B * N, N, nullptr, ctx->d_depth, ctx->d_anc, ctx->att_splits_ver, kvb));
-  RUN(run_final_norm(ctx, B * N, true));
-  RUN(run_lin(ctx, ctx->ver_lm));
+  if (ctx->use_chain) {
+    RUN(enqueue_layers_chain(ctx, ctx->ver_chain, N, nullptr, ctx->d_depth, ctx->d_anc, ctx->att_splits_ver, kvb));
+  } else {
+    for (int l = 0; l < ctx->L; ++l)
+      RUN(enqueue_layer(ctx, l, &ctx->ver[5 * l], B * N, N, nullptr, ctx->d_depth, ctx->d_anc, ctx->att_splits_ver,
+                        kvb));
+    RUN(run_final_norm(ctx, B * N, true));
+    RUN(run_lin(ctx, ctx->ver_lm));
+  }
   LAUNCH(CHIMERA_KIND_ARGMAX, 0, argmax_rows(ctx->logits, V, B * N, ctx->d_amax, s, ctx->d_stats));
   // ---- accept and commit ----
   ctx->cur_phase = CHIMERA_PHASE_COMMIT;
@@ -644,8 +698,12 @@ cudaError_t enqueue_step(chimera_ctx* ctx) {
                        ctx->D1, ctx->d_pt, ctx->max_pages, B, s));
   LAUNCH(CHIMERA_KIND_OTHER, 0, launch_gather_hidden(ctx->dtype, ctx->hfin32, d, N, ctx->d_path, ctx->d_L, ctx->D1, ctx->hsel, ctx->headin,
                              ctx->headin_lo, B, s));
-  RUN(run_norm(ctx, ctx->hsel, ctx->draft.attn_norm, B * ctx->D1, ctx->kvtmp, 2 * d));
-  RUN(run_lin(ctx, ctx->commit_kv));
+  if (ctx->use_chain) {
+    RUN(run_chain(ctx, ctx->commit_chain));
+  } else {
+    RUN(run_norm(ctx, ctx->hsel, ctx->draft.attn_norm, B * ctx->D1, ctx->kvtmp, 2 * d));
+    RUN(run_lin(ctx, ctx->commit_kv));
+  }
   RUN(run_rope(ctx, true, 0, ctx->kvtmp, 2 * d, -1, 0, d, ctx->D1, ctx->d_L, 1, 0, 0, nullptr));
   LAUNCH(CHIMERA_KIND_OTHER, 0, launch_finalize(ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_L, ctx->d_bonus, ctx->d_count_log, LOG_CAP,
                         ctx->d_step, B, s));
@@ -665,10 +723,14 @@ cudaError_t enqueue_ar_step(chimera_ctx* ctx) {
   LAUNCH(CHIMERA_KIND_EMBED, 0, embed(ctx->dtype, ctx->embed, d, V, ctx->x, B, 1, nullptr, ctx->d_tok, ctx->tok_stride,
                                       ctx->d_n, ctx->d_one, ctx->d_err, s));
   const double kvb = kv_read_bytes(ctx, 1, false);
-  for (int l = 0; l < ctx->L; ++l)
-    RUN(enqueue_layer(ctx, l, &ctx->ar[5 * l], B, 1, nullptr, nullptr, ctx->d_chain, ctx->att_splits_ar, kvb));
-  RUN(run_final_norm(ctx, B, true));
-  RUN(run_lin(ctx, ctx->ar_lm));
+  if (ctx->use_chain) {
+    RUN(enqueue_layers_chain(ctx, ctx->ar_chain, 1, nullptr, nullptr, ctx->d_chain, ctx->att_splits_ar, kvb));
+  } else {
+    for (int l = 0; l < ctx->L; ++l)
+      RUN(enqueue_layer(ctx, l, &ctx->ar[5 * l], B, 1, nullptr, nullptr, ctx->d_chain, ctx->att_splits_ar, kvb));
+    RUN(run_final_norm(ctx, B, true));
+    RUN(run_lin(ctx, ctx->ar_lm));
+  }
   LAUNCH(CHIMERA_KIND_ARGMAX, 0, argmax_rows(ctx->logits, V, B, ctx->d_amax, s));
   ctx->cur_phase = CHIMERA_PHASE_COMMIT;
   // a tree of the root alone: the path is [root], the bonus is its argmax
@@ -677,8 +739,12 @@ cudaError_t enqueue_ar_step(chimera_ctx* ctx) {
                                                ctx->d_bonus, B, s));
   LAUNCH(CHIMERA_KIND_OTHER, 0, launch_gather_hidden(ctx->dtype, ctx->hfin32, d, 1, ctx->d_path, ctx->d_L, ctx->D1,
                                                      ctx->hsel, ctx->headin, ctx->headin_lo, B, s));
-  RUN(run_norm(ctx, ctx->hsel, ctx->draft.attn_norm, B * ctx->D1, ctx->kvtmp, 2 * d));
-  RUN(run_lin(ctx, ctx->commit_kv));
+  if (ctx->use_chain) {
+    RUN(run_chain(ctx, ctx->commit_chain));
+  } else {
+    RUN(run_norm(ctx, ctx->hsel, ctx->draft.attn_norm, B * ctx->D1, ctx->kvtmp, 2 * d));
+    RUN(run_lin(ctx, ctx->commit_kv));
+  }
   RUN(run_rope(ctx, true, 0, ctx->kvtmp, 2 * d, -1, 0, d, ctx->D1, ctx->d_L, 1, 0, 0, nullptr));
   LAUNCH(CHIMERA_KIND_OTHER, 0, launch_finalize(ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_L, ctx->d_bonus,
                                                 ctx->d_count_log, LOG_CAP, ctx->d_step, B, s));
@@ -696,6 +762,163 @@ cudaError_t capture_step(chimera_ctx* ctx, cudaGraphExec_t* out, bool ar = false
   if (e == cudaSuccess) e = cudaGraphInstantiate(out, g, 0);
   if (g) cudaGraphDestroy(g);
   return e;
+}
+
+// ---------------------------------------------------------------------------
+// chain plans (bf16 models)
+// ---------------------------------------------------------------------------
+struct ChainBuilder {
+  chimera_ctx* ctx;
+  ChainPlan* c;
+  bool ok = true;
+  char msg[256] = {0};
+  ChainBuilder(chimera_ctx* x, ChainPlan* plan, int M) : ctx(x), c(plan) {
+    if (chain_plan(c, M, ctx->split, msg, sizeof(msg)) != 0 || ctx->chain_bar_next >= CHAIN_BAR_BLOCKS) {
+      fail_msg(msg[0] ? msg : "too many chain launches");
+      return;
+    }
+    c->p.err = ctx->d_err;
+    c->p.bars = ctx->chain_bars + static_cast<size_t>(ctx->chain_bar_next++) * CHAIN_BAR_INTS;
+  }
+  void fail_msg(const char* m) {
+    if (ok) ctx->err = m;
+    ok = false;
+  }
+  int gemm(int wait, const void* X, const void* X_lo, int ldx, int K, const void* W, int N, float* Y, int ldy,
+           const void* W2 = nullptr, int N2 = 0) {
+    if (!ok) return -1;
+    const int st = chain_add_gemm(c, wait, X, X_lo, ldx, K, W, N, W2, N2, Y, ldy, msg, sizeof(msg));
+    if (st < 0) fail_msg(msg);
+    return st;
+  }
+  int row(int kind, int wait, const ChainRow& r) {
+    if (!ok) return -1;
+    const int st = chain_add_row(c, kind, wait, r, msg, sizeof(msg));
+    if (st < 0) fail_msg(msg);
+    return st;
+  }
+};
+
+ChainRow norm_row(const chimera_ctx* ctx, const float* X, const void* g, void* Y, void* Y_lo, float* Z, int zcols,
+                  int rows, float* Y32 = nullptr) {
+  ChainRow r{};
+  r.X = X;
+  r.ldx = ctx->d;
+  r.g = g;
+  r.Y = Y;
+  r.Y_lo = Y_lo;
+  r.ldy = ctx->d;
+  r.Y32 = Y32;
+  r.ld32 = ctx->d;
+  r.Z = Z;
+  r.ldz = zcols;
+  r.zcols = Z ? zcols : 0;
+  r.rows = rows;
+  r.cols = ctx->d;
+  r.eps = ctx->cfg.rms_eps;
+  return r;
+}
+
+ChainRow swiglu_row(const chimera_ctx* ctx, int rows) {
+  ChainRow r{};
+  r.X = ctx->gu;
+  r.ldx = 2 * ctx->F;
+  r.Y = ctx->hf;
+  r.Y_lo = ctx->hf_lo;
+  r.ldy = ctx->F;
+  r.rows = rows;
+  r.cols = ctx->F;
+  return r;
+}
+
+// O projection .. down of layer l (or of the draft block `w`) appended to `b`, the
+// residual stream `x` (M rows); returns the step index of the down projection.
+int chain_ffn_half(chimera_ctx* ctx, ChainBuilder& b, const chimera_block_weights& w, float* x, int M) {
+  const int d = ctx->d, F = ctx->F;
+  const int sO = b.gemm(-1, ctx->ao, ctx->ao_lo, d, d, w.wo, d, x, d);
+  const int sN = b.row(CH_NORM, sO, norm_row(ctx, x, w.ffn_norm, ctx->xn, ctx->xn_lo, ctx->gu, 2 * F, M));
+  const int sG = b.gemm(sN, ctx->xn, ctx->xn_lo, d, d, w.w_gate, F, ctx->gu, 2 * F, w.w_up, F);
+  const int sS = b.row(CH_SWIGLU, sG, swiglu_row(ctx, M));
+  return b.gemm(sS, ctx->hf, ctx->hf_lo, F, F, w.w_down, d, x, d);
+}
+
+bool build_layer_chains(chimera_ctx* ctx, std::vector<ChainPlan>& ch, int M) {
+  const int d = ctx->d, V = ctx->V, L = ctx->L;
+  ch.assign(L + 1, ChainPlan());
+  {
+    ChainBuilder b(ctx, &ch[0], M);
+    const int sN = b.row(CH_NORM, -1, norm_row(ctx, ctx->x, ctx->layers[0].attn_norm, ctx->xn, ctx->xn_lo, ctx->qkv,
+                                               3 * d, M));
+    b.gemm(sN, ctx->xn, ctx->xn_lo, d, d, ctx->layers[0].wqkv, 3 * d, ctx->qkv, 3 * d);
+    if (!b.ok) return false;
+  }
+  for (int l = 0; l < L; ++l) {
+    ChainBuilder b(ctx, &ch[l + 1], M);
+    const int sD = chain_ffn_half(ctx, b, ctx->layers[l], ctx->x, M);
+    if (l + 1 < L) {
+      const int sN = b.row(CH_NORM, sD, norm_row(ctx, ctx->x, ctx->layers[l + 1].attn_norm, ctx->xn, ctx->xn_lo,
+                                                 ctx->qkv, 3 * d, M));
+      b.gemm(sN, ctx->xn, ctx->xn_lo, d, d, ctx->layers[l + 1].wqkv, 3 * d, ctx->qkv, 3 * d);
+    } else {  // final norm (H_LLM rows, fp32 copy) and the LM head
+      const int sF = b.row(CH_NORM, sD, norm_row(ctx, ctx->x, ctx->final_norm, ctx->hfin, ctx->hfin_lo, ctx->logits, V,
+                                                 M, ctx->hfin32));
+      b.gemm(sF, ctx->hfin, ctx->hfin_lo, d, d, ctx->lm_head, V, ctx->logits, V);
+    }
+    if (!b.ok) return false;
+  }
+  return true;
+}
+
+bool build_chains(chimera_ctx* ctx, int B) {
+  const int d = ctx->d, V = ctx->V, K = ctx->K, N = ctx->N;
+  ctx->chain_bar_next = 0;
+  if (!build_layer_chains(ctx, ctx->ver_chain, B * N)) return false;
+  if (!build_layer_chains(ctx, ctx->ar_chain, B)) return false;
+  const chimera_block_weights& w = ctx->draft;
+  const bool no_resid = (ctx->draft_mode & 2) != 0;
+  const int hk = no_resid ? d : 2 * d;
+  const void* hx = no_resid ? eoff(ctx, ctx->headin, d) : ctx->headin;
+  const void* hx_lo = ctx->headin_lo ? (no_resid ? eoff(ctx, ctx->headin_lo, d) : ctx->headin_lo) : nullptr;
+  ctx->draft_chain_a.assign(K, ChainPlan());
+  ctx->draft_chain_b.assign(K, ChainPlan());
+  for (int k = 0; k < K; ++k) {
+    const bool head_only = k > 0 && (ctx->draft_mode & 1);
+    if (!head_only) {
+      ChainBuilder a(ctx, &ctx->draft_chain_a[k], B);
+      const int sN = a.row(CH_NORM, -1, norm_row(ctx, ctx->dres, w.attn_norm, ctx->xn, ctx->xn_lo, ctx->qkv, 3 * d, B));
+      a.gemm(sN, ctx->xn, ctx->xn_lo, d, d, w.wqkv, 3 * d, ctx->qkv, 3 * d);
+      if (!a.ok) return false;
+    }
+    ChainBuilder b(ctx, &ctx->draft_chain_b[k], B);
+    const int sD = head_only ? -1 : chain_ffn_half(ctx, b, w, ctx->dres, B);
+    // h_full (the block output) into the head input [h_LLM_n ; h_full] and the per-head
+    // log; the head's score rows cleared
+    ChainRow cp{};
+    cp.X = ctx->dres;
+    cp.ldx = d;
+    cp.Y = eoff(ctx, ctx->headin, d);
+    cp.Y_lo = ctx->headin_lo ? eoff(ctx, ctx->headin_lo, d) : nullptr;
+    cp.ldy = 2 * d;
+    cp.Y32 = ctx->hfull_log + static_cast<size_t>(k) * B * d;
+    cp.ld32 = d;
+    cp.Z = ctx->hlog + static_cast<size_t>(k) * B * V;
+    cp.ldz = V;
+    cp.zcols = V;
+    cp.rows = B;
+    cp.cols = d;
+    const int sC = b.row(CH_COPY, sD, cp);
+    b.gemm(sC, hx, hx_lo, 2 * d, hk, ctx->heads[k], V, ctx->hlog + static_cast<size_t>(k) * B * V, V);
+    if (!b.ok) return false;
+  }
+  {
+    ChainBuilder c(ctx, &ctx->commit_chain, B * ctx->D1);
+    const int sN = c.row(CH_NORM, -1, norm_row(ctx, ctx->hsel, w.attn_norm, ctx->xn, ctx->xn_lo, ctx->kvtmp, 2 * d,
+                                               B * ctx->D1));
+    const void* dl_kv = eoff(ctx, const_cast<void*>(w.wqkv), static_cast<size_t>(d) * d);
+    c.gemm(sN, ctx->xn, ctx->xn_lo, d, d, dl_kv, 2 * d, ctx->kvtmp, 2 * d);
+    if (!c.ok) return false;
+  }
+  return true;
 }
 
 // (Re)build every linear call site for `batch` sequences.
@@ -777,6 +1000,7 @@ bool build_plans(chimera_ctx* ctx, int B) {
   ctx->att_splits_pre = att_splits(ctx, B, CHUNK, ctx->plan_keys);
   ctx->att_splits_draft = att_splits(ctx, B, 1, ctx->plan_keys);
   ctx->att_splits_ar = att_splits(ctx, B, 1, ctx->plan_keys + 1);
+  if (ctx->use_chain && !build_chains(ctx, B)) return false;
   return true;
 }
 
@@ -821,6 +1045,9 @@ chimera_status check_err(chimera_ctx* ctx) {
   e = ctx->h_stage[0];
   if (e == 0) return CHIMERA_OK;
   CK(cudaMemsetAsync(ctx->d_err, 0, sizeof(int), ctx->stream));
+  if ((e & ERR_TIMEOUT) && ctx->chain_bars)  // an aborted chain can leave step counters raised
+    CK(cudaMemsetAsync(ctx->chain_bars, 0, static_cast<size_t>(CHAIN_BAR_BLOCKS) * CHAIN_BAR_INTS * sizeof(int),
+                       ctx->stream));
   if (e & ERR_TIMEOUT) return fail(ctx, CHIMERA_ETIMEDOUT, "a bounded device wait timed out");
   if (e & ERR_CAPACITY) return fail(ctx, CHIMERA_ECAPACITY, "a kernel hit the KV capacity bound");
   return fail(ctx, CHIMERA_EINVAL, "a kernel saw an out-of-range token id or index");
@@ -1086,6 +1313,10 @@ chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
   }
   ok = ok && dalloc(ctx, &ctx->d_child_start1, 2);
   ok = ok && dalloc(ctx, &ctx->d_child1, 1);
+  // bf16 models run the linears between two attentions as one persistent chain launch;
+  // CHIMERA_SEPARATE_KERNELS=1 keeps one launch per linear and row kernel instead
+  ctx->use_chain = ctx->dtype == 1 && !getenv("CHIMERA_SEPARATE_KERNELS");
+  if (ctx->use_chain) ok = ok && dalloc(ctx, &ctx->chain_bars, static_cast<size_t>(CHAIN_BAR_BLOCKS) * CHAIN_BAR_INTS);
   if (ctx->dtype == 1) {
     ok = ok && dalloc(ctx, &ctx->lin_ws, tc_ws_floats(256));
     ok = ok && dalloc(ctx, &ctx->lin_cnt, static_cast<size_t>(tc_max_tiles()));
@@ -1116,6 +1347,9 @@ chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
   if (ctx->lin_cnt)
     zok = zok && cudaMemsetAsync(ctx->lin_cnt, 0, static_cast<size_t>(tc_max_tiles()) * sizeof(int), s) == cudaSuccess;
   zok = zok && cudaMemsetAsync(ctx->d_err, 0, sizeof(int), s) == cudaSuccess;
+  if (ctx->chain_bars)
+    zok = zok && cudaMemsetAsync(ctx->chain_bars, 0, static_cast<size_t>(CHAIN_BAR_BLOCKS) * CHAIN_BAR_INTS * sizeof(int),
+                                 s) == cudaSuccess;
   zok = zok && cudaMemsetAsync(ctx->d_ovr_flag, 0, sizeof(int), s) == cudaSuccess;
   zok = zok && cudaMemsetAsync(ctx->d_step, 0, sizeof(int), s) == cudaSuccess;
   zok = zok && cudaMemsetAsync(ctx->d_topk, 0, static_cast<size_t>(B) * K * ctx->KMAX * sizeof(int), s) == cudaSuccess;
@@ -1449,7 +1683,7 @@ chimera_status chimera_profile_kind(chimera_ctx* ctx, int kind, int n_reps, floa
   // committed KV rows), so the replays leave the committed state intact
   const bool allowed = kind == CHIMERA_KIND_LINEAR || kind == CHIMERA_KIND_ATTENTION || kind == CHIMERA_KIND_NORM ||
                        kind == CHIMERA_KIND_SWIGLU || kind == CHIMERA_KIND_EMBED || kind == CHIMERA_KIND_TOPK ||
-                       kind == CHIMERA_KIND_ARGMAX || kind == CHIMERA_KIND_ROPE_KV;
+                       kind == CHIMERA_KIND_ARGMAX || kind == CHIMERA_KIND_ROPE_KV || kind == CHIMERA_KIND_CHAIN;
   if (!allowed || n_reps < 1 || !ms) return fail(ctx, CHIMERA_EINVAL, "bad kernel class or repetition count");
   chimera_status st = steps_prepare(ctx, 1);
   if (st != CHIMERA_OK) return st;

@@ -55,9 +55,9 @@ def test_no_restrict_pointer_in_dependent_launch_kernels():
 def test_prewait_attention_follows_a_tensor_core_linear():
     """The tensor-core tree attention with fused RoPE (its `qkv` argument set) reads
     n_ctx, the page table and committed KV rows before its dependency wait.  That is
-    only safe when the launch directly before it is a tensor-core linear (which lets
-    its dependents launch only after its own wait).  Every such call site in the
-    runtime must therefore have a linear as its previous launch."""
+    only safe when the launch directly before it is a tensor-core linear or chain (both
+    let their dependents launch only after their own wait).  Every such call site in
+    the runtime must therefore have one of them as its previous launch."""
     import re
     src = open(os.path.join(os.path.dirname(pkg.__file__), "csrc", "runtime.cu")).read()
     lines = src.split("\n")
@@ -77,5 +77,6 @@ def test_prewait_attention_follows_a_tensor_core_linear():
         k = i - 1
         while k >= 0 and not launch.search(lines[k]):
             k -= 1
-        assert k >= 0 and "run_lin(" in lines[k], f"runtime.cu:{i + 1}: previous launch is {lines[k].strip()!r}"
+        assert k >= 0 and ("run_lin(" in lines[k] or "run_chain(" in lines[k]), \
+            f"runtime.cu:{i + 1}: previous launch is {lines[k].strip()!r}"
     assert sites >= 2  # the verify layers and the draft block
