@@ -95,6 +95,11 @@ typedef struct {
                            (d_model fp32 values) keyed by its three token ids; the least
                            recently used way of a set is replaced.  A sub-step whose trigrams
                            all hit skips the encoder's two linears; results are unchanged. */
+  int fused_chain;      /* bf16 models: 1 runs the linears and row steps between two attentions
+                           (O, RMSNorm, gate|up, SwiGLU, down, the next RMSNorm and QKV; the
+                           draft block and head; the commit projection) as one persistent
+                           launch with grid-wide step counters; 0 (default) launches each
+                           linear and row kernel separately.  Same results either way. */
 } chimera_config;
 
 /* One Llama block: RMSNorm gains [d]; wqkv [3d][d] (rows q, then k, then v; head h

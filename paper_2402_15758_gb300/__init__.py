@@ -39,7 +39,7 @@ class Config(ctypes.Structure):
                 ("topk", ctypes.c_int * 8), ("max_batch", ctypes.c_int), ("max_seq_len", ctypes.c_int),
                 ("kv_block", ctypes.c_int), ("precision", ctypes.c_int), ("draft_mode", ctypes.c_int),
                 ("accept_mode", ctypes.c_int), ("typical_eps", ctypes.c_float), ("typical_delta", ctypes.c_float),
-                ("trigram_cache", ctypes.c_int)]
+                ("trigram_cache", ctypes.c_int), ("fused_chain", ctypes.c_int)]
 
 
 class BlockWeights(ctypes.Structure):
@@ -139,6 +139,7 @@ def make_config(cfg: dict, max_batch: int | None = None, max_seq_len: int | None
     c.typical_eps = cfg.get("typical_eps", 0.09)
     c.typical_delta = cfg.get("typical_delta", 0.3)
     c.trigram_cache = cfg.get("trigram_cache", 0)
+    c.fused_chain = cfg.get("fused_chain", 0)
     return c
 
 

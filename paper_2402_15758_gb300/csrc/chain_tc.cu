@@ -27,6 +27,14 @@
 // that arrives last on the launch's final counter resets all counters to zero for the
 // next launch.  The launch lets its dependents start only after its own dependency
 // wait, so a dependent that reads before its own wait sees every earlier kernel done.
+//
+// Measured on a GB300 (7B shape, 64 tree rows): a layer-boundary chain takes ~141 us for
+// 405 MB (2.9 TB/s), against ~100 us for the same linears and row kernels launched
+// separately.  Every step waits for the slowest CTA of the previous one (a 3-6 us
+// spread at each boundary), and a row step under full HBM load costs 6-9 us including
+// its two grid-wide counter rounds; separate launches hide those tails because the next
+// kernel starts on whichever SMs free up first.  The chain is therefore an option
+// (config field fused_chain), not the default.
 #include <cstdio>
 #include <cstring>
 #include <mutex>
@@ -47,8 +55,6 @@ constexpr int MAX_STAGES = 12;
 constexpr int THREADS = 192;
 constexpr int PIPE_SMEM = 200 * 1024;
 constexpr int NORM_VEC = 16;        // float4 per epilogue thread: d <= 8192
-constexpr int SWI_VEC = 8;          // float4 pairs loaded per epilogue thread before computing
-constexpr uint32_t PF_AHEAD = 8;    // weight tiles requested into L2 beyond the ring while a step waits
 
 __device__ __forceinline__ uint32_t unit_begin(uint32_t c, uint32_t U, uint32_t G) {
   return static_cast<uint32_t>((static_cast<unsigned long long>(c) * U) / G);
@@ -58,13 +64,6 @@ __device__ __forceinline__ int ld_acquire(const int* p) {
   int v;
   asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
   return v;
-}
-
-// Request one box of a tensor into L2 (no shared-memory destination, no barrier).
-__device__ __forceinline__ void prefetch_tensor_2d(const CUtensorMap* map, int c0, int c1) {
-  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(reinterpret_cast<uint64_t>(map)),
-               "r"(c0), "r"(c1)
-               : "memory");
 }
 
 __device__ __forceinline__ void fence_proxy_async_global() {
@@ -112,12 +111,11 @@ __device__ __forceinline__ float4 gain4(const bf16* g, int i) {
   return make_float4(__bfloat162float(h[0]), __bfloat162float(h[1]), __bfloat162float(h[2]), __bfloat162float(h[3]));
 }
 
-// four consecutive values as bf16 hi (+ lo) planes, one 8-byte store per plane
 __device__ __forceinline__ void store_split4(bf16* hi, bf16* lo, size_t i, float4 v) {
-  if (lo)
-    store4_split<bf16>(hi + i, lo + i, v);
-  else
-    store4<bf16>(hi + i, v);
+  store_act(hi, lo, i, v.x);
+  store_act(hi, lo, i + 1, v.y);
+  store_act(hi, lo, i + 2, v.z);
+  store_act(hi, lo, i + 3, v.w);
 }
 
 __global__ void __launch_bounds__(THREADS, 1) chain_kernel(const __grid_constant__ ChainParams p) {
@@ -232,71 +230,45 @@ __global__ void __launch_bounds__(THREADS, 1) chain_kernel(const __grid_constant
       }
       pdl_wait();
       pdl_trigger();
-      auto x_ready = [&]() -> bool {
-        if (xg_ready == xg) return true;
-        const int w = p.wait[p.gemm_step[xg]];
-        if (w >= 0 && ld_acquire(p.bars + w) < static_cast<int>(G)) return false;
-        fence_proxy_async_global();  // the TMA reads below see what the step published
-        xg_ready = xg;
-        return true;
-      };
-      // L2 prefetch cursor: units [wq, pq) have their weight tiles requested into L2
-      uint32_t pq = wq;
-      int pg = wg;
-      uint32_t pu = wu;
       uint64_t t_last = global_timer_ns();
       while (xq < total && !*abort) {
-        if (x_ready()) {
-          if (xq < wq) {  // activation half of a unit whose weights are on their way
+        bool moved = false;
+        // activation tile of unit xq once its producing step has completed
+        if (xq < wq) {
+          bool ready = xg_ready == xg;
+          if (!ready) {
+            const int st = p.gemm_step[xg];
+            const int w = p.wait[st];
+            ready = w < 0 || ld_acquire(p.bars + w) >= static_cast<int>(G);
+            if (ready) {
+              fence_proxy_async_global();
+              xg_ready = xg;
+            }
+          }
+          if (ready) {
             issue_x(xq, xg, xu);
             ++xq;
             ++xu;
             norm_cursor(xg, xu);
-          } else {  // next unit: wait (blocking) for its ring slot, then its weights
-            const int st = static_cast<int>(wq % p.stages);
-            if (wq >= static_cast<uint32_t>(p.stages) &&
-                !mbar_wait(&empty[st], ((wq / p.stages) - 1u) & 1u, abort, p.wait_ns))
-              break;
+            moved = true;
+          }
+        }
+        // weight tile of unit wq once its ring slot is free (unit wq - stages consumed)
+        if (wq < total && wq < xq + static_cast<uint32_t>(p.stages)) {
+          const int s = static_cast<int>(wq % p.stages);
+          if (mbar_test(&empty[s], ((wq / p.stages) - 1u) & 1u)) {
             issue_w(wq, wg, wu);
             ++wq;
             ++wu;
             norm_cursor(wg, wu);
+            moved = true;
           }
+        }
+        if (moved) {
           t_last = global_timer_ns();
-          continue;
+        } else if (global_timer_ns() - t_last > p.wait_ns) {
+          *abort = 1;
         }
-        // the activation of unit xq waits for its producing step: keep HBM busy with the
-        // weights of the next units, into free ring slots, then into L2
-        if (wq < total && wq < xq + static_cast<uint32_t>(p.stages) &&
-            (wq < static_cast<uint32_t>(p.stages) || mbar_test(&empty[wq % p.stages], ((wq / p.stages) - 1u) & 1u))) {
-          issue_w(wq, wg, wu);
-          ++wq;
-          ++wu;
-          norm_cursor(wg, wu);
-          t_last = global_timer_ns();
-          continue;
-        }
-        if (pq < wq) {
-          pq = wq;
-          pg = wg;
-          pu = wu;
-        }
-        if (pq < total && pq < wq + PF_AHEAD) {
-          const ChainGemm& gm = p.gemm[pg];
-          const int t = static_cast<int>(pu / gm.kblocks), kb = static_cast<int>(pu % gm.kblocks);
-          const int ft = t / p.tok_tiles;
-          const bool second = ft >= gm.ft_split;
-          const CUtensorMap* map = second ? &gm.tmA2 : &gm.tmA;
-          const int row = (second ? ft - gm.ft_split : ft) * BM;
-#pragma unroll
-          for (int a = 0; a < BKA; ++a) prefetch_tensor_2d(map, kb * BK + a * ATOM, row);
-          ++pq;
-          ++pu;
-          norm_cursor(pg, pu);
-          continue;
-        }
-        __nanosleep(128);
-        if (global_timer_ns() - t_last > p.wait_ns) *abort = 1;
       }
       if (*abort) {
         // every started stage must land before the CTA exits: request the activation
@@ -371,16 +343,7 @@ __global__ void __launch_bounds__(THREADS, 1) chain_kernel(const __grid_constant
     int buf = 0;
     uint32_t aphase = 0;
     bool dead = false;
-    // this CTA's share of the fp32 accumulators that the chain's linears add into
-    for (int z = 0; z < CHAIN_MAX_ZERO; ++z) {
-      if (!p.zero[z]) continue;
-      const long long n4 = p.zero_n4[z];
-      float4* zp = reinterpret_cast<float4*>(p.zero[z]);
-      for (long long i = static_cast<long long>(cta) * n4 / G + et; i < static_cast<long long>(cta + 1) * n4 / G; i += 128)
-        zp[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-    }
-    // wait until step `w` has all G arrivals: one thread polls (acquire, bounded), the
-    // named barrier orders the other threads' reads after it
+    // wait until step `w` has all G arrivals (one thread polls, bounded)
     auto wait_step = [&](int w) -> bool {
       int ok = 1;
       if (w >= 0 && et == 0) {
@@ -391,19 +354,16 @@ __global__ void __launch_bounds__(THREADS, 1) chain_kernel(const __grid_constant
             ok = 0;
             break;
           }
-          __nanosleep(32);
         }
       }
-      return !bar_any(1, 128, !ok);
+      const bool bad = bar_any(1, 128, !ok);
+      __threadfence();
+      return !bad;
     };
-    // publish the step: every thread's writes precede the named barrier, then one
-    // thread's gpu-scope fence and arrival (cumulative release)
     auto signal = [&](int s) {
+      __threadfence();
       named_bar(1, 128);
-      if (et == 0) {
-        __threadfence();
-        atomicAdd(p.bars + s, 1);
-      }
+      if (et == 0) atomicAdd(p.bars + s, 1);
     };
     for (int s = 0; s < p.n_steps && !dead; ++s) {
       const int kind = p.kind[s];
@@ -481,28 +441,12 @@ __global__ void __launch_bounds__(THREADS, 1) chain_kernel(const __grid_constant
         // h = SiLU(gate) * up over this CTA's share of the rows x F/4 float4 chunks
         const long long F4 = r.cols / 4, C = static_cast<long long>(r.rows) * F4;
         const long long c0 = static_cast<long long>(cta) * C / G, c1 = static_cast<long long>(cta + 1) * C / G;
-        for (long long i0 = c0 + et; i0 < c1; i0 += 128 * SWI_VEC) {
-          float4 a[SWI_VEC], u[SWI_VEC];
-#pragma unroll
-          for (int k = 0; k < SWI_VEC; ++k) {  // every load of the batch in flight at once
-            const long long i = i0 + k * 128;
-            if (i < c1) {
-              const int row = static_cast<int>(i / F4), f = static_cast<int>(i % F4) * 4;
-              const float* gu = r.X + static_cast<size_t>(row) * r.ldx;
-              a[k] = ldcg4(gu + f);
-              u[k] = ldcg4(gu + r.cols + f);
-            }
-          }
-#pragma unroll
-          for (int k = 0; k < SWI_VEC; ++k) {
-            const long long i = i0 + k * 128;
-            if (i < c1) {
-              const int row = static_cast<int>(i / F4), f = static_cast<int>(i % F4) * 4;
-              store_split4(static_cast<bf16*>(r.Y), static_cast<bf16*>(r.Y_lo), static_cast<size_t>(row) * r.ldy + f,
-                           make_float4(silu_f(a[k].x) * u[k].x, silu_f(a[k].y) * u[k].y, silu_f(a[k].z) * u[k].z,
-                                       silu_f(a[k].w) * u[k].w));
-            }
-          }
+        for (long long i = c0 + et; i < c1; i += 128) {
+          const int row = static_cast<int>(i / F4), f = static_cast<int>(i % F4) * 4;
+          const float* gu = r.X + static_cast<size_t>(row) * r.ldx;
+          const float4 a = ldcg4(gu + f), u = ldcg4(gu + r.cols + f);
+          store_split4(static_cast<bf16*>(r.Y), static_cast<bf16*>(r.Y_lo), static_cast<size_t>(row) * r.ldy + f,
+                       make_float4(silu_f(a.x) * u.x, silu_f(a.y) * u.y, silu_f(a.z) * u.z, silu_f(a.w) * u.w));
         }
       } else {  // CH_COPY: rows of X into the bf16 operand Y (+ lo) and the fp32 copy Y32; Z rows cleared
         for (int row = static_cast<int>(cta); row < r.rows; row += static_cast<int>(G)) {
@@ -621,18 +565,6 @@ int chain_add_gemm(ChainPlan* plan, int wait, const void* X, const void* X_lo, i
   p.n_gemm++;
   plan->weight_bytes += 2.0 * (static_cast<double>(N) + (W2 ? N2 : 0)) * K;
   return s;
-}
-
-int chain_add_zero(ChainPlan* plan, float* ptr, long long floats) {
-  ChainParams& p = plan->p;
-  if (!ptr || floats < 0 || (floats & 3) || (reinterpret_cast<uintptr_t>(ptr) & 15)) return -1;
-  for (int z = 0; z < CHAIN_MAX_ZERO; ++z)
-    if (!p.zero[z]) {
-      p.zero[z] = ptr;
-      p.zero_n4[z] = floats / 4;
-      return 0;
-    }
-  return -1;
 }
 
 int chain_add_row(ChainPlan* plan, int kind, int wait, const ChainRow& row, char* msg, size_t msg_len) {

@@ -81,7 +81,6 @@ int noalloc_take_error(int* word);
 constexpr int CHAIN_MAX_GEMM = 4;
 constexpr int CHAIN_MAX_ROW = 4;
 constexpr int CHAIN_MAX_STEPS = 8;
-constexpr int CHAIN_MAX_ZERO = 2;
 enum : int { CH_GEMM = 0, CH_NORM = 1, CH_SWIGLU = 2, CH_COPY = 3 };
 
 // One linear of a chain: Y[M][N] (fp32) += X[M][K] . W[N][K]^T (X bf16, optional lo half).
@@ -118,8 +117,6 @@ struct ChainParams {
   int wait[CHAIN_MAX_STEPS];       // step whose completion the step's input needs (-1: none)
   int gemm_step[CHAIN_MAX_GEMM];   // step of each linear
   int M, BN, tok_tiles, has_lo, stages;
-  float* zero[CHAIN_MAX_ZERO];      // fp32 accumulators cleared at the start (spread over the CTAs)
-  long long zero_n4[CHAIN_MAX_ZERO];
   int* bars;                       // [CHAIN_MAX_STEPS + 1] counters, all zero between launches
   int* err;
   unsigned long long wait_ns;
@@ -138,9 +135,6 @@ int chain_plan(ChainPlan* plan, int M, int has_lo, char* msg, size_t msg_len);
 int chain_add_gemm(ChainPlan* plan, int wait, const void* X, const void* X_lo, int ldx, int K, const void* W, int N,
                    const void* W2, int N2, float* Y, int ldy, char* msg, size_t msg_len);
 int chain_add_row(ChainPlan* plan, int kind, int wait, const ChainRow& row, char* msg, size_t msg_len);
-// Clear [ptr, ptr + floats) at the start of the launch (before any step; the linears
-// that add into it wait for a later step).  0 on success.
-int chain_add_zero(ChainPlan* plan, float* ptr, long long floats);
 cudaError_t chain_launch(const ChainPlan& plan, cudaStream_t s);
 
 // ----------------------------------------------------------------------------

@@ -4,7 +4,6 @@
 #include <algorithm>
 #include <cmath>
 #include <cstdio>
-#include <cstdlib>
 #include <cstring>
 #include <functional>
 #include <mutex>
@@ -791,9 +790,6 @@ struct ChainBuilder {
     if (st < 0) fail_msg(msg);
     return st;
   }
-  void zero(float* ptr, long long floats) {
-    if (ok && chain_add_zero(c, ptr, floats) != 0) fail_msg("chain: cannot clear the accumulator");
-  }
   int row(int kind, int wait, const ChainRow& r) {
     if (!ok) return -1;
     const int st = chain_add_row(c, kind, wait, r, msg, sizeof(msg));
@@ -839,37 +835,32 @@ ChainRow swiglu_row(const chimera_ctx* ctx, int rows) {
 int chain_ffn_half(chimera_ctx* ctx, ChainBuilder& b, const chimera_block_weights& w, float* x, int M) {
   const int d = ctx->d, F = ctx->F;
   const int sO = b.gemm(-1, ctx->ao, ctx->ao_lo, d, d, w.wo, d, x, d);
-  const int sN = b.row(CH_NORM, sO, norm_row(ctx, x, w.ffn_norm, ctx->xn, ctx->xn_lo, nullptr, 0, M));
+  const int sN = b.row(CH_NORM, sO, norm_row(ctx, x, w.ffn_norm, ctx->xn, ctx->xn_lo, ctx->gu, 2 * F, M));
   const int sG = b.gemm(sN, ctx->xn, ctx->xn_lo, d, d, w.w_gate, F, ctx->gu, 2 * F, w.w_up, F);
   const int sS = b.row(CH_SWIGLU, sG, swiglu_row(ctx, M));
   return b.gemm(sS, ctx->hf, ctx->hf_lo, F, F, w.w_down, d, x, d);
 }
 
-// The accumulators a chain's linears add into are cleared at the start of the chain
-// (spread over all CTAs); the linears that add into them wait for a later step.
 bool build_layer_chains(chimera_ctx* ctx, std::vector<ChainPlan>& ch, int M) {
-  const int d = ctx->d, V = ctx->V, L = ctx->L, F = ctx->F;
+  const int d = ctx->d, V = ctx->V, L = ctx->L;
   ch.assign(L + 1, ChainPlan());
   {
     ChainBuilder b(ctx, &ch[0], M);
-    b.zero(ctx->qkv, static_cast<long long>(M) * 3 * d);
-    const int sN = b.row(CH_NORM, -1, norm_row(ctx, ctx->x, ctx->layers[0].attn_norm, ctx->xn, ctx->xn_lo, nullptr, 0, M));
+    const int sN = b.row(CH_NORM, -1, norm_row(ctx, ctx->x, ctx->layers[0].attn_norm, ctx->xn, ctx->xn_lo, ctx->qkv,
+                                               3 * d, M));
     b.gemm(sN, ctx->xn, ctx->xn_lo, d, d, ctx->layers[0].wqkv, 3 * d, ctx->qkv, 3 * d);
     if (!b.ok) return false;
   }
   for (int l = 0; l < L; ++l) {
     ChainBuilder b(ctx, &ch[l + 1], M);
-    b.zero(ctx->gu, static_cast<long long>(M) * 2 * F);
     const int sD = chain_ffn_half(ctx, b, ctx->layers[l], ctx->x, M);
     if (l + 1 < L) {
-      b.zero(ctx->qkv, static_cast<long long>(M) * 3 * d);
       const int sN = b.row(CH_NORM, sD, norm_row(ctx, ctx->x, ctx->layers[l + 1].attn_norm, ctx->xn, ctx->xn_lo,
-                                                 nullptr, 0, M));
+                                                 ctx->qkv, 3 * d, M));
       b.gemm(sN, ctx->xn, ctx->xn_lo, d, d, ctx->layers[l + 1].wqkv, 3 * d, ctx->qkv, 3 * d);
     } else {  // final norm (H_LLM rows, fp32 copy) and the LM head
-      b.zero(ctx->logits, static_cast<long long>(M) * V);
-      const int sF = b.row(CH_NORM, sD, norm_row(ctx, ctx->x, ctx->final_norm, ctx->hfin, ctx->hfin_lo, nullptr, 0, M,
-                                                 ctx->hfin32));
+      const int sF = b.row(CH_NORM, sD, norm_row(ctx, ctx->x, ctx->final_norm, ctx->hfin, ctx->hfin_lo, ctx->logits, V,
+                                                 M, ctx->hfin32));
       b.gemm(sF, ctx->hfin, ctx->hfin_lo, d, d, ctx->lm_head, V, ctx->logits, V);
     }
     if (!b.ok) return false;
@@ -891,19 +882,16 @@ bool build_chains(chimera_ctx* ctx, int B) {
   ctx->draft_chain_b.assign(K, ChainPlan());
   for (int k = 0; k < K; ++k) {
     const bool head_only = k > 0 && (ctx->draft_mode & 1);
-    float* hlog_k = ctx->hlog + static_cast<size_t>(k) * B * V;
     if (!head_only) {
       ChainBuilder a(ctx, &ctx->draft_chain_a[k], B);
-      a.zero(ctx->qkv, static_cast<long long>(B) * 3 * d);
-      const int sN = a.row(CH_NORM, -1, norm_row(ctx, ctx->dres, w.attn_norm, ctx->xn, ctx->xn_lo, nullptr, 0, B));
+      const int sN = a.row(CH_NORM, -1, norm_row(ctx, ctx->dres, w.attn_norm, ctx->xn, ctx->xn_lo, ctx->qkv, 3 * d, B));
       a.gemm(sN, ctx->xn, ctx->xn_lo, d, d, w.wqkv, 3 * d, ctx->qkv, 3 * d);
       if (!a.ok) return false;
     }
     ChainBuilder b(ctx, &ctx->draft_chain_b[k], B);
-    if (!head_only) b.zero(ctx->gu, static_cast<long long>(B) * 2 * ctx->F);
-    b.zero(hlog_k, static_cast<long long>(B) * V);
     const int sD = head_only ? -1 : chain_ffn_half(ctx, b, w, ctx->dres, B);
-    // h_full (the block output) into the head input [h_LLM_n ; h_full] and the per-head log
+    // h_full (the block output) into the head input [h_LLM_n ; h_full] and the per-head
+    // log; the head's score rows cleared
     ChainRow cp{};
     cp.X = ctx->dres;
     cp.ldx = d;
@@ -912,16 +900,18 @@ bool build_chains(chimera_ctx* ctx, int B) {
     cp.ldy = 2 * d;
     cp.Y32 = ctx->hfull_log + static_cast<size_t>(k) * B * d;
     cp.ld32 = d;
+    cp.Z = ctx->hlog + static_cast<size_t>(k) * B * V;
+    cp.ldz = V;
+    cp.zcols = V;
     cp.rows = B;
     cp.cols = d;
     const int sC = b.row(CH_COPY, sD, cp);
-    b.gemm(sC, hx, hx_lo, 2 * d, hk, ctx->heads[k], V, hlog_k, V);
+    b.gemm(sC, hx, hx_lo, 2 * d, hk, ctx->heads[k], V, ctx->hlog + static_cast<size_t>(k) * B * V, V);
     if (!b.ok) return false;
   }
   {
     ChainBuilder c(ctx, &ctx->commit_chain, B * ctx->D1);
-    c.zero(ctx->kvtmp, static_cast<long long>(B) * ctx->D1 * 2 * d);
-    const int sN = c.row(CH_NORM, -1, norm_row(ctx, ctx->hsel, w.attn_norm, ctx->xn, ctx->xn_lo, nullptr, 0,
+    const int sN = c.row(CH_NORM, -1, norm_row(ctx, ctx->hsel, w.attn_norm, ctx->xn, ctx->xn_lo, ctx->kvtmp, 2 * d,
                                                B * ctx->D1));
     const void* dl_kv = eoff(ctx, const_cast<void*>(w.wqkv), static_cast<size_t>(d) * d);
     c.gemm(sN, ctx->xn, ctx->xn_lo, d, d, dl_kv, 2 * d, ctx->kvtmp, 2 * d);
@@ -1169,7 +1159,9 @@ chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
       (c.precision != 0 && c.precision != 1))
     return CHIMERA_EINVAL;
   if (c.dtype == 1 && (c.d_model % 64 != 0 || c.ffn_dim % 128 != 0)) return CHIMERA_EINVAL;
-  if (c.draft_mode < 0 || c.draft_mode > 3 || (c.accept_mode != 0 && c.accept_mode != 1)) return CHIMERA_EINVAL;
+  if (c.draft_mode < 0 || c.draft_mode > 3 || (c.accept_mode != 0 && c.accept_mode != 1) ||
+      (c.fused_chain != 0 && c.fused_chain != 1))
+    return CHIMERA_EINVAL;
   if (c.accept_mode == 1 && (!(c.typical_eps >= 0.f) || !(c.typical_delta >= 0.f))) return CHIMERA_EINVAL;
   if (c.trigram_cache < 0 || c.trigram_cache > 65536 ||
       (c.trigram_cache && (c.trigram_cache % 4 || ((c.trigram_cache / 4) & (c.trigram_cache / 4 - 1)))))
@@ -1322,9 +1314,10 @@ chimera_status chimera_init(const chimera_config* cfg, const chimera_weights* w,
   }
   ok = ok && dalloc(ctx, &ctx->d_child_start1, 2);
   ok = ok && dalloc(ctx, &ctx->d_child1, 1);
-  // bf16 models run the linears between two attentions as one persistent chain launch;
-  // CHIMERA_SEPARATE_KERNELS=1 keeps one launch per linear and row kernel instead
-  ctx->use_chain = ctx->dtype == 1 && !getenv("CHIMERA_SEPARATE_KERNELS");
+  // bf16 models with fused_chain run the linears and row steps between two attentions
+  // as one persistent chain launch; otherwise every linear and row kernel is launched
+  // on its own (the default: faster on this GPU, see the chain kernel's notes)
+  ctx->use_chain = ctx->dtype == 1 && c.fused_chain == 1;
   if (ctx->use_chain) ok = ok && dalloc(ctx, &ctx->chain_bars, static_cast<size_t>(CHAIN_BAR_BLOCKS) * CHAIN_BAR_INTS);
   if (ctx->dtype == 1) {
     ok = ok && dalloc(ctx, &ctx->lin_ws, tc_ws_floats(256));

@@ -203,8 +203,9 @@ def _force_chain(W, cfg, st, tree, toks, L, branch=(0, 0, 0, 0)):
     return toks
 
 
-def _run_bf16(name, n_steps, forced_seq, device_gen="cpu", max_seq=None, precision=1, branch=(0, 0, 0, 0)):
+def _run_bf16(name, n_steps, forced_seq, device_gen="cpu", max_seq=None, precision=1, branch=(0, 0, 0, 0), **over):
     cfg, w_cpu, w_dev = _setup(name, device_gen)
+    cfg.update(over)
     W = co.OracleWeights(w_cpu, cache=(name != "7b"))
     prompts = synth.make_prompts(cfg)
     B, K, kmax, V, tol = len(prompts), cfg["n_draft_heads"], max(cfg["topk"]), cfg["vocab"], tol_of(cfg)
@@ -304,6 +305,14 @@ def test_mini_overlapping_compaction():
     assert max(acc) >= 3
 
 
+@pytest.mark.parametrize("name", ["mini", "mini_b4"])
+def test_bf16_steps_fused_chain(name):
+    # the persistent chain launches (fused_chain = 1) against the oracle, with forced
+    # acceptance along an off-rank-0 branch (overlapping compaction)
+    acc = _run_bf16(name, 3, [4, 1, 3], branch=(1, 0, 0, 0), fused_chain=1)
+    assert max(acc) >= 1
+
+
 def test_mini_b4_ragged_batch():
     acc = _run_bf16("mini_b4", 3, [1, 0, 4, 2])
     assert max(acc) >= 2
@@ -320,6 +329,11 @@ def _host_mem_gb():
 def test_7b_full_size_step():
     # the benchmark's workload: 7B shape, bs1, 512-token prompt, 64-node tree
     _run_bf16("7b", 1, [2], device_gen="cuda", max_seq=1024)
+
+
+@pytest.mark.skipif(_host_mem_gb() < 96, reason="the fp64 oracle of the 7B model needs >= 96 GB of host memory")
+def test_7b_full_size_step_fused_chain():
+    _run_bf16("7b", 1, [3], device_gen="cuda", max_seq=1024, fused_chain=1)
 
 
 # ----------------------------------------------------------------------------
@@ -357,9 +371,10 @@ def test_tiny_ar_and_spec_steps_mix(tiny):
     ctx.close()
 
 
-@pytest.mark.parametrize("name", ["mini", "mini_b4"])
-def test_bf16_ar_steps_match_oracle(name):
+@pytest.mark.parametrize("name,fused", [("mini", 0), ("mini_b4", 0), ("mini", 1)])
+def test_bf16_ar_steps_match_oracle(name, fused):
     cfg, w_cpu, w_dev = _setup(name)
+    cfg["fused_chain"] = fused
     W = co.OracleWeights(w_cpu)
     prompts = synth.make_prompts(cfg)
     B, tol = len(prompts), tol_of(cfg)

@@ -189,8 +189,9 @@ def test_tiny_draft_variants(mode):
     ctx.close()
 
 
-def test_mini_draft_one_pass_no_residual():
-    cfg, w_cpu, w_dev = _setup("mini", draft_mode=3)
+@pytest.mark.parametrize("fused", [0, 1])
+def test_mini_draft_one_pass_no_residual(fused):
+    cfg, w_cpu, w_dev = _setup("mini", draft_mode=3, fused_chain=fused)
     W = co.OracleWeights(w_cpu)
     prompt = synth.make_prompts(cfg)[0]
     ctx = pkg.Chimera(cfg, w_dev, max_batch=1, max_seq_len=256)
