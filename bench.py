@@ -211,7 +211,8 @@ def op_bench(args, hbm, peak_kind):
         out = torch.empty(nq, H * hd, dtype=torch.bfloat16, device=dev)
         out_lo = torch.empty_like(out)
         # as the step: one cluster of <= 8 CTAs per head, all heads resident at once
-        splits = max(1, min(8, torch.cuda.get_device_properties(0).multi_processor_count // H, -(-n_keys // 64)))
+        splits = args.splits or max(1, min(8, torch.cuda.get_device_properties(0).multi_processor_count // H,
+                                           -(-n_keys // 64)))
         nbytes = n_keys * H * hd * 4 * 2 + nq * H * hd * 4 + 2 * nq * H * hd * 2
 
         def launch(i):
@@ -286,10 +287,13 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--layers", type=int, default=None,
                     help="profiling only: the 7B shapes with fewer base layers (not the benchmark workload)")
+    ap.add_argument("--fused-chain", action="store_true",
+                    help="run the linears between two attentions as persistent chain launches (fused_chain = 1)")
     ap.add_argument("--op", choices=["linear", "attention"], default=None,
                     help="time one kernel entry point instead of the step")
     ap.add_argument("--shape", default="64,22016,4096", help="--op linear: M,N,K")
     ap.add_argument("--ctx", type=int, default=1024, help="--op attention: committed context rows")
+    ap.add_argument("--splits", type=int, default=0, help="--op attention: KV splits per head (0: as the step)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -315,6 +319,8 @@ def main():
     cfg = synth.get_config(WORKLOAD)
     if args.layers:
         cfg["n_layers"] = args.layers
+    if args.fused_chain:
+        cfg["fused_chain"] = 1
     B, N = cfg["batch"], cfg["tree_nodes"]
     prompt = synth.make_prompts(cfg)[0]
     w = synth.make_weights(cfg, device="cuda")
@@ -462,6 +468,7 @@ def main():
     }
     if args.layers:
         line["config"]["workload"] += f" [profiling run: {args.layers} base layers, not the benchmark workload]"
+    line["config"]["launch"] = "persistent chains" if args.fused_chain else "one launch per linear and row kernel"
     if rank == 0:
         print(json.dumps(line))
     if world > 1:

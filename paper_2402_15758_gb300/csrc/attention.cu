@@ -16,6 +16,8 @@
 #include <algorithm>
 #include <cmath>
 
+#include <mutex>
+
 #include "common.cuh"
 #include "launch.cuh"
 #include "kernels.h"
@@ -261,13 +263,25 @@ __global__ void __launch_bounds__(WARPS * 32) attn_kernel(const AttnParams p) {
   if (threadIdx.x == 0) p.counters[b * p.H + h] = 0;
 }
 
+constexpr int ATT_MAX_DEVICES = 64;
+std::mutex g_attr_mu;
+
 template <typename TKV, typename T, int HD>
 cudaError_t launch(const AttnParams& p, cudaStream_t s) {
   const size_t smem = (KT * (HD + 1) + KT * HD + static_cast<size_t>(p.nq_max) * HD) * sizeof(float);
-  static bool attr = false;
-  if (!attr) {
-    cudaFuncSetAttribute(attn_kernel<TKV, T, HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
-    attr = true;
+  // the shared-memory limit is a per-device attribute: raised once per device
+  static bool attr[ATT_MAX_DEVICES];
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= ATT_MAX_DEVICES) return cudaErrorInvalidDevice;
+  {
+    std::lock_guard<std::mutex> lk(g_attr_mu);
+    if (!attr[dev]) {
+      e = cudaFuncSetAttribute(attn_kernel<TKV, T, HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+      if (e != cudaSuccess) return e;
+      attr[dev] = true;
+    }
   }
   dim3 grid(p.splits, p.H, p.B);
   launch_pdl(attn_kernel<TKV, T, HD>, dim3(grid), dim3(WARPS * 32), smem, s, p);

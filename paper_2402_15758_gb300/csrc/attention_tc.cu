@@ -25,6 +25,7 @@
 #include <algorithm>
 #include <cmath>
 #include <cstring>
+#include <mutex>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -723,19 +724,32 @@ size_t tc_smem() {
   return 1024 + 2 * TILE64 + 4 * NQ * 128 + STAGES * np * TILE64 + 18 * 8 + 16 + PAGE_CACHE * 4 + 8 * NQ * 4;
 }
 
+// The dynamic shared memory limit is an attribute of the device that is current when it
+// is set: raised once per device (and kernel variant), the return code checked.
+constexpr int ATT_MAX_DEVICES = 64;
+std::mutex g_att_attr_mu;
+bool g_att_attr[2][ATT_MAX_DEVICES];
+
 template <bool SPLIT>
-void tc_attr() {
-  static bool done = false;
-  if (!done) {
-    cudaFuncSetAttribute(attn_tc_kernel<SPLIT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         static_cast<int>(tc_smem<SPLIT>()));
-    done = true;
+cudaError_t tc_attr() {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= ATT_MAX_DEVICES) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lk(g_att_attr_mu);
+  if (!g_att_attr[SPLIT ? 1 : 0][dev]) {
+    e = cudaFuncSetAttribute(attn_tc_kernel<SPLIT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(tc_smem<SPLIT>()));
+    if (e != cudaSuccess) return e;
+    g_att_attr[SPLIT ? 1 : 0][dev] = true;
   }
+  return cudaSuccess;
 }
 
 template <bool SPLIT>
 cudaError_t launch_tc(const AttnParams& p, cudaStream_t s) {
-  tc_attr<SPLIT>();
+  cudaError_t ae = tc_attr<SPLIT>();
+  if (ae != cudaSuccess) return ae;
   TcArgs args;
   memset(&args, 0, sizeof(args));
   args.p = p;
@@ -766,7 +780,7 @@ cudaError_t launch_tc(const AttnParams& p, cudaStream_t s) {
 
 template <bool SPLIT>
 int tc_splits(int BH, int want) {
-  tc_attr<SPLIT>();
+  if (tc_attr<SPLIT>() != cudaSuccess) return 1;
   int S = std::max(1, std::min(8, want));
   for (; S > 1; --S) {
     cudaLaunchAttribute at[1];
