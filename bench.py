@@ -287,6 +287,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--layers", type=int, default=None,
                     help="profiling only: the 7B shapes with fewer base layers (not the benchmark workload)")
+    ap.add_argument("--trigram-cache", type=int, default=0,
+                    help="entries of the device trigram cache (0: off)")
     ap.add_argument("--fused-chain", action="store_true",
                     help="run the linears between two attentions as persistent chain launches (fused_chain = 1)")
     ap.add_argument("--op", choices=["linear", "attention"], default=None,
@@ -321,6 +323,8 @@ def main():
         cfg["n_layers"] = args.layers
     if args.fused_chain:
         cfg["fused_chain"] = 1
+    if args.trigram_cache:
+        cfg["trigram_cache"] = args.trigram_cache
     B, N = cfg["batch"], cfg["tree_nodes"]
     prompt = synth.make_prompts(cfg)[0]
     w = synth.make_weights(cfg, device="cuda")
@@ -396,6 +400,13 @@ def main():
         out = ctx.step()
         emitted += sum(len(o) for o in out)
     t_e2e = max_over_ranks((time.perf_counter() - t0) / args.steps, world)
+    hit_rate = None
+    if args.trigram_cache:  # sub-steps whose trigram hit the cache, over a few more steps
+        hits = []
+        for _ in range(5):
+            ctx.step()
+            hits.append(float(ctx.read("trigram_hits").mean()))
+        hit_rate = sum(hits) / len(hits)
     d2h = B * 4 + 4 + int(round(4 * emitted / args.steps))
     n_mid = (n0 + n1) // 2
     ctx.close()
@@ -469,6 +480,9 @@ def main():
     if args.layers:
         line["config"]["workload"] += f" [profiling run: {args.layers} base layers, not the benchmark workload]"
     line["config"]["launch"] = "persistent chains" if args.fused_chain else "one launch per linear and row kernel"
+    line["config"]["trigram_cache"] = args.trigram_cache
+    if hit_rate is not None:
+        line["breakdown"]["trigram_hit_rate"] = hit_rate
     if rank == 0:
         print(json.dumps(line))
     if world > 1:
