@@ -96,7 +96,7 @@ __device__ __forceinline__ void red16(const ChainGemm& g, int M, int m0, int f0,
     const int c = idx >> 3, k = (idx & 7) * 4;
     if (m0 + c < M && f0 + k < g.N) {
       const float* s = sw + c * 33 + k;
-      atomicAdd(reinterpret_cast<float4*>(g.Y + static_cast<size_t>(m0 + c) * g.ldy + f0 + k),
+      red_add_v4(g.Y + static_cast<size_t>(m0 + c) * g.ldy + f0 + k,
                 make_float4(s[0], s[1], s[2], s[3]));
     }
   }

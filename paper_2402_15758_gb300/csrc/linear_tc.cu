@@ -69,7 +69,7 @@ __device__ __forceinline__ void epi_store16(const TcLinearParams& p, int m0, int
     float* y = static_cast<float*>(p.Y);
 #pragma unroll
     for (int j = 0; j < 16; ++j)
-      if (m0 + j < p.M) atomicAdd(y + static_cast<size_t>(m0 + j) * p.ldy + f, v[j]);  // red.global.add
+      if (m0 + j < p.M) red_add_f32(y + static_cast<size_t>(m0 + j) * p.ldy + f, v[j]);
     return;
   }
 #pragma unroll
@@ -99,8 +99,7 @@ __device__ __forceinline__ void epi_red16(const TcLinearParams& p, int m0, int f
     const int c = idx >> 3, k = (idx & 7) * 4;  // token c, features f0 + k .. f0 + k + 3
     if (m0 + c < p.M && f0 + k < p.N) {
       const float* s = sw + c * 33 + k;
-      atomicAdd(reinterpret_cast<float4*>(y + static_cast<size_t>(m0 + c) * p.ldy + f0 + k),
-                make_float4(s[0], s[1], s[2], s[3]));
+      red_add_v4(y + static_cast<size_t>(m0 + c) * p.ldy + f0 + k, make_float4(s[0], s[1], s[2], s[3]));
     }
   }
   __syncwarp();
