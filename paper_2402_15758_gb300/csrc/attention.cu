@@ -116,10 +116,7 @@ __device__ void combine_splits(const AttnParams& p, const float* wsb, int nq, in
       if (it >= items) continue;
       const int qi = it / c4n, c = (it % c4n) * 4;
       const size_t o = static_cast<size_t>(b * p.q_rows + qi) * p.ldo + h * hd + c;
-      store_act(out, out_lo, o, acc[j].x);
-      store_act(out, out_lo, o + 1, acc[j].y);
-      store_act(out, out_lo, o + 2, acc[j].z);
-      store_act(out, out_lo, o + 3, acc[j].w);
+      store_act4(out, out_lo, o, acc[j]);
     }
   }
 }

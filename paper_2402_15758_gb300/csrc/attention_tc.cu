@@ -711,10 +711,7 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
       }
     }
     const size_t o_idx = static_cast<size_t>(b * p.q_rows + q0 + rl) * p.ldo + h * HD + c;
-    store_act(out, out_lo, o_idx, acc.x);
-    store_act(out, out_lo, o_idx + 1, acc.y);
-    store_act(out, out_lo, o_idx + 2, acc.z);
-    store_act(out, out_lo, o_idx + 3, acc.w);
+    store_act4(out, out_lo, o_idx, acc);
   }
 }
 

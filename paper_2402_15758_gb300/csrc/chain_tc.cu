@@ -111,12 +111,7 @@ __device__ __forceinline__ float4 gain4(const bf16* g, int i) {
   return make_float4(__bfloat162float(h[0]), __bfloat162float(h[1]), __bfloat162float(h[2]), __bfloat162float(h[3]));
 }
 
-__device__ __forceinline__ void store_split4(bf16* hi, bf16* lo, size_t i, float4 v) {
-  store_act(hi, lo, i, v.x);
-  store_act(hi, lo, i + 1, v.y);
-  store_act(hi, lo, i + 2, v.z);
-  store_act(hi, lo, i + 3, v.w);
-}
+__device__ __forceinline__ void store_split4(bf16* hi, bf16* lo, size_t i, float4 v) { store_act4(hi, lo, i, v); }
 
 __global__ void __launch_bounds__(THREADS, 1) chain_kernel(const __grid_constant__ ChainParams p) {
   extern __shared__ uint8_t smem_raw[];

@@ -80,6 +80,18 @@ __device__ __forceinline__ void store4_split<bf16>(bf16* hi, bf16* lo, float4 v)
   *reinterpret_cast<uint2*>(lo) = w;
 }
 
+// Four consecutive activations (i a multiple of 4) as vector stores: fp32, bf16, or the
+// bf16 two-term split when `lo` is given.
+__device__ __forceinline__ void store_act4(float* hi, float* /*lo*/, size_t i, float4 v) {
+  *reinterpret_cast<float4*>(hi + i) = v;
+}
+__device__ __forceinline__ void store_act4(bf16* hi, bf16* lo, size_t i, float4 v) {
+  if (lo)
+    store4_split<bf16>(hi + i, lo + i, v);
+  else
+    store4<bf16>(hi + i, v);
+}
+
 // Rotate-half RoPE of four pairs (x1[i], x2[i]) = (x[j+i], x[j+i+hd/2]) with
 // c = cos, s = sin of their angles: the first and the second half of the result.
 __device__ __forceinline__ float4 rot_lo(float4 x1, float4 x2, float4 c, float4 s) {

@@ -1,5 +1,6 @@
 // Row-wise kernels of the step: RMSNorm, RoPE + paged KV write, SwiGLU, embedding
 // gather, argmax and top-k over the vocabulary.
+#include <algorithm>
 #include <cmath>
 
 #include "common.cuh"
@@ -34,14 +35,6 @@ __device__ float block_sum(float v, float* red) {
 // Side job: zero row r of Z (the fp32 output that the next linear accumulates into).
 constexpr int NORM_THREADS = 256;
 constexpr int NORM_VEC = 8;  // float4 per thread: d <= 8192
-
-template <typename T>
-__device__ __forceinline__ void store_act4(T* hi, T* lo, size_t i, float4 v) {
-  store_act(hi, lo, i, v.x);
-  store_act(hi, lo, i + 1, v.y);
-  store_act(hi, lo, i + 2, v.z);
-  store_act(hi, lo, i + 3, v.w);
-}
 
 template <typename T>
 __device__ __forceinline__ float4 load_g4(const T* g, int i);
@@ -178,18 +171,39 @@ __global__ void rope_kv_kernel(const RopeKvParams p) {
 }
 
 // SwiGLU: h = SiLU(gate) * up, gate in columns [0, F), up in [F, 2F).
+// One wave of CTAs (at most two per SM, next to a resident linear CTA); each thread
+// takes SWIGLU_IT float4 of the rows, all loads issued before any store.
+constexpr int SWIGLU_THREADS = 256;
+constexpr int SWIGLU_IT = 4;
 template <typename T>
-__global__ void swiglu_kernel(const float* gu, int ldgu, int F, T* h,
-                              T* h_lo, int ldh) {
+__global__ void __launch_bounds__(SWIGLU_THREADS) swiglu_kernel(const float* gu, int ldgu, int F, T* h,
+                                                                T* h_lo, int ldh, int rows) {
   pdl_trigger();  // the next kernel may start its prologue
   pdl_wait();     // inputs of this kernel are complete
-  const float* g = gu + static_cast<size_t>(blockIdx.y) * ldgu;
-  const size_t row = static_cast<size_t>(blockIdx.y) * ldh;
-  const int f = (blockIdx.x * blockDim.x + threadIdx.x) * 4;
-  if (f >= F) return;
-  const float4 a = *reinterpret_cast<const float4*>(g + f);
-  const float4 u = *reinterpret_cast<const float4*>(g + F + f);
-  store_act4(h, h_lo, row + f, make_float4(silu_f(a.x) * u.x, silu_f(a.y) * u.y, silu_f(a.z) * u.z, silu_f(a.w) * u.w));
+  const int per_row = F / 4;
+  const long long total = static_cast<long long>(rows) * per_row;
+  const long long stride = static_cast<long long>(gridDim.x) * SWIGLU_THREADS * SWIGLU_IT;
+  for (long long base = static_cast<long long>(blockIdx.x) * SWIGLU_THREADS * SWIGLU_IT + threadIdx.x; base < total;
+       base += stride) {
+    float4 a[SWIGLU_IT], u[SWIGLU_IT];
+#pragma unroll
+    for (int k = 0; k < SWIGLU_IT; ++k) {
+      const long long it = base + static_cast<long long>(k) * SWIGLU_THREADS;
+      if (it < total) {
+        const float* g = gu + (it / per_row) * ldgu + (it % per_row) * 4;
+        a[k] = *reinterpret_cast<const float4*>(g);
+        u[k] = *reinterpret_cast<const float4*>(g + F);
+      }
+    }
+#pragma unroll
+    for (int k = 0; k < SWIGLU_IT; ++k) {
+      const long long it = base + static_cast<long long>(k) * SWIGLU_THREADS;
+      if (it < total)
+        store_act4(h, h_lo, static_cast<size_t>((it / per_row) * ldh + (it % per_row) * 4),
+                   make_float4(silu_f(a[k].x) * u[k].x, silu_f(a[k].y) * u[k].y, silu_f(a[k].z) * u[k].z,
+                               silu_f(a[k].w) * u[k].w));
+    }
+  }
 }
 
 template <typename T>
@@ -507,12 +521,16 @@ cudaError_t rope_kv(const RopeKvParams& p, int dtype, cudaStream_t s) {
 cudaError_t swiglu(int dtype, const float* gu, int ldgu, int F, void* h, void* h_lo, int ldh, int rows,
                    cudaStream_t s) {
   if (rows <= 0) return cudaSuccess;
-  if ((F & 3) || (ldh & 3)) return cudaErrorInvalidValue;
-  dim3 grid((F / 4 + 255) / 256, rows);
+  if ((F & 3) || (ldh & 3) || (ldgu & 3)) return cudaErrorInvalidValue;
+  const long long items = static_cast<long long>(rows) * (F / 4);
+  const long long want = (items + SWIGLU_THREADS * SWIGLU_IT - 1) / (SWIGLU_THREADS * SWIGLU_IT);
+  const int grid = static_cast<int>(std::max(1ll, std::min(want, 2ll * tc_num_sms())));
   if (dtype == 0)
-    launch_pdl(swiglu_kernel<float>, dim3(grid), dim3(256), 0, s, gu, ldgu, F, static_cast<float*>(h), nullptr, ldh);
+    launch_pdl(swiglu_kernel<float>, dim3(grid), dim3(SWIGLU_THREADS), 0, s, gu, ldgu, F, static_cast<float*>(h),
+               nullptr, ldh, rows);
   else
-    launch_pdl(swiglu_kernel<bf16>, dim3(grid), dim3(256), 0, s, gu, ldgu, F, static_cast<bf16*>(h), static_cast<bf16*>(h_lo), ldh);
+    launch_pdl(swiglu_kernel<bf16>, dim3(grid), dim3(SWIGLU_THREADS), 0, s, gu, ldgu, F, static_cast<bf16*>(h),
+               static_cast<bf16*>(h_lo), ldh, rows);
   return cudaGetLastError();
 }
 

@@ -53,10 +53,7 @@ __global__ void hfull_store_kernel(const float* dres, int d, T* headin,
   for (int c = threadIdx.x * 4; c < d; c += blockDim.x * 4) {
     const float4 v = *reinterpret_cast<const float4*>(dres + static_cast<size_t>(b) * d + c);
     const size_t o = static_cast<size_t>(b) * 2 * d + d + c;
-    store_act(headin, headin_lo, o, v.x);
-    store_act(headin, headin_lo, o + 1, v.y);
-    store_act(headin, headin_lo, o + 2, v.z);
-    store_act(headin, headin_lo, o + 3, v.w);
+    store_act4(headin, headin_lo, o, v);
     *reinterpret_cast<float4*>(hlog + static_cast<size_t>(b) * d + c) = v;
   }
 }
