@@ -133,6 +133,12 @@ __device__ __forceinline__ void split_pair(float a, float b, uint32_t& hi, uint3
   lo = pack_bf16x2(a - hf.x, b - hf.y);
 }
 
+// Two-term bf16 split of four values: hi (4 x bf16) and lo = the rounding residual.
+__device__ __forceinline__ void split4(float4 v, uint2& hi, uint2& lo) {
+  split_pair(v.x, v.y, hi.x, lo.x);
+  split_pair(v.z, v.w, hi.y, lo.y);
+}
+
 // Under the M = 64 data-path layout, query rows 16q .. 16q + 15 sit in TMEM lanes 0..15 of
 // sub-partition q (warp w reaches sub-partition w % 4).
 
@@ -193,14 +199,25 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
 
   if (!p.prewait_kv) pdl_wait();
   const int nctx = p.n_ctx[b];
-  const int ntiles = (nctx + p.n_local + KT - 1) / KT;
-  const int tps = (ntiles + S - 1) / S;
-  const int t0 = min(ntiles, s * tps);
-  const int t1 = min(ntiles, t0 + tps);
-  const int nt = t1 - t0;
-  const bool cached = nt * 4 <= PAGE_CACHE;
+  // Local mode (fused projections, local rows starting at row 0: verify, prefill, plain
+  // decoding, the draft's first sub-step): every local row is written by this launch,
+  // so the local rows form one extra tile that the CTA owning it builds in shared
+  // memory from the projections (no round trip through the pool); the committed rows
+  // are tiles of the pool.  The local tile is the last of the split's virtual tiles
+  // (so it goes to the CTA with the fewest committed tiles) and that CTA's first tile
+  // (stage 0, free at start).  Otherwise the tiles cover slots [0, nctx + n_local).
+  const bool lmode = p.qkv != nullptr && p.q_local0 == 0;
+  const int ntiles = lmode ? (nctx + KT - 1) / KT : (nctx + p.n_local + KT - 1) / KT;  // tiles of the pool
+  const int T = ntiles + (lmode ? 1 : 0);
+  const int tps = (T + S - 1) / S;
+  const int v0 = min(T, s * tps), v1 = min(T, v0 + tps);
+  const int hl = (lmode && v0 < v1 && v1 == T) ? 1 : 0;  // this CTA holds the local tile (index 0)
+  const int t0 = v0;                                    // pool tiles [t0, t1), tile indices hl ..
+  const int t1 = hl ? T - 1 : v1;
+  const int nt = hl + (t1 - t0);
+  const bool cached = (t1 - t0) * 4 <= PAGE_CACHE;
   if (cached) {
-    const int np = min(nt * 4, p.max_pages - t0 * 4);
+    const int np = min((t1 - t0) * 4, p.max_pages - t0 * 4);
     for (int i = threadIdx.x; i < np; i += blockDim.x) s_pages[i] = p.page_table[b * p.max_pages + t0 * 4 + i];
   }
   tc_fence_before();
@@ -247,12 +264,14 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
     if (warp == SOFT_WARPS) {
       if (lane == 0) prefetch_tensormap(&args.kv_map);
       __syncwarp();
-      while (pre < nt && pre < STAGES && (t0 + pre + 1) * KT <= nctx) {
-        issue_half(t0 + pre, pre, nctx, false);
-        issue_half(t0 + pre, pre, nctx, true);
+      // pool tiles whose rows are all committed (local mode: rows at or past nctx are
+      // masked; the pool holds finite values there, the pools being cleared at set-up)
+      while (hl + pre < nt && hl + pre < STAGES && (lmode || (t0 + pre + 1) * KT <= nctx)) {
+        issue_half(t0 + pre, (hl + pre) & 1, nctx, false);
+        issue_half(t0 + pre, (hl + pre) & 1, nctx, true);
         ++pre;
       }
-      for (; pf < nt && pf < STAGES + L2_AHEAD && (t0 + pf + 1) * KT <= nctx; ++pf)
+      for (; pf < t1 - t0 && pf < STAGES + L2_AHEAD && (lmode || (t0 + pf + 1) * KT <= nctx); ++pf)
         if (pf >= pre) prefetch_tile(t0 + pf, nctx);
     }
     pdl_wait();
@@ -312,8 +331,73 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
   }
   // the P tiles' rows are all rewritten every tile; nothing else to clear
 
-  // ---- fresh local rows of this CTA's key range: rotate k, write k and v to the pool ----
-  if (p.qkv) {
+  // ---- local mode: the owner of the local tile rotates k, writes k and v of the fresh
+  // rows to the pool (for later steps) and into its stage-0 K and V tiles; rows past the
+  // fresh ones are zero there ----
+  if (hl) {
+    for (int it = threadIdx.x; it < KT * 16; it += blockDim.x) {
+      const int i = it >> 4, j = (it & 15) * 4;  // local row, pair index j .. j + 3 of the first half
+      uint2 kh0 = make_uint2(0u, 0u), kl0 = kh0, kh1 = kh0, kl1 = kh0, vh0 = kh0, vl0 = kh0, vh1 = kh0, vl1 = kh0;
+      if (i < nq) {
+        const int slot = nctx + i;
+        const int pos = nctx + p.pos_base + (p.pos_off ? p.pos_off[i] : i);
+        if (pos < 0 || pos >= p.max_pos || (slot >> 4) >= p.max_pages) {
+          if (p.err) atomicOr(p.err, ERR_CAPACITY);
+        } else {
+          const float* src = p.qkv + static_cast<size_t>(b * p.q_rows + i) * p.ldqkv + h * HD + j;
+          const float4 k1 = *reinterpret_cast<const float4*>(src + dm);
+          const float4 k2 = *reinterpret_cast<const float4*>(src + dm + HD / 2);
+          const float4 v1 = *reinterpret_cast<const float4*>(src + 2 * dm);
+          const float4 v2 = *reinterpret_cast<const float4*>(src + 2 * dm + HD / 2);
+          const float2* tab = p.rope + static_cast<size_t>(pos) * (HD / 2) + j;
+          const float4 cs01 = *reinterpret_cast<const float4*>(tab);
+          const float4 cs23 = *reinterpret_cast<const float4*>(tab + 2);
+          const float4 c = make_float4(cs01.x, cs01.z, cs23.x, cs23.z);
+          const float4 sn = make_float4(cs01.y, cs01.w, cs23.y, cs23.w);
+          split4(rot_lo(k1, k2, c, sn), kh0, kl0);
+          split4(rot_hi(k1, k2, c, sn), kh1, kl1);
+          split4(v1, vh0, vl0);
+          split4(v2, vh1, vl1);
+          const int page = p.page_table[b * p.max_pages + (slot >> 4)];
+          bf16* base = pool + (static_cast<size_t>(page) * p.H + h) * NP * 16 * HD + (slot & 15) * HD + j;
+          constexpr size_t plane = 16 * HD;
+          if (SPLIT) {
+            *reinterpret_cast<uint2*>(base) = kh0;
+            *reinterpret_cast<uint2*>(base + plane) = kl0;
+            *reinterpret_cast<uint2*>(base + HD / 2) = kh1;
+            *reinterpret_cast<uint2*>(base + plane + HD / 2) = kl1;
+            *reinterpret_cast<uint2*>(base + 2 * plane) = vh0;
+            *reinterpret_cast<uint2*>(base + 3 * plane) = vl0;
+            *reinterpret_cast<uint2*>(base + 2 * plane + HD / 2) = vh1;
+            *reinterpret_cast<uint2*>(base + 3 * plane + HD / 2) = vl1;
+          } else {
+            *reinterpret_cast<uint2*>(base) = kh0;
+            *reinterpret_cast<uint2*>(base + HD / 2) = kh1;
+            *reinterpret_cast<uint2*>(base + plane) = vh0;
+            *reinterpret_cast<uint2*>(base + plane + HD / 2) = vh1;
+          }
+        }
+      }
+      // stage 0: row i, dims j .. j + 3 (atom 0) and 64 + j .. (atom 1): half of chunk j / 8
+      const uint32_t o0 = swz(i, j >> 3) + ((j & 7) << 1);
+      const uint32_t o1 = ATOM_ROWS64 + o0;
+      uint8_t* kt = kbuf;
+      uint8_t* vt = vbuf;
+      *reinterpret_cast<uint2*>(kt + o0) = kh0;
+      *reinterpret_cast<uint2*>(kt + o1) = kh1;
+      *reinterpret_cast<uint2*>(vt + o0) = vh0;
+      *reinterpret_cast<uint2*>(vt + o1) = vh1;
+      if (SPLIT) {
+        *reinterpret_cast<uint2*>(kt + TILE64 + o0) = kl0;
+        *reinterpret_cast<uint2*>(kt + TILE64 + o1) = kl1;
+        *reinterpret_cast<uint2*>(vt + TILE64 + o0) = vl0;
+        *reinterpret_cast<uint2*>(vt + TILE64 + o1) = vl1;
+      }
+    }
+  }
+  // ---- otherwise: fresh local rows of this CTA's key range: rotate k, write k and v to
+  // the pool, read back by TMA ----
+  if (p.qkv && !lmode) {
     const int fresh0 = nctx + p.q_local0;
     const int f0 = max(0, t0 * KT - fresh0), f1 = min(nq, t1 * KT - fresh0);
     for (int it = threadIdx.x; it < (f1 - f0) * 16; it += blockDim.x) {
@@ -352,9 +436,13 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
     }
     fence_async_global();  // the rows are read back by TMA (async proxy)
   }
-  fence_async_smem();  // the Q tiles are read by the tensor cores (async proxy)
+  fence_async_smem();  // the Q tiles (and the local K, V tile) are read by the tensor cores (async proxy)
   __threadfence_block();
   __syncthreads();
+  if (hl && threadIdx.x == 0) {  // the local tile is in place: stage 0 of K and V is full
+    mbar_arrive(&k_full[0]);
+    mbar_arrive(&v_full[0]);
+  }
 
   if (warp == SOFT_WARPS) {
     // ---------------- KV loader (the whole warp; lane 0 polls and decides) ----------------
@@ -362,22 +450,24 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
     __syncwarp();
     // K of tile j needs the QK product of tile j - 2 done, V of tile j the PV product
     // of tile j - 2; both are polled so that neither waits behind the other
-    int nk = pre, nv = pre;
+    // tile index i: the local tile (i = 0 when hl) or pool tile t0 + i - hl, stage i & 1
+    const int kend = lmode ? nctx : total;
+    int nk = hl + pre, nv = hl + pre;
     uint64_t last_progress = global_timer_ns();
     while (nk < nt || nv < nt) {
       bool moved = false;
       const int kgo = __shfl_sync(0xffffffffu, (lane == 0 && nk < nt &&
                                                 (nk < STAGES || mbar_test(&k_empty[nk & 1], ((nk - STAGES) >> 1) & 1))) ? 1 : 0, 0);
       if (kgo) {
-        issue_half(t0 + nk, nk & 1, total, false);
-        for (pf = max(pf, nk + 1); pf < nt && pf <= nk + L2_AHEAD; ++pf) prefetch_tile(t0 + pf, total);
+        issue_half(t0 + nk - hl, nk & 1, kend, false);
+        for (pf = max(pf, nk - hl + 1); pf < t1 - t0 && pf <= nk - hl + L2_AHEAD; ++pf) prefetch_tile(t0 + pf, kend);
         ++nk;
         moved = true;
       }
       const int vgo = __shfl_sync(0xffffffffu, (lane == 0 && nv < nk &&
                                                 (nv < STAGES || mbar_test(&v_empty[nv & 1], ((nv - STAGES) >> 1) & 1))) ? 1 : 0, 0);
       if (vgo) {
-        issue_half(t0 + nv, nv & 1, total, true);
+        issue_half(t0 + nv - hl, nv & 1, kend, true);
         ++nv;
         moved = true;
       }
@@ -493,8 +583,10 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
     const uint32_t tlane = static_cast<uint32_t>(quad * 32) << 16;
     float m_used = -INFINITY, l = 0.f;
     bool dead = false;
-    for (int t = t0; t < t1; ++t) {
-      const int i = t - t0, sb = i & 1;
+    for (int i = 0; i < nt; ++i) {
+      const int sb = i & 1;
+      const bool loc = hl && i == 0;
+      const int t = t0 + i - hl;
       bool ok = !dead && mbar_wait(&s_full[sb], (i >> 1) & 1, abort);
       dead = !__all_sync(0xffffffffu, ok);
       tc_fence_after();
@@ -509,15 +601,23 @@ __global__ void __launch_bounds__(THREADS, 1) attn_tc_kernel(const __grid_consta
       tc_fence_before();
       __syncwarp();
       if (lane == 0 && !dead) mbar_arrive(&s_free[sb]);
-      // visibility of this lane's 16 keys (bit j: key 64t + kofs + j)
+      // visibility of this lane's 16 keys (bit j: key kofs + j of the tile): the local
+      // tile's keys are local rows (ancestor mask), a pool tile's keys are slots 64 t ..
       uint32_t vbits = 0u;
       if (live) {
-        const int base = t * KT;
-        const int nc = nctx - base, nv = total - base, off = base - nctx;
-        const unsigned long long cm = nc >= 64 ? ~0ull : (nc <= 0 ? 0ull : ((1ull << nc) - 1ull));
-        const unsigned long long lm = off >= 0 ? (off < 64 ? (anc >> off) : 0ull) : (-off < 64 ? (anc << -off) : 0ull);
-        const unsigned long long vm = nv >= 64 ? ~0ull : (nv <= 0 ? 0ull : ((1ull << nv) - 1ull));
-        vbits = static_cast<uint32_t>(((cm | lm) & vm) >> kofs) & 0xFFFFu;
+        unsigned long long vis;
+        if (loc) {
+          vis = anc & (nloc >= 64 ? ~0ull : ((1ull << nloc) - 1ull));
+        } else {
+          const int base = t * KT;
+          const int nc = nctx - base, nv = total - base, off = base - nctx;
+          const unsigned long long cm = nc >= 64 ? ~0ull : (nc <= 0 ? 0ull : ((1ull << nc) - 1ull));
+          const unsigned long long lm =
+              lmode ? 0ull : (off >= 0 ? (off < 64 ? (anc >> off) : 0ull) : (-off < 64 ? (anc << -off) : 0ull));
+          const unsigned long long vm = nv >= 64 ? ~0ull : (nv <= 0 ? 0ull : ((1ull << nv) - 1ull));
+          vis = (cm | lm) & vm;
+        }
+        vbits = static_cast<uint32_t>(vis >> kofs) & 0xFFFFu;
       }
       float ta = -INFINITY, tb = -INFINITY;  // two chains of maxima
 #pragma unroll
