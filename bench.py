@@ -79,30 +79,42 @@ def job_rate(units_per_rank: float, world: int, ms_job: float) -> float:
 
 
 def step_bytes(cfg, n_ctx):
-    """Algorithmic HBM bytes of one step at committed length n_ctx (batch 1).
+    """Algorithmic HBM bytes of one step at committed lengths n_ctx (an int for batch 1,
+    else one length per sequence).
 
     Every weight matrix counts once per use (the trigram encoder and the draft block
-    once per draft sub-step, the heads once), embeddings only for the gathered rows, KV
-    as the rows read at the model's element size (bf16: 2 bytes per K or V value); the
-    activations are excluded.  `kv_planes_extra` is what the stored hi + lo planes of
-    precision mode 1 read on top (the same again): traffic, not algorithmic bytes."""
+    once per draft sub-step, the heads once; a batch shares every weight read), embeddings
+    only for the gathered rows, KV as the rows read at the model's element size (bf16: 2
+    bytes per K or V value); the activations are excluded.  `kv_planes_extra` is what the
+    stored hi + lo planes of precision mode 1 read on top (the same again): traffic, not
+    algorithmic bytes."""
     d, F, V, L, K, N = (cfg["d_model"], cfg["ffn_dim"], cfg["vocab"], cfg["n_layers"],
                         cfg["n_draft_heads"], cfg["tree_nodes"])
+    ns = [n_ctx] if isinstance(n_ctx, (int, float)) else list(n_ctx)
+    B = len(ns)
     e = 2 if cfg["dtype"] == "bf16" else 4
     layer = (3 * d * d + d * d + 3 * d * F) * e
     kv_row = 2 * d * e
-    verify_w = L * layer + V * d * e + N * d * e
-    verify_kv = L * (n_ctx + N) * kv_row
-    draft_w = K * ((3 * d * d + d * d) * e + layer) + K * V * 2 * d * e + K * 3 * d * e
-    draft_kv = sum((n_ctx + k + 1) * kv_row for k in range(K))
-    commit = 2 * d * d * e + 2 * L * 4 * kv_row
+    verify_w = L * layer + V * d * e + B * N * d * e
+    verify_kv = L * sum(n + N for n in ns) * kv_row
+    draft_w = K * ((3 * d * d + d * d) * e + layer) + K * V * 2 * d * e + B * K * 3 * d * e
+    draft_kv = sum((n + k + 1) * kv_row for n in ns for k in range(K))
+    commit = 2 * d * d * e + B * 2 * L * 4 * kv_row
     return dict(verify=verify_w + verify_kv, verify_weights=verify_w, verify_kv=verify_kv,
                 draft=draft_w + draft_kv, commit=commit, total=verify_w + verify_kv + draft_w + draft_kv + commit,
                 kv_planes_extra=verify_kv + draft_kv)
 
 
+WORKLOAD_NAMES = {
+    "7b": "7B-shaped bs1 draft-and-verify step (N=64, topk 5,5,5,5, 512-token prompt)",
+    "13b": "13B-shaped bs1 draft-and-verify step (N=64, topk 5,5,5,5, 2048-token prompt)",
+    "7b_16k": "7B-shaped bs1 draft-and-verify step at a 16384-token context (N=64, paged KV block 16)",
+    "7b_b8": "7B-shaped batch-8 ragged draft-and-verify step (N=32 per sequence, prompts 256..4096)",
+}
+
+
 def workload_config(cfg, prompt_len):
-    return {"workload": "7B-shaped bs1 draft-and-verify step (N=64, topk 5,5,5,5, 512-token prompt)",
+    return {"workload": WORKLOAD_NAMES[cfg["name"]],
             "batch": cfg["batch"], "tree_nodes": cfg["tree_nodes"], "prompt_len": prompt_len,
             "layers": cfg["n_layers"], "d_model": cfg["d_model"], "ffn_dim": cfg["ffn_dim"], "vocab": cfg["vocab"],
             "draft_heads": cfg["n_draft_heads"], "topk": cfg["topk"]}
@@ -298,6 +310,9 @@ def main():
                     help="entries of the device trigram cache (0: off)")
     ap.add_argument("--fused-chain", action="store_true",
                     help="run the linears between two attentions as persistent chain launches (fused_chain = 1)")
+    ap.add_argument("--workload", default=WORKLOAD, choices=sorted(WORKLOAD_NAMES),
+                    help="the configuration stepped (default: the benchmark's, 7B bs1); the others are "
+                         "measured the same way, without the CPU baseline")
     ap.add_argument("--op", choices=["linear", "attention"], default=None,
                     help="time one kernel entry point instead of the step")
     ap.add_argument("--shape", default="64,22016,4096", help="--op linear: M,N,K")
@@ -325,7 +340,7 @@ def main():
     pkg_build.build()
     pkg.load()
 
-    cfg = synth.get_config(WORKLOAD)
+    cfg = synth.get_config(args.workload)
     if args.layers:
         cfg["n_layers"] = args.layers
     if args.fused_chain:
@@ -333,18 +348,20 @@ def main():
     if args.trigram_cache:
         cfg["trigram_cache"] = args.trigram_cache
     B, N = cfg["batch"], cfg["tree_nodes"]
-    prompt = synth.make_prompts(cfg)[0]
+    prompts = synth.make_prompts(cfg)
+    prompt = prompts[0]
     w = synth.make_weights(cfg, device="cuda")
     torch.cuda.synchronize()
     reps = max(3, min(args.steps, 20))
     total_steps = args.warmup + 3 * args.steps + reps + 8
-    max_seq = ((len(prompt) + total_steps * 5 + N + 64 + 15) // 16) * 16
+    max_seq = ((max(len(p) for p in prompts) + total_steps * 5 + N + 64 + 15) // 16) * 16
     stream = torch.cuda.Stream()
     ctx = pkg.Chimera(cfg, w, max_batch=B, max_seq_len=max_seq, stream=stream)
-    ctx.prefill([prompt])
+    ctx.prefill(prompts)
     ctx.step_async(args.warmup)
     ctx.sync()
-    n0 = int(ctx.read("n")[0])
+    n0s = [int(v) for v in ctx.read("n")[:B]]
+    n0 = n0s[0]
 
     # ---- device-resident timing: K graph replays back to back ----
     clocks = Clocks(local)
@@ -361,8 +378,9 @@ def main():
     torch.cuda.synchronize()
     ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, world)
     clk = clocks.stop()
-    n1 = int(ctx.read("n")[0])
-    mean_accept = (n1 - n0) / args.steps
+    n1s = [int(v) for v in ctx.read("n")[:B]]
+    n1 = n1s[0]
+    mean_accept = sum(b - a for a, b in zip(n0s, n1s)) / (B * args.steps)
 
     # ---- per-step distribution: one event pair around each graph replay ----
     ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
@@ -415,7 +433,7 @@ def main():
             hits.append(float(ctx.read("trigram_hits").mean()))
         hit_rate = sum(hits) / len(hits)
     d2h = B * 4 + 4 + int(round(4 * emitted / args.steps))
-    n_mid = (n0 + n1) // 2
+    n_mid = [(a + b) // 2 for a, b in zip(n0s, n1s)]
     ctx.close()
 
     hbm, peak_kind = peaks()
@@ -426,7 +444,7 @@ def main():
     lin_gbs = lin_bytes_per_launch / (lin_per_launch_ms * 1e-3) / 1e9
     ratio, src_hash = linear_traffic_ratio(dom)
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and args.workload == WORKLOAD:
         w_cpu = {k: v.cpu() for k, v in w.items()}
         del w
         torch.cuda.empty_cache()
@@ -437,15 +455,16 @@ def main():
                           f"({len(prompt)}-token prompt, prefill {setup:.1f} s untimed): {times[0]:.2f} s"),
                "host": ht}
     line = {
-        "metric": "tree tokens/s at 7B bs1 (draft-and-verify step)",
+        "metric": ("tree tokens/s at 7B bs1 (draft-and-verify step)" if args.workload == WORKLOAD
+                   else f"tree tokens/s ({args.workload} draft-and-verify step)"),
         "value": value, "unit": "tree tokens/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic: random-init N(0,0.02) weights, uniform-random prompt ids",
-        "config": dict(workload_config(cfg, len(prompt)),
-                       n_ctx=[n0, n1], parallelism="replicas" if world > 1 else "single",
+        "config": dict(workload_config(cfg, [len(p) for p in prompts] if B > 1 else len(prompt)),
+                       n_ctx=[n0s, n1s] if B > 1 else [n0, n1], parallelism="replicas" if world > 1 else "single",
                        precision="bf16 weights; split hi+lo bf16 GEMM operands, fp32 accumulation, "
                                  "KV cache as hi+lo bf16 planes",
-                       l2="inputs larger than L2: 17.8 GB of weights streamed per step"),
+                       l2=f"inputs larger than L2: {nb['total'] / 1e9:.1f} GB of weights and KV read per step"),
         "breakdown": {
             "verify_ms": verify_med, "verify_ms_p90": verify_p90, "draft_ms": draft_med, "commit_ms": commit_med,
             "phase_timing": "CUDA events at the phase boundaries of a graph replay of the step, one step at a time",

@@ -380,10 +380,22 @@ bool make_lin(chimera_ctx* ctx, Lin* l, int M, int N, int K, const void* X, cons
 // KV splits per (sequence, head): enough CTAs to cover the SMs for single-query
 // attention (the draft), and about three 64-key tiles per split for tree queries so
 // the per-split partials stay few (their merge is latency-bound).
+#ifndef CHIMERA_ATT_TILES_PER_CTA
+#define CHIMERA_ATT_TILES_PER_CTA 32
+#endif
 int att_splits(const chimera_ctx* ctx, int B, int nq, int n_keys) {
   if (attn_fuses_rope(ctx->dtype, ctx->hd)) {
-    // tensor-core tree attention: one cluster of S CTAs per (b, h), all resident at once
-    const int want = std::max(1, std::min(ctx->num_sms / (B * ctx->H), (n_keys + 63) / 64));
+    // tensor-core tree attention: one cluster of S CTAs per (b, h).  While the B * H
+    // clusters fit on the SMs at once, as many splits as keep them all resident; with
+    // more (sequence, head) pairs than SMs the launch runs in waves whatever S is, so
+    // long contexts are cut into splits of at most ~CHIMERA_ATT_TILES_PER_CTA 64-key
+    // tiles (a CTA that held a whole long context would set the last wave's length;
+    // measured on the 7B batch-8 step: 64 tiles 14.97, 32 tiles 13.66, 16 tiles 14.81,
+    // 8 tiles 18.89 ms per step, the CTAs' fixed prologue and merge taking over)
+    const int tiles = (n_keys + 63) / 64;
+    if (B * ctx->H >= ctx->num_sms)
+      return std::max(1, std::min(8, (tiles + CHIMERA_ATT_TILES_PER_CTA - 1) / CHIMERA_ATT_TILES_PER_CTA));
+    const int want = std::max(1, std::min(ctx->num_sms / (B * ctx->H), tiles));
     return attn_pick_splits(ctx->dtype, ctx->hd, ctx->kv_planes, B, ctx->H, want);
   }
   const int target = 2 * ctx->num_sms;
