@@ -17,26 +17,28 @@ __global__ void trigram_gather_kernel(const T* E, int d, int V, const int* n_arr
                                       int KMAX, int k, T* out, int* err, float* zero) {
   pdl_trigger();  // the next kernel may start its prologue
   pdl_wait();     // inputs of this kernel are complete
-  const int b = blockIdx.x;
-  const int n = n_arr[b];
-  for (int c = threadIdx.x * 4; c < d; c += blockDim.x * 4)
-    *reinterpret_cast<float4*>(zero + static_cast<size_t>(b) * d + c) = make_float4(0.f, 0.f, 0.f, 0.f);
-  for (int t = 0; t < 3; ++t) {
-    const int i = n - 2 + k + t;
-    int id = -1;
-    if (i >= 0) id = i <= n ? tok[static_cast<size_t>(b) * tok_stride + i]
-                            : topk[(b * K + (i - n - 1)) * KMAX];
-    if (id >= V) {
-      if (threadIdx.x == 0) atomicOr(err, ERR_BAD_INDEX);
-      id = 0;
-    }
-    T* o = out + static_cast<size_t>(b) * 3 * d + t * d;
-    const T* e = E + static_cast<size_t>(id < 0 ? 0 : id) * d;
-    // 16-byte chunks (d * sizeof(T) is a multiple of 16)
-    constexpr int PER = 16 / sizeof(T);
-    for (int c = threadIdx.x * PER; c < d; c += blockDim.x * PER)
-      *reinterpret_cast<uint4*>(o + c) = id < 0 ? make_uint4(0, 0, 0, 0) : *reinterpret_cast<const uint4*>(e + c);
+  // blockIdx.y = t < 3: block t of the trigram; t = 3: the residual row (the CTAs run
+  // side by side, so the three dependent gathers overlap)
+  const int b = blockIdx.x, t = blockIdx.y;
+  if (t == 3) {
+    for (int c = threadIdx.x * 4; c < d; c += blockDim.x * 4)
+      *reinterpret_cast<float4*>(zero + static_cast<size_t>(b) * d + c) = make_float4(0.f, 0.f, 0.f, 0.f);
+    return;
   }
+  const int n = n_arr[b];
+  const int i = n - 2 + k + t;
+  int id = -1;
+  if (i >= 0) id = i <= n ? tok[static_cast<size_t>(b) * tok_stride + i] : topk[(b * K + (i - n - 1)) * KMAX];
+  if (id >= V) {
+    if (threadIdx.x == 0) atomicOr(err, ERR_BAD_INDEX);
+    id = 0;
+  }
+  T* o = out + static_cast<size_t>(b) * 3 * d + t * d;
+  const T* e = E + static_cast<size_t>(id < 0 ? 0 : id) * d;
+  // 16-byte chunks (d * sizeof(T) is a multiple of 16)
+  constexpr int PER = 16 / sizeof(T);
+  for (int c = threadIdx.x * PER; c < d; c += blockDim.x * PER)
+    *reinterpret_cast<uint4*>(o + c) = id < 0 ? make_uint4(0, 0, 0, 0) : *reinterpret_cast<const uint4*>(e + c);
 }
 
 // headin[b][d..2d) = h_full (the draft block output), kept per head for debugging;
@@ -362,10 +364,10 @@ cudaError_t launch_trigram_gather(int dtype, const void* E, int d, int V, const 
                                   int tok_stride, const int* topk, int K, int KMAX, int k, void* out,
                                   int B, int* err, float* zero, cudaStream_t s) {
   if (dtype == 0)
-    launch_pdl(trigram_gather_kernel<float>, dim3(B), dim3(256), 0, s, static_cast<const float*>(E), d, V, n, tok, tok_stride,
+    launch_pdl(trigram_gather_kernel<float>, dim3(B, 4), dim3(256), 0, s, static_cast<const float*>(E), d, V, n, tok, tok_stride,
                                                    topk, K, KMAX, k, static_cast<float*>(out), err, zero);
   else
-    launch_pdl(trigram_gather_kernel<bf16>, dim3(B), dim3(256), 0, s, static_cast<const bf16*>(E), d, V, n, tok, tok_stride,
+    launch_pdl(trigram_gather_kernel<bf16>, dim3(B, 4), dim3(256), 0, s, static_cast<const bf16*>(E), d, V, n, tok, tok_stride,
                                                   topk, K, KMAX, k, static_cast<bf16*>(out), err, zero);
   return cudaGetLastError();
 }
