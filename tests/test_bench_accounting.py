@@ -40,3 +40,20 @@ def test_step_bytes_from_weight_shapes():
 def test_job_rate_and_single_rank_max():
     assert bench.max_over_ranks(3.25, 1) == 3.25
     assert abs(bench.job_rate(64, 4, 2.0) - 4 * 64 / 2e-3) < 1e-6
+
+
+def test_step_bytes_batch_shares_weights_and_sums_kv():
+    # a batch reads every weight once and each sequence's own KV rows; a batch of one
+    # given as a list is the int case
+    cfg = synth.get_config("7b_b8")
+    d, L, N, K = cfg["d_model"], cfg["n_layers"], cfg["tree_nodes"], cfg["n_draft_heads"]
+    ns = [2943, 3503, 2192, 1807, 3696, 649, 3521, 1451]
+    b = bench.step_bytes(cfg, ns)
+    one = bench.step_bytes(cfg, ns[0])
+    assert bench.step_bytes(cfg, [ns[0]]) == one
+    kv_row = 2 * d * 2
+    assert b["verify_kv"] == L * sum(n + N for n in ns) * kv_row
+    # weights: the single-sequence count minus its gathered rows, plus the batch's rows
+    assert b["verify_weights"] == one["verify_weights"] + (len(ns) - 1) * N * d * 2
+    assert b["draft"] - sum((n + k + 1) * kv_row for n in ns for k in range(K)) == \
+        one["draft"] - sum((ns[0] + k + 1) * kv_row for k in range(K)) + (len(ns) - 1) * K * 3 * d * 2
