@@ -483,6 +483,9 @@ def main():
             "attention_class_ms": att["ms"], "attention_launches": att["launches"],
             "kernel_ms_by_kind_eager": {k: round(v, 4) for k, v in sorted(kind_ms.items(), key=lambda t: -t[1])},
             "mean_accepted_tokens_per_step": mean_accept,
+            "committed_tokens_per_s": B * mean_accept / (ms * 1e-3),
+            "accept_note": "random-init draft heads: the draft rarely matches, so a step commits ~1 token "
+                           "per sequence (the root); reported, not optimised",
         },
         "roofline": {"bound": "hbm",
                      "kernel": ("chain_kernel (persistent tcgen05 chain: the linears and row steps between two "
