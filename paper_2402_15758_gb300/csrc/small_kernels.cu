@@ -171,38 +171,38 @@ __global__ void rope_kv_kernel(const RopeKvParams p) {
 }
 
 // SwiGLU: h = SiLU(gate) * up, gate in columns [0, F), up in [F, 2F).
-// One wave of CTAs (at most two per SM, next to a resident linear CTA); each thread
-// takes SWIGLU_IT float4 of the rows, all loads issued before any store.
+// A whole number of waves of CTAs (the tree verify: two per SM, next to a resident linear
+// CTA), each taking an equal contiguous share of the float4 items: every SM gets the
+// same work, so no SM holds up the next kernel.  A thread takes at most SWIGLU_IT
+// items of its CTA's share, all loads issued before any store.
 constexpr int SWIGLU_THREADS = 256;
 constexpr int SWIGLU_IT = 4;
 template <typename T>
 __global__ void __launch_bounds__(SWIGLU_THREADS) swiglu_kernel(const float* gu, int ldgu, int F, T* h,
-                                                                T* h_lo, int ldh, int rows) {
+                                                                T* h_lo, int ldh, int rows, int per_cta) {
   pdl_trigger();  // the next kernel may start its prologue
   pdl_wait();     // inputs of this kernel are complete
   const int per_row = F / 4;
   const long long total = static_cast<long long>(rows) * per_row;
-  const long long stride = static_cast<long long>(gridDim.x) * SWIGLU_THREADS * SWIGLU_IT;
-  for (long long base = static_cast<long long>(blockIdx.x) * SWIGLU_THREADS * SWIGLU_IT + threadIdx.x; base < total;
-       base += stride) {
-    float4 a[SWIGLU_IT], u[SWIGLU_IT];
+  const long long c0 = static_cast<long long>(blockIdx.x) * per_cta;
+  const long long c1 = min(total, c0 + per_cta);
+  float4 a[SWIGLU_IT], u[SWIGLU_IT];
 #pragma unroll
-    for (int k = 0; k < SWIGLU_IT; ++k) {
-      const long long it = base + static_cast<long long>(k) * SWIGLU_THREADS;
-      if (it < total) {
-        const float* g = gu + (it / per_row) * ldgu + (it % per_row) * 4;
-        a[k] = *reinterpret_cast<const float4*>(g);
-        u[k] = *reinterpret_cast<const float4*>(g + F);
-      }
+  for (int k = 0; k < SWIGLU_IT; ++k) {
+    const long long it = c0 + threadIdx.x + static_cast<long long>(k) * SWIGLU_THREADS;
+    if (it < c1) {
+      const float* g = gu + (it / per_row) * ldgu + (it % per_row) * 4;
+      a[k] = *reinterpret_cast<const float4*>(g);
+      u[k] = *reinterpret_cast<const float4*>(g + F);
     }
+  }
 #pragma unroll
-    for (int k = 0; k < SWIGLU_IT; ++k) {
-      const long long it = base + static_cast<long long>(k) * SWIGLU_THREADS;
-      if (it < total)
-        store_act4(h, h_lo, static_cast<size_t>((it / per_row) * ldh + (it % per_row) * 4),
-                   make_float4(silu_f(a[k].x) * u[k].x, silu_f(a[k].y) * u[k].y, silu_f(a[k].z) * u[k].z,
-                               silu_f(a[k].w) * u[k].w));
-    }
+  for (int k = 0; k < SWIGLU_IT; ++k) {
+    const long long it = c0 + threadIdx.x + static_cast<long long>(k) * SWIGLU_THREADS;
+    if (it < c1)
+      store_act4(h, h_lo, static_cast<size_t>((it / per_row) * ldh + (it % per_row) * 4),
+                 make_float4(silu_f(a[k].x) * u[k].x, silu_f(a[k].y) * u[k].y, silu_f(a[k].z) * u[k].z,
+                             silu_f(a[k].w) * u[k].w));
   }
 }
 
@@ -523,14 +523,17 @@ cudaError_t swiglu(int dtype, const float* gu, int ldgu, int F, void* h, void* h
   if (rows <= 0) return cudaSuccess;
   if ((F & 3) || (ldh & 3) || (ldgu & 3)) return cudaErrorInvalidValue;
   const long long items = static_cast<long long>(rows) * (F / 4);
-  const long long want = (items + SWIGLU_THREADS * SWIGLU_IT - 1) / (SWIGLU_THREADS * SWIGLU_IT);
-  const int grid = static_cast<int>(std::max(1ll, std::min(want, 2ll * tc_num_sms())));
+  const long long cap = SWIGLU_THREADS * SWIGLU_IT;  // items one CTA can take
+  const int sms = tc_num_sms();
+  long long grid = (items + cap - 1) / cap;
+  if (grid > sms) grid = ((grid + sms - 1) / sms) * sms;  // whole waves of equal shares
+  const int per_cta = static_cast<int>((items + grid - 1) / grid);  // <= cap
   if (dtype == 0)
-    launch_pdl(swiglu_kernel<float>, dim3(grid), dim3(SWIGLU_THREADS), 0, s, gu, ldgu, F, static_cast<float*>(h),
-               nullptr, ldh, rows);
+    launch_pdl(swiglu_kernel<float>, dim3(static_cast<unsigned>(grid)), dim3(SWIGLU_THREADS), 0, s, gu, ldgu, F,
+               static_cast<float*>(h), nullptr, ldh, rows, per_cta);
   else
-    launch_pdl(swiglu_kernel<bf16>, dim3(grid), dim3(SWIGLU_THREADS), 0, s, gu, ldgu, F, static_cast<bf16*>(h),
-               static_cast<bf16*>(h_lo), ldh, rows);
+    launch_pdl(swiglu_kernel<bf16>, dim3(static_cast<unsigned>(grid)), dim3(SWIGLU_THREADS), 0, s, gu, ldgu, F,
+               static_cast<bf16*>(h), static_cast<bf16*>(h_lo), ldh, rows, per_cta);
   return cudaGetLastError();
 }
 
