@@ -619,16 +619,19 @@ cudaError_t enqueue_step(chimera_ctx* ctx) {
     }
     if (k > 0 && one_pass) {  // every head scores h_full_{n+1}: only the head k launch below
       LAUNCH(CHIMERA_KIND_OTHER, 0, launch_hfull_store(ctx->dtype, ctx->dres, d, ctx->headin, ctx->headin_lo,
-                                 ctx->hfull_log + static_cast<size_t>(k) * B * d, ctx->hlog + static_cast<size_t>(k) * B * V,
-                                 V, B, s));
+                                 ctx->hfull_log + static_cast<size_t>(k) * B * d, nullptr, V, B, s));
       RUN(run_lin(ctx, ctx->dhead[k]));
       LAUNCH(CHIMERA_KIND_TOPK, 0, topk_rows(ctx->hlog + static_cast<size_t>(k) * B * V, V, B, ctx->KMAX,
                                              ctx->d_topk + k * ctx->KMAX, ctx->d_topk_val + k * ctx->KMAX, K * ctx->KMAX,
                                              ctx->topk_ws_v, ctx->topk_ws_i, ctx->topk_cnt, s));
       continue;
     }
+    // sub-step 0 also clears every head's score rows, which the head linears accumulate
+    // into (off the chain of the later sub-steps)
+    const bool sep_heads = !ctx->use_chain;
     LAUNCH(CHIMERA_KIND_EMBED, 0, launch_trigram_gather(ctx->dtype, ctx->embed, d, V, ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_topk, K,
-                                ctx->KMAX, k, ctx->tbuf, B, ctx->d_err, ctx->dres, s));
+                                ctx->KMAX, k, ctx->tbuf, B, ctx->d_err, ctx->dres, s,
+                                (sep_heads && k == 0) ? ctx->hlog : nullptr, static_cast<long long>(K) * B * V));
     if (ctx->tc_entries)
       LAUNCH(CHIMERA_KIND_OTHER, 0, launch_trigram_lookup(ctx->d_n, ctx->d_tok, ctx->tok_stride, ctx->d_topk, K, ctx->KMAX, k,
                                                           B, d, ctx->tc_nsets, ctx->tc_keys, ctx->tc_stamp, ctx->tc_vals,
@@ -667,8 +670,7 @@ cudaError_t enqueue_step(chimera_ctx* ctx) {
     LAUNCH(CHIMERA_KIND_SWIGLU, 0, swiglu(ctx->dtype, ctx->gu, 2 * ctx->F, ctx->F, ctx->hf, ctx->hf_lo, ctx->F, B, s));
     RUN(run_lin(ctx, ctx->ddown));
     LAUNCH(CHIMERA_KIND_OTHER, 0, launch_hfull_store(ctx->dtype, ctx->dres, d, ctx->headin, ctx->headin_lo,
-                             ctx->hfull_log + static_cast<size_t>(k) * B * d, ctx->hlog + static_cast<size_t>(k) * B * V,
-                             V, B, s));
+                             ctx->hfull_log + static_cast<size_t>(k) * B * d, nullptr, V, B, s));
     RUN(run_lin(ctx, ctx->dhead[k]));
     LAUNCH(CHIMERA_KIND_TOPK, 0, topk_rows(ctx->hlog + static_cast<size_t>(k) * B * V, V, B, ctx->KMAX, ctx->d_topk + k * ctx->KMAX,
                     ctx->d_topk_val + k * ctx->KMAX, K * ctx->KMAX, ctx->topk_ws_v, ctx->topk_ws_i,

@@ -14,12 +14,20 @@ namespace {
 template <typename T>
 __global__ void trigram_gather_kernel(const T* E, int d, int V, const int* n_arr,
                                       const int* tok, int tok_stride, const int* topk, int K,
-                                      int KMAX, int k, T* out, int* err, float* zero) {
+                                      int KMAX, int k, T* out, int* err, float* zero, float* zero2,
+                                      long long zero2_floats) {
   pdl_trigger();  // the next kernel may start its prologue
   pdl_wait();     // inputs of this kernel are complete
-  // blockIdx.y = t < 3: block t of the trigram; t = 3: the residual row (the CTAs run
-  // side by side, so the three dependent gathers overlap)
+  // blockIdx.y = t < 3: block t of the trigram; t = 3: the residual row; t > 3: a share
+  // of zero2 (the CTAs run side by side, so the three dependent gathers overlap)
   const int b = blockIdx.x, t = blockIdx.y;
+  if (t > 3) {
+    const long long n4 = zero2_floats / 4, nz = static_cast<long long>(gridDim.x) * (gridDim.y - 4);
+    const long long per = (n4 + nz - 1) / nz, z0 = (static_cast<long long>(t - 4) * gridDim.x + b) * per;
+    float4* z = reinterpret_cast<float4*>(zero2);
+    for (long long i = z0 + threadIdx.x; i < min(n4, z0 + per); i += blockDim.x) z[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    return;
+  }
   if (t == 3) {
     for (int c = threadIdx.x * 4; c < d; c += blockDim.x * 4)
       *reinterpret_cast<float4*>(zero + static_cast<size_t>(b) * d + c) = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -42,7 +50,8 @@ __global__ void trigram_gather_kernel(const T* E, int d, int V, const int* n_arr
 }
 
 // headin[b][d..2d) = h_full (the draft block output), kept per head for debugging;
-// also zeroes row b of the head's score buffer (V floats) that its linear accumulates into.
+// with `zero`, also zeroes row b of the head's score buffer (V floats) that its linear
+// accumulates into.
 template <typename T>
 __global__ void hfull_store_kernel(const float* dres, int d, T* headin,
                                    T* headin_lo, float* hlog,
@@ -50,8 +59,9 @@ __global__ void hfull_store_kernel(const float* dres, int d, T* headin,
   pdl_trigger();  // the next kernel may start its prologue
   pdl_wait();     // inputs of this kernel are complete
   const int b = blockIdx.x;
-  for (int c = threadIdx.x * 4; c < V; c += blockDim.x * 4)
-    *reinterpret_cast<float4*>(zero + static_cast<size_t>(b) * V + c) = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (zero)
+    for (int c = threadIdx.x * 4; c < V; c += blockDim.x * 4)
+      *reinterpret_cast<float4*>(zero + static_cast<size_t>(b) * V + c) = make_float4(0.f, 0.f, 0.f, 0.f);
   for (int c = threadIdx.x * 4; c < d; c += blockDim.x * 4) {
     const float4 v = *reinterpret_cast<const float4*>(dres + static_cast<size_t>(b) * d + c);
     const size_t o = static_cast<size_t>(b) * 2 * d + d + c;
@@ -362,13 +372,15 @@ __global__ void accept_typical_kernel(const int* n_arr, int* tok, int tok_stride
 
 cudaError_t launch_trigram_gather(int dtype, const void* E, int d, int V, const int* n, const int* tok,
                                   int tok_stride, const int* topk, int K, int KMAX, int k, void* out,
-                                  int B, int* err, float* zero, cudaStream_t s) {
+                                  int B, int* err, float* zero, cudaStream_t s, float* zero2, long long zero2_floats) {
+  if (zero2 && ((zero2_floats & 3) || (reinterpret_cast<uintptr_t>(zero2) & 15))) return cudaErrorInvalidValue;
+  const int zy = zero2 ? 16 : 0;  // CTAs per sequence that clear zero2
   if (dtype == 0)
-    launch_pdl(trigram_gather_kernel<float>, dim3(B, 4), dim3(256), 0, s, static_cast<const float*>(E), d, V, n, tok, tok_stride,
-                                                   topk, K, KMAX, k, static_cast<float*>(out), err, zero);
+    launch_pdl(trigram_gather_kernel<float>, dim3(B, 4 + zy), dim3(256), 0, s, static_cast<const float*>(E), d, V, n, tok,
+               tok_stride, topk, K, KMAX, k, static_cast<float*>(out), err, zero, zero2, zero2_floats);
   else
-    launch_pdl(trigram_gather_kernel<bf16>, dim3(B, 4), dim3(256), 0, s, static_cast<const bf16*>(E), d, V, n, tok, tok_stride,
-                                                  topk, K, KMAX, k, static_cast<bf16*>(out), err, zero);
+    launch_pdl(trigram_gather_kernel<bf16>, dim3(B, 4 + zy), dim3(256), 0, s, static_cast<const bf16*>(E), d, V, n, tok,
+               tok_stride, topk, K, KMAX, k, static_cast<bf16*>(out), err, zero, zero2, zero2_floats);
   return cudaGetLastError();
 }
 

@@ -7,7 +7,8 @@ namespace chimera {
 
 cudaError_t launch_trigram_gather(int dtype, const void* E, int d, int V, const int* n, const int* tok,
                                   int tok_stride, const int* topk, int K, int KMAX, int k, void* out,
-                                  int B, int* err, float* zero, cudaStream_t s);
+                                  int B, int* err, float* zero, cudaStream_t s, float* zero2 = nullptr,
+                                  long long zero2_floats = 0);
 cudaError_t launch_hfull_store(int dtype, const float* dres, int d, void* headin, void* headin_lo, float* hlog,
                                float* zero, int V, int B, cudaStream_t s);
 cudaError_t launch_tree_expand(const int* n, const int* tok, int tok_stride, const int* topk, int K, int KMAX,
