@@ -183,6 +183,14 @@ const char* chimera_last_error(const chimera_ctx* ctx);
 chimera_status chimera_tree(const chimera_ctx* ctx, int32_t* depth, int32_t* parent,
                             int32_t* rank, uint64_t* anc);
 
+/* The same static tree from the configuration alone, on the host, with no context and
+ * no GPU: topk host int32 [n_heads], each 1..8 (ranks past the five of Table 4 have no
+ * marginal and never enter the tree), 1 <= n_heads <= 4, 2 <= n_nodes <= 64.  Outputs
+ * as chimera_tree, host arrays of n_nodes; any may be NULL.  CHIMERA_EINVAL for an
+ * argument out of range or when n_nodes - 1 exceeds the rank tuples the limits allow. */
+chimera_status chimera_static_tree(const int32_t* topk, int n_heads, int n_nodes, int32_t* depth,
+                                   int32_t* parent, int32_t* rank, uint64_t* anc);
+
 /* Per-kernel timing of one step, launched eagerly with CUDA events around every
  * launch (test and benchmark hook).  kinds: host int32 [max] kernel class (see
  * CHIMERA_KIND_*), ms: host float [max], bytes: host double [max] algorithmic HBM

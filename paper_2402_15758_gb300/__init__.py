@@ -68,6 +68,7 @@ _SIGS = {
     "chimera_free": (None, [ctypes.c_void_p]),
     "chimera_last_error": (ctypes.c_char_p, [ctypes.c_void_p]),
     "chimera_tree": (ctypes.c_int, [ctypes.c_void_p] + [ctypes.c_void_p] * 4),
+    "chimera_static_tree": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int, ctypes.c_int] + [ctypes.c_void_p] * 4),
     "chimera_profile_step": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int] + [ctypes.c_void_p] * 5),
     "chimera_profile_phases": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int] + [ctypes.c_void_p] * 3),
     "chimera_profile_kind": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int, ctypes.c_int] + [ctypes.c_void_p] * 3),
@@ -310,6 +311,21 @@ class Chimera:
 
 
 # ---- kernel-level entry points ----
+def static_tree(topk, n_nodes: int) -> dict:
+    """The static tree the library builds for these head limits and node count (host
+    only, needs no GPU): depth, parent, rank and ancestor masks per node."""
+    lib = load()
+    tk = np.asarray(topk, np.int32)
+    d = np.zeros(n_nodes, np.int32)
+    p, r = np.zeros_like(d), np.zeros_like(d)
+    a = np.zeros(n_nodes, np.uint64)
+    st = lib.chimera_static_tree(tk.ctypes.data, len(tk), n_nodes, d.ctypes.data, p.ctypes.data,
+                                 r.ctypes.data, a.ctypes.data)
+    if st != 0:
+        raise ChimeraError(st, "chimera_static_tree: limits or node count out of range")
+    return dict(depth=d.tolist(), parent=p.tolist(), rank=r.tolist(), anc=[int(x) for x in a])
+
+
 def op_linear(X, W, Y, epi: int = 0, out_f32: bool = False, X_lo=None, stream=None):
     """Y (epilogue)= (X + X_lo) W^T through chimera_op_linear (X, X_lo [M][K], W [N][K],
     Y [M][N] device tensors)."""

@@ -1605,6 +1605,26 @@ chimera_status chimera_tree(const chimera_ctx* ctx, int32_t* depth, int32_t* par
   return CHIMERA_OK;
 }
 
+chimera_status chimera_static_tree(const int32_t* topk, int n_heads, int n_nodes, int32_t* depth,
+                                   int32_t* parent, int32_t* rank, uint64_t* anc) {
+  if (!topk || n_heads < 1 || n_heads > 4 || n_nodes < 2 || n_nodes > 64) return CHIMERA_EINVAL;
+  int lim[4];
+  for (int k = 0; k < n_heads; ++k) {
+    if (topk[k] < 1 || topk[k] > MAX_KMAX) return CHIMERA_EINVAL;
+    lim[k] = topk[k];
+  }
+  Tree t;
+  std::string err;
+  if (!build_tree(lim, n_heads, n_nodes, &t, &err)) return CHIMERA_EINVAL;
+  for (int i = 0; i < n_nodes; ++i) {
+    if (depth) depth[i] = t.depth[i];
+    if (parent) parent[i] = t.parent[i];
+    if (rank) rank[i] = t.rank[i];
+    if (anc) anc[i] = t.anc[i];
+  }
+  return CHIMERA_OK;
+}
+
 chimera_status chimera_profile_step(chimera_ctx* ctx, int max, int32_t* kinds, int32_t* phases, float* ms,
                                     double* bytes, int32_t* count) {
   if (!ctx) return CHIMERA_EINVAL;
