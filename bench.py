@@ -32,7 +32,7 @@ sys.path.insert(0, ROOT)
 for _v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
     os.environ.setdefault(_v, str(os.cpu_count() or 1))
 
-import numpy as np  # noqa: E402
+import numpy  # noqa: E402,F401  (its BLAS starts with the thread count set above)
 import torch  # noqa: E402
 
 import synth  # noqa: E402
